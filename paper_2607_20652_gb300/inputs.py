@@ -1,0 +1,89 @@
+"""Seeded synthetic inputs, shared by the oracle tests and the CUDA path.
+
+This module only draws random numbers (numpy PCG64, fixed seeds) and rounds
+them to bf16. It holds none of the DPB arithmetic: planted codes are returned
+as a tree of *choices* (root coordinates, parent slots, generator slots,
+coefficients); each consumer turns the choices into feature indices with its
+own child map and into activations with its own decoder.
+
+The paper's workloads are residual-stream activations of FineWeb-Edu-trained
+models, which are not available here; these distributions stand in for them:
+
+* gaussian_rows: x ~ N(0, 1), optionally with a fraction of rows scaled
+  (outlier tokens), the GPT-2-width workload.
+* planted_tree: a sparse code with the hierarchy's shape (roots at level 0,
+  then children of planted nodes level by level), coefficients +-U[1, 2],
+  the wide workload (x = decoded code + N(0, 0.1^2) noise).
+"""
+from __future__ import annotations
+
+import dataclasses
+
+import numpy as np
+
+
+def rng(seed: int) -> np.random.Generator:
+    return np.random.default_rng(np.random.PCG64(seed))
+
+
+def to_bf16(a: np.ndarray) -> np.ndarray:
+    """Round float32 values to the nearest bf16 (ties to even); returns
+    float32 values that are exactly representable in bf16."""
+    a = np.ascontiguousarray(a, dtype=np.float32)
+    u = a.view(np.uint32).astype(np.uint64)
+    u = (u + 0x7FFF + ((u >> 16) & 1)) & 0xFFFF0000
+    return u.astype(np.uint32).view(np.float32)
+
+
+def bf16_bits(a: np.ndarray) -> np.ndarray:
+    """The upper 16 bits of float32 values already rounded by to_bf16."""
+    return (np.ascontiguousarray(a, dtype=np.float32).view(np.uint32) >> 16).astype(np.uint16)
+
+
+def gaussian_rows(T: int, d: int, seed: int, outlier_frac: float = 0.0,
+                  outlier_scale: float = 10.0) -> np.ndarray:
+    """x[T, d] float32 ~ N(0, 1); a random `outlier_frac` of rows scaled."""
+    g = rng(seed)
+    x = g.standard_normal((T, d), dtype=np.float32)
+    if outlier_frac > 0:
+        n = int(round(outlier_frac * T))
+        rows = g.choice(T, size=n, replace=False)
+        x[rows] *= np.float32(outlier_scale)
+    return x
+
+
+def normal(shape, seed: int, scale: float = 1.0) -> np.ndarray:
+    return (rng(seed).standard_normal(shape, dtype=np.float32) * np.float32(scale))
+
+
+@dataclasses.dataclass
+class PlantedTree:
+    """Random choices of a planted hierarchical code, per token.
+
+    roots[t, r]            level-0 coordinates (distinct, < d)
+    parent[l][t, e]        slot of the parent among level l-1's planted nodes
+    gen[l][t, e]           generator slot j < children[l] used for that child
+    coef[t, e]             coefficients, level by level (roots first)
+    """
+    roots: np.ndarray
+    parent: list
+    gen: list
+    coef: np.ndarray
+
+
+def planted_tree(T: int, d: int, levels: int, children, per_level, seed: int) -> PlantedTree:
+    g = rng(seed)
+    n0 = per_level[0]
+    roots = np.stack([g.choice(d, size=n0, replace=False) for _ in range(T)]).astype(np.int64)
+    parent, gen = [None], [None]
+    for l in range(1, levels):
+        n_prev, n_here = per_level[l - 1], per_level[l]
+        # distinct (parent slot, generator slot) pairs per token
+        pairs = np.stack([g.choice(n_prev * children[l], size=n_here, replace=False)
+                          for _ in range(T)])
+        parent.append(pairs // children[l])
+        gen.append(pairs % children[l])
+    k = int(sum(per_level[:levels]))
+    mag = g.uniform(1.0, 2.0, size=(T, k))
+    sign = np.where(g.random((T, k)) < 0.5, -1.0, 1.0)
+    return PlantedTree(roots=roots, parent=parent, gen=gen, coef=(mag * sign))
