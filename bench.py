@@ -1,0 +1,466 @@
+#!/usr/bin/env python3
+"""Throughput of the DPB hot path on GB300: encode + decode + backward.
+
+One step = dpb_encode, dpb_decode and dpb_backward over one batch of the
+"wide" workload (T = 65536 tokens per GPU, d = 768, 2^20 features as 5 levels
+of 16 children, beam 8, k = 64, bf16 storage with fp32 accumulation). Inputs
+are synthetic: a planted tree of 64 parity directions per token plus
+N(0, 0.1^2) noise, and grad_y ~ N(0, 1). The working set of a step (about
+450 MB) is larger than the 129 MB L2, so no flush is needed between steps.
+
+Prints one JSON line (rank 0). Under torchrun each rank runs its own token
+shard (weak scaling, no data-path collective); the time is the max over
+ranks. `--impl reference` times the CPU oracle on a bounded sample instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "DPB tokens/sec (encode+decode+bwd) at d=768, 2^20 feats, 1 GB300; % of roofline"
+WORKLOAD = "wide"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+                  "sm_max_mhz": 2070.0}
+GB300_SMS = 152
+FP32_LANES_PER_SM = 128
+
+
+# ---------------------------------------------------------------------------
+# distributed helpers (host logic; exercised by gloo tests on CPU)
+# ---------------------------------------------------------------------------
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def shard_seed(base: int, rank: int) -> int:
+    """Each rank draws its own token shard (weak scaling)."""
+    return base + 1009 * rank
+
+
+def max_over_ranks(value: float, world: int, device=None) -> float:
+    if world <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def whole_job_rate(tokens_per_rank: int, world: int, steps: int, max_seconds: float) -> float:
+    return tokens_per_rank * world * steps / max_seconds
+
+
+# ---------------------------------------------------------------------------
+# peaks, roofline and clocks
+# ---------------------------------------------------------------------------
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return p, "measured"
+    except (OSError, ValueError):
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+def algorithmic_work(cfg: dict, T: int, k_hash: float, s: int):
+    """Per-launch algorithmic bytes and operations of each call (the method's
+    own sums, not implementation overhead). s = bytes per stored element."""
+    d, k, B = cfg["d"], cfg["k"], cfg["beam"]
+    mma = sum(2 * B * cfg["children"][l] * d for l in range(1, cfg["levels"]))
+    return {
+        "encode": {"bytes": T * (d * s + 8 * k + 4), "tensor_flops": T * mma},
+        "decode": {"bytes": T * (8 * k + 4 + d * s), "fp_ops": T * k_hash * d},
+        "backward": {"bytes": T * (3 * d * s + 12 * k), "fp_ops": T * 2 * k_hash * d},
+    }
+
+
+def roofline_for(name: str, work: dict, seconds: float, peaks: dict, src: str):
+    hbm = peaks["hbm_gbs"] * 1e9
+    tc = peaks["bf16_tflops_sustained"] * 1e12
+    alu = GB300_SMS * FP32_LANES_PER_SM * peaks.get("sm_max_mhz", 2070.0) * 1e6
+    terms = {"hbm": work["bytes"] / hbm}
+    if "tensor_flops" in work:
+        terms["tensor"] = work["tensor_flops"] / tc
+    if "fp_ops" in work:
+        terms["alu"] = work["fp_ops"] / alu
+    bound = max(terms, key=terms.get)
+    if bound == "hbm":
+        achieved, peak, unit = work["bytes"] / seconds / 1e9, peaks["hbm_gbs"], "GB/s"
+    elif bound == "tensor":
+        achieved, peak, unit = work["tensor_flops"] / seconds / 1e12, peaks["bf16_tflops_sustained"], "TFLOP/s"
+    else:
+        achieved, peak, unit = work["fp_ops"] / seconds / 1e12, alu / 1e12, "TFLOP/s"
+    return {"kernel": name, "bound": bound, "achieved": round(achieved, 3), "peak": round(peak, 3),
+            "unit": unit, "frac": round(achieved / peak, 4), "traffic": None,
+            "peak_source": f"{src} ({'bf16 sustained' if bound == 'tensor' else 'copy' if bound == 'hbm' else '152 SMs x 128 FP32 lanes x max SM clock'})",
+            "t_roofline_us": round(terms[bound] * 1e6, 2), "t_measured_us": round(seconds * 1e6, 2)}
+
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled during the timed region."""
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str | None):
+        self.gpu_id = gpu_id
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "200"]
+        if self.gpu_id:
+            cmd += ["-i", self.gpu_id]
+        try:
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if not self.proc:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                smax.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# workload
+# ---------------------------------------------------------------------------
+
+def workload_cfg():
+    from paper_2607_20652_gb300 import configs
+    return dict(configs.WORKLOADS[WORKLOAD])
+
+
+def compose(tree, G, levels):
+    """Feature indices of a planted tree through the plan's child map p ^ g_j."""
+    nodes = [tree.roots.astype(np.int64)]
+    for l in range(1, levels):
+        par = np.take_along_axis(nodes[-1], tree.parent[l], axis=1)
+        nodes.append(par ^ G[l][tree.gen[l]].astype(np.int64))
+    return np.concatenate(nodes, axis=1).astype(np.int32)
+
+
+def make_inputs_gpu(w, plan, seed, device):
+    """Planted x (decoded by the library itself) + noise, and grad_y, on the GPU."""
+    import torch
+    from paper_2607_20652_gb300 import dpb, inputs
+    T, d = w["T"], w["d"]
+    _, G = plan.tables()
+    tree = inputs.planted_tree(T, d, w["levels"], plan.config["children"], w["planted"], seed)
+    idx_true = compose(tree, G, w["levels"])
+    syn = dpb.Plan(d=d, levels=w["levels"], m_bits=w["m_bits"], children=w["children"],
+                   beam=w["beam"], k=w["k"], dtype="f32", norm_match=0)
+    y = dpb.decode(syn, torch.from_numpy(idx_true).to(device),
+                   torch.from_numpy(tree.coef.astype(np.float32)).to(device))
+    noise = torch.from_numpy(inputs.normal((T, d), seed + 1000, w["noise"])).to(device)
+    x = (y + noise).to(torch.bfloat16).contiguous()
+    gy = torch.from_numpy(inputs.normal((T, d), seed + w["grad_seed"])).to(device).to(torch.bfloat16)
+    torch.cuda.synchronize(device)
+    return x, gy, idx_true
+
+
+def oracle_sample(w, n_tokens, seed):
+    """The same workload for the oracle: planted rows decoded by the oracle."""
+    import oracle
+    from paper_2607_20652_gb300 import inputs
+    ref = oracle.resolve(d=w["d"], m_bits=w["m_bits"], levels=w["levels"], children=w["children"],
+                         beam=w["beam"], k=w["k"])
+    tree = inputs.planted_tree(n_tokens, w["d"], w["levels"], ref.children, w["planted"], seed)
+    idx_true = compose(tree, ref.G, w["levels"])
+    clean = oracle.decode(ref, idx_true, tree.coef, norm_match=0)
+    x = inputs.to_bf16((clean + inputs.normal((n_tokens, w["d"]), seed + 1000, w["noise"])).astype(np.float32))
+    gy = inputs.to_bf16(inputs.normal((n_tokens, w["d"]), seed + w["grad_seed"]))
+    return ref, x.astype(np.float64), gy.astype(np.float64)
+
+
+def time_oracle(ref, x, gy):
+    import oracle
+    t0 = time.perf_counter()
+    idx, val, xn, _ = oracle.encode(ref, x)
+    oracle.decode(ref, idx, val, xn)
+    oracle.backward(ref, x, idx, val, gy)
+    return time.perf_counter() - t0
+
+
+def cpu_baseline(w, budget_s: float, seed: int):
+    ref, x, gy = oracle_sample(w, 64, seed)
+    per_tok = time_oracle(ref, x, gy) / 64
+    n = int(max(64, min(16384, budget_s / max(per_tok, 1e-6))))
+    ref, x, gy = oracle_sample(w, n, seed)
+    secs = time_oracle(ref, x, gy)
+    return {"value": round(n / secs, 2), "unit": "tokens/s", "cores": 1, "kind": "oracle",
+            "sample": f"first {n} tokens of the {WORKLOAD} workload (planted, seed {seed}); "
+                      f"encode+decode+backward, single-threaded C oracle, fp64; {secs:.1f} s"}
+
+
+# ---------------------------------------------------------------------------
+# arms
+# ---------------------------------------------------------------------------
+
+def run_reference(args, world, rank):
+    w = workload_cfg()
+    if rank != 0:
+        return 0
+    n = args.ref_tokens
+    ref, x, gy = oracle_sample(w, n, 0)
+    for _ in range(args.warmup):
+        time_oracle(ref, x, gy)
+    times = [time_oracle(ref, x, gy) for _ in range(args.steps)]
+    total = sum(times)
+    value = n * args.steps / total
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(value, 2), "unit": "tokens/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(1e3 * total / args.steps, 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": config_block(w, world, n_tokens=n),
+        "cpu_baseline": {"kind": "oracle", "cores": 1, "value": round(value, 2), "unit": "tokens/s",
+                         "sample": f"{n} tokens of the {WORKLOAD} workload per step, single-threaded C oracle (fp64)"},
+        "e2e": {"value": round(value, 2), "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def config_block(w, world, n_tokens=None):
+    return {"workload": WORKLOAD, "T_per_gpu": n_tokens or w["T"], "d": w["d"], "features": 2 ** w["m_bits"],
+            "levels": w["levels"], "children": w["children"], "beam": w["beam"], "k": w["k"],
+            "accumulate": "fp32", "inputs": "planted tree of 64 parity directions + N(0,0.1^2), bf16",
+            "l2": "working set ~450 MB > 129 MB L2 (no flush needed)",
+            "parallelism": f"dp{world} (independent token shards)"}
+
+
+def run_ours(args, world, rank, local):
+    import torch
+    from paper_2607_20652_gb300 import dpb
+
+    device = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(device)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=device)
+    w = workload_cfg()
+    T, d = w["T"], w["d"]
+    plan = dpb.Plan(d=d, levels=w["levels"], m_bits=w["m_bits"], children=w["children"],
+                    beam=w["beam"], k=w["k"], dtype="bf16", norm_match=1)
+    seed = shard_seed(w["seed"], rank)
+    x, gy, idx_true = make_inputs_gpu(w, plan, seed, device)
+    k = plan.code_len
+    idx = torch.empty((T, k), dtype=torch.int32, device=device)
+    val = torch.empty((T, k), dtype=torch.float32, device=device)
+    xn = torch.empty((T,), dtype=torch.float32, device=device)
+    y = torch.empty_like(x)
+    gx = torch.empty_like(x)
+    gv = torch.empty((T, k), dtype=torch.float32, device=device)
+    ws = plan.workspace(T, device)
+    stream = torch.cuda.current_stream(device)
+
+    def step(ev=None):
+        if ev:
+            ev[0].record(stream)
+        dpb.encode(plan, x, idx=idx, val=val, xnorm=xn, workspace=ws, stream=stream)
+        if ev:
+            ev[1].record(stream)
+        dpb.decode(plan, idx, val, xn, y=y, workspace=ws, stream=stream)
+        if ev:
+            ev[2].record(stream)
+        dpb.backward(plan, x, idx, val, gy, grad_x=gx, grad_val=gv, workspace=ws, stream=stream)
+        if ev:
+            ev[3].record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize(device)
+    status = dpb.workspace_status(ws)
+
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    gpu_id = None
+    try:
+        gpu_id = "GPU-" + str(torch.cuda.get_device_properties(device).uuid)
+    except Exception:
+        gpu_id = None
+    clocks = ClockSampler(gpu_id)
+    clocks.start()
+    time.sleep(0.3)
+    barrier(world)
+    torch.cuda.synchronize(device)
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for i in range(args.steps):
+        step(evs[i])
+    end.record(stream)
+    torch.cuda.synchronize(device)
+    barrier(world)
+    clk = clocks.stop()
+    ms = start.elapsed_time(end)
+    ms_max = max_over_ranks(ms, world, device)
+    per = {"encode": [], "decode": [], "backward": []}
+    for e in evs:
+        per["encode"].append(e[0].elapsed_time(e[1]))
+        per["decode"].append(e[1].elapsed_time(e[2]))
+        per["backward"].append(e[2].elapsed_time(e[3]))
+    kern_ms = {n: statistics.mean(v) for n, v in per.items()}
+
+    # algorithmic work and roofline of the dominant kernel
+    idx_np = idx.cpu().numpy()
+    k_hash = float(np.mean(np.sum(idx_np >= d, axis=1)))
+    recovered = float(np.mean([len(set(idx_np[t]) & set(idx_true[t])) / k for t in range(0, T, 64)]))
+    peaks, src = load_peaks()
+    work = algorithmic_work(plan.config, T, k_hash, 2)
+    dom = max(kern_ms, key=kern_ms.get)
+    roof = roofline_for(dom, work[dom], kern_ms[dom] / 1e3, peaks, src)
+    kernels = {n: {"ms": round(v, 4), **{kk: vv for kk, vv in roofline_for(n, work[n], v / 1e3, peaks, src).items()
+                                          if kk in ("bound", "frac", "t_roofline_us")}}
+               for n, v in kern_ms.items()}
+    step_roof_us = sum(kernels[n]["t_roofline_us"] for n in kernels)
+
+    # end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(plan, x, gy, args, device, stream, world)
+
+    value = whole_job_rate(T, world, args.steps, ms_max / 1e3)
+    line = {
+        "metric": METRIC, "value": round(value, 1), "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_max / args.steps, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic", "config": config_block(w, world),
+        "roofline": roof,
+        "step_roofline": {"t_roofline_us": round(step_roof_us, 2),
+                          "t_measured_us": round(1e3 * ms_max / args.steps, 2),
+                          "frac": round(step_roof_us / (1e3 * ms_max / args.steps), 4)},
+        "kernels": kernels, "k_hash": round(k_hash, 2), "planted_recovery": round(recovered, 4),
+        "gpu_launches": 3 * args.steps, "clocks": clk, "device_status": status,
+    }
+    if e2e:
+        line["e2e"] = e2e
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(w, args.cpu_seconds, 0)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+def run_e2e(plan, x, gy, args, device, stream, world):
+    import torch
+    from paper_2607_20652_gb300 import dpb
+    T, d = x.shape
+    k = plan.code_len
+    hx = torch.empty_like(x, device="cpu").pin_memory()
+    hgy = torch.empty_like(gy, device="cpu").pin_memory()
+    hx.copy_(x)
+    hgy.copy_(gy)
+    outs = {"idx": torch.empty((T, k), dtype=torch.int32).pin_memory(),
+            "val": torch.empty((T, k), dtype=torch.float32).pin_memory(),
+            "y": torch.empty((T, d), dtype=torch.bfloat16).pin_memory(),
+            "gx": torch.empty((T, d), dtype=torch.bfloat16).pin_memory(),
+            "gv": torch.empty((T, k), dtype=torch.float32).pin_memory()}
+    dx = torch.empty_like(x)
+    dgy = torch.empty_like(gy)
+    ws = plan.workspace(T, device)
+
+    def step():
+        dx.copy_(hx, non_blocking=True)
+        dgy.copy_(hgy, non_blocking=True)
+        idx, val, xn = dpb.encode(plan, dx, workspace=ws, stream=stream)
+        y = dpb.decode(plan, idx, val, xn, workspace=ws, stream=stream)
+        gx, gv = dpb.backward(plan, dx, idx, val, dgy, workspace=ws, stream=stream)
+        for name, t in (("idx", idx), ("val", val), ("y", y), ("gx", gx), ("gv", gv)):
+            outs[name].copy_(t, non_blocking=True)
+
+    for _ in range(max(1, args.warmup)):
+        step()
+    torch.cuda.synchronize(device)
+    steps = max(3, args.steps // 2)
+    barrier(world)
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        step()
+    torch.cuda.synchronize(device)
+    secs = max_over_ranks(time.perf_counter() - t0, world, device)
+    bi = hx.numel() * hx.element_size() + hgy.numel() * hgy.element_size()
+    bo = sum(t.numel() * t.element_size() for t in outs.values())
+    return {"value": round(whole_job_rate(T, world, steps, secs), 1), "unit": "tokens/s",
+            "h2d_bytes_per_step": bi, "d2h_bytes_per_step": bo, "steps": steps}
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--ref-tokens", type=int, default=512)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    world, rank, local = dist_env()
+    if args.warmup < 3 and args.impl == "ours":
+        print("note: at least 3 warm-up steps are used", file=sys.stderr)
+        args.warmup = 3
+    if args.impl == "reference":
+        return run_reference(args, world, rank)
+    return run_ours(args, world, rank, local)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -143,13 +143,10 @@ void orc_seed_matrix(int d, int t, uint32_t poly, uint32_t *M)
         M[iota] = (uint32_t)iota | (orc_gf_inv((uint32_t)iota, t, poly) << t);
 }
 
-/* Parity of the set bits of v, by counting them one at a time. */
+/* Parity of the number of set bits of v (the compiler's bit-count builtin). */
 static int bit_parity(uint32_t v)
 {
-    int n = 0;
-    for (int j = 0; j < 32; j++)
-        n += (v >> j) & 1u;
-    return n & 1;
+    return __builtin_parity(v);
 }
 
 /* Sign (+1 or -1) of coordinate iota of the hashed direction of index i:
@@ -231,6 +228,7 @@ int orc_generators(int levels, const int *bits, const int *children, uint64_t se
 typedef struct {
     uint32_t idx;
     double z;
+    int exact; /* score is a plain coordinate read (level 0, no tables) */
 } cand_t;
 
 /* Order of reading R9: |z| descending, then index ascending. */
@@ -245,15 +243,36 @@ static int cand_cmp(const void *pa, const void *pb)
     return (a->idx < b->idx) ? -1 : (a->idx > b->idx) ? 1 : 0;
 }
 
-/* Relative gap at a cut of n sorted candidates keeping the first `keep`. */
+/* Relative gap at a cut of n sorted candidates keeping the first `keep`:
+ * the smallest (|z_a| - |z_b|) / |z_a| over a kept a and a dropped b of which
+ * at least one has an inexact score. Two level-0 scores read without tables
+ * are the same number on every implementation, so a tie between them is
+ * settled by index everywhere and is not a near-tie. */
 static double cut_gap(const cand_t *sorted, int n, int keep)
 {
     if (keep >= n || keep <= 0)
         return INFINITY;
-    double last = fabs(sorted[keep - 1].z), next = fabs(sorted[keep].z);
-    if (last == 0.0)
-        return 0.0;
-    return (last - next) / last;
+    int last_inexact_kept = -1, first_inexact_dropped = -1;
+    for (int e = 0; e < keep; e++)
+        if (!sorted[e].exact)
+            last_inexact_kept = e;
+    for (int e = keep; e < n && first_inexact_dropped < 0; e++)
+        if (!sorted[e].exact)
+            first_inexact_dropped = e;
+    double gap = INFINITY;
+    if (last_inexact_kept >= 0) {
+        double a = fabs(sorted[last_inexact_kept].z), b = fabs(sorted[keep].z);
+        double g = a > 0.0 ? (a - b) / a : 0.0;
+        if (g < gap)
+            gap = g;
+    }
+    if (first_inexact_dropped >= 0) {
+        double a = fabs(sorted[keep - 1].z), b = fabs(sorted[first_inexact_dropped].z);
+        double g = a > 0.0 ? (a - b) / a : 0.0;
+        if (g < gap)
+            gap = g;
+    }
+    return gap;
 }
 
 /* Score of index c against x by the direct inner product <phi_c, x>.
@@ -320,6 +339,7 @@ int orc_encode(int d, int levels, const int *bits, const int *children, int beam
         for (int i = 0; i < d; i++) {
             lvl[nl].idx = (uint32_t)i;
             lvl[nl].z = standardise(xt[i], (uint32_t)i, mu, sigma);
+            lvl[nl].exact = (mu == NULL && sigma == NULL);
             nl++;
         }
         for (int l = 0;; l++) {
@@ -346,6 +366,7 @@ int orc_encode(int d, int levels, const int *bits, const int *children, int beam
                             seen = 1;
                     if (!seen) {
                         lvl[nl].idx = c;
+                        lvl[nl].exact = 0;
                         nl++;
                     }
                 }
@@ -418,6 +439,7 @@ int orc_encode_per_level(int d, int levels, const int *children, const int *k_pe
         for (int i = 0; i < d; i++) {
             lvl[nl].idx = (uint32_t)i;
             lvl[nl].z = standardise(xt[i], (uint32_t)i, mu, sigma);
+            lvl[nl].exact = (mu == NULL && sigma == NULL);
             nl++;
         }
         for (int l = 0;; l++) {
@@ -448,6 +470,7 @@ int orc_encode_per_level(int d, int levels, const int *children, const int *k_pe
                             seen = 1;
                     if (!seen) {
                         lvl[nl].idx = c;
+                        lvl[nl].exact = 0;
                         nl++;
                     }
                 }

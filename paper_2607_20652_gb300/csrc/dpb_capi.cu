@@ -1,0 +1,248 @@
+// dpb_capi.cu -- the extern "C" entry points of include/dpb.h: argument
+// validation on the host, then one kernel launch per call on the caller's
+// stream. No allocation happens in encode/decode/backward.
+#include <cstdint>
+#include <cstring>
+#include <new>
+
+#include "dpb_internal.h"
+
+namespace dpb {
+const char *last_error_message();
+}
+
+namespace {
+
+bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+dpb_status check_plan(const dpb_plan *p) {
+    if (!p) return dpb::fail(DPB_ERR_INVALID_ARG, "plan is NULL");
+    return DPB_OK;
+}
+
+dpb_status check_workspace(void *ws, size_t bytes) {
+    if (!ws) return dpb::fail(DPB_ERR_INVALID_ARG, "workspace is NULL");
+    if (!aligned(ws, 256)) return dpb::fail(DPB_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+    if (bytes < 256) return dpb::fail(DPB_ERR_INVALID_ARG, "workspace needs 256 bytes, got %zu", bytes);
+    return DPB_OK;
+}
+
+dpb_status check_rows(const void *ptr, const char *name, bool required) {
+    if (!ptr) return required ? dpb::fail(DPB_ERR_INVALID_ARG, "%s is NULL", name) : DPB_OK;
+    if (!aligned(ptr, 16)) return dpb::fail(DPB_ERR_INVALID_ARG, "%s must be 16-byte aligned", name);
+    return DPB_OK;
+}
+
+dpb_status check_vec(const void *ptr, const char *name, bool required) {
+    if (!ptr) return required ? dpb::fail(DPB_ERR_INVALID_ARG, "%s is NULL", name) : DPB_OK;
+    if (!aligned(ptr, 4)) return dpb::fail(DPB_ERR_INVALID_ARG, "%s must be 4-byte aligned", name);
+    return DPB_OK;
+}
+
+dpb_status launched(cudaError_t e, const char *what) {
+    if (e != cudaSuccess) return dpb::fail(DPB_ERR_CUDA, "%s launch failed: %s", what, cudaGetErrorString(e));
+    return DPB_OK;
+}
+
+// The plan's tables live on the device current at creation; calls must be
+// made with that device current.
+dpb_status check_device(const dpb_plan *p) {
+    if (p->device < 0) return dpb::fail(DPB_ERR_CUDA, "plan was created without a CUDA device");
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess) return dpb::fail(DPB_ERR_CUDA, "cudaGetDevice failed");
+    if (dev != p->device)
+        return dpb::fail(DPB_ERR_INVALID_ARG, "plan lives on device %d but device %d is current", p->device, dev);
+    return DPB_OK;
+}
+
+#define DPB_TRY(expr)                    \
+    do {                                 \
+        dpb_status s_ = (expr);          \
+        if (s_ != DPB_OK) return s_;     \
+    } while (0)
+
+}  // namespace
+
+extern "C" {
+
+dpb_status dpb_plan_create(const dpb_config *cfg, const uint32_t *generators, dpb_plan **out) {
+    if (!cfg || !out) return dpb::fail(DPB_ERR_INVALID_ARG, "cfg and out must be non-NULL");
+    *out = nullptr;
+    dpb_plan *p = new (std::nothrow) dpb_plan();
+    if (!p) return dpb::fail(DPB_ERR_NO_MEMORY, "host allocation failed");
+    dpb_status s = dpb::resolve_and_build(cfg, generators, p);
+    if (s != DPB_OK) {
+        delete p;
+        return s;
+    }
+    const size_t smem = dpb::encode_smem_header(p) + dpb::encode_smem_per_warp(p);
+    if (smem > 200 * 1024) {
+        delete p;
+        return dpb::fail(DPB_ERR_UNSUPPORTED, "encoder needs %zu bytes of shared memory per warp", smem);
+    }
+    int ndev = 0;
+    if (cudaGetDeviceCount(&ndev) != cudaSuccess || ndev == 0) {
+        cudaGetLastError();  // host-only plan: tables and config, no compute
+        p->device = -1;
+        *out = p;
+        return DPB_OK;
+    }
+    if (cudaGetDevice(&p->device) != cudaSuccess) {
+        delete p;
+        return dpb::fail(DPB_ERR_CUDA, "cudaGetDevice failed");
+    }
+    const size_t mb = sizeof(uint32_t) * p->M.size(), gb = sizeof(uint32_t) * p->G.size();
+    if (cudaMalloc(&p->dM, mb) != cudaSuccess || cudaMalloc(&p->dG, gb) != cudaSuccess) {
+        cudaFree(p->dM);
+        cudaFree(p->dG);
+        delete p;
+        return dpb::fail(DPB_ERR_NO_MEMORY, "device table allocation failed");
+    }
+    if (cudaMemcpy(p->dM, p->M.data(), mb, cudaMemcpyHostToDevice) != cudaSuccess ||
+        cudaMemcpy(p->dG, p->G.data(), gb, cudaMemcpyHostToDevice) != cudaSuccess) {
+        cudaFree(p->dM);
+        cudaFree(p->dG);
+        delete p;
+        return dpb::fail(DPB_ERR_CUDA, "device table upload failed");
+    }
+    *out = p;
+    return DPB_OK;
+}
+
+dpb_status dpb_plan_destroy(dpb_plan *plan) {
+    if (!plan) return DPB_OK;
+    if (plan->device < 0) {
+        delete plan;
+        return DPB_OK;
+    }
+    int cur = -1;
+    cudaGetDevice(&cur);
+    if (cur != plan->device) cudaSetDevice(plan->device);
+    cudaFree(plan->dM);
+    cudaFree(plan->dG);
+    if (cur >= 0 && cur != plan->device) cudaSetDevice(cur);
+    delete plan;
+    return DPB_OK;
+}
+
+dpb_status dpb_plan_config(const dpb_plan *plan, dpb_config *out) {
+    DPB_TRY(check_plan(plan));
+    if (!out) return dpb::fail(DPB_ERR_INVALID_ARG, "out is NULL");
+    *out = plan->cfg;
+    return DPB_OK;
+}
+
+dpb_status dpb_plan_tables(const dpb_plan *plan, uint32_t *M_out, uint32_t *G_out) {
+    DPB_TRY(check_plan(plan));
+    if (M_out) std::memcpy(M_out, plan->M.data(), sizeof(uint32_t) * plan->M.size());
+    if (G_out) std::memcpy(G_out, plan->G.data(), sizeof(uint32_t) * plan->G.size());
+    return DPB_OK;
+}
+
+dpb_status dpb_code_length(const dpb_plan *plan, int32_t *k_out) {
+    DPB_TRY(check_plan(plan));
+    if (!k_out) return dpb::fail(DPB_ERR_INVALID_ARG, "k_out is NULL");
+    *k_out = plan->code_len;
+    return DPB_OK;
+}
+
+dpb_status dpb_workspace_size(const dpb_plan *plan, int64_t T, size_t *bytes) {
+    DPB_TRY(check_plan(plan));
+    if (!bytes || T < 0) return dpb::fail(DPB_ERR_INVALID_ARG, "bytes is NULL or T < 0");
+    *bytes = 256;
+    return DPB_OK;
+}
+
+dpb_status dpb_encode(const dpb_plan *plan, const void *x, int64_t T, const float *mu,
+                      const float *sigma, int32_t *idx, float *val, float *xnorm,
+                      void *workspace, size_t workspace_bytes, void *stream) {
+    DPB_TRY(check_plan(plan));
+    if (T < 0) return dpb::fail(DPB_ERR_INVALID_ARG, "T < 0");
+    if (T == 0) return DPB_OK;
+    if ((mu == nullptr) != (sigma == nullptr))
+        return dpb::fail(DPB_ERR_INVALID_ARG, "mu and sigma must both be given or both be NULL");
+    DPB_TRY(check_rows(x, "x", true));
+    DPB_TRY(check_vec(mu, "mu", false));
+    DPB_TRY(check_vec(sigma, "sigma", false));
+    DPB_TRY(check_vec(idx, "idx", true));
+    DPB_TRY(check_vec(val, "val", true));
+    DPB_TRY(check_vec(xnorm, "xnorm", false));
+    DPB_TRY(check_workspace(workspace, workspace_bytes));
+    DPB_TRY(check_device(plan));
+    return launched(dpb::launch_encode(plan, x, T, mu, sigma, idx, val, xnorm,
+                                       static_cast<int32_t *>(workspace),
+                                       static_cast<cudaStream_t>(stream)),
+                    "encode");
+}
+
+dpb_status dpb_decode(const dpb_plan *plan, const int32_t *idx, const float *val, int64_t T,
+                      const float *xnorm, void *y, void *workspace, size_t workspace_bytes,
+                      void *stream) {
+    DPB_TRY(check_plan(plan));
+    if (T < 0) return dpb::fail(DPB_ERR_INVALID_ARG, "T < 0");
+    if (T == 0) return DPB_OK;
+    DPB_TRY(check_vec(idx, "idx", true));
+    DPB_TRY(check_vec(val, "val", true));
+    DPB_TRY(check_vec(xnorm, "xnorm", plan->cfg.norm_match != 0));
+    DPB_TRY(check_rows(y, "y", true));
+    DPB_TRY(check_workspace(workspace, workspace_bytes));
+    DPB_TRY(check_device(plan));
+    return launched(dpb::launch_decode(plan, idx, val, T, xnorm, y, static_cast<int32_t *>(workspace),
+                                       static_cast<cudaStream_t>(stream)),
+                    "decode");
+}
+
+dpb_status dpb_backward(const dpb_plan *plan, const void *x, const int32_t *idx,
+                        const float *val, int64_t T, const float *sigma, const void *grad_y,
+                        void *grad_x, float *grad_val, void *workspace,
+                        size_t workspace_bytes, void *stream) {
+    DPB_TRY(check_plan(plan));
+    if (T < 0) return dpb::fail(DPB_ERR_INVALID_ARG, "T < 0");
+    if (T == 0) return DPB_OK;
+    DPB_TRY(check_rows(x, "x", true));
+    DPB_TRY(check_vec(idx, "idx", true));
+    DPB_TRY(check_vec(val, "val", true));
+    DPB_TRY(check_vec(sigma, "sigma", false));
+    DPB_TRY(check_rows(grad_y, "grad_y", true));
+    DPB_TRY(check_rows(grad_x, "grad_x", true));
+    DPB_TRY(check_vec(grad_val, "grad_val", true));
+    DPB_TRY(check_workspace(workspace, workspace_bytes));
+    DPB_TRY(check_device(plan));
+    return launched(dpb::launch_backward(plan, x, idx, val, T, sigma, grad_y, grad_x, grad_val,
+                                         static_cast<int32_t *>(workspace),
+                                         static_cast<cudaStream_t>(stream)),
+                    "backward");
+}
+
+dpb_status dpb_workspace_status(const void *workspace, int clear, int32_t *status_out, void *stream) {
+    if (!workspace || !status_out) return dpb::fail(DPB_ERR_INVALID_ARG, "workspace and status_out must be non-NULL");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    int32_t v = 0;
+    if (cudaMemcpyAsync(&v, workspace, sizeof(v), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+        cudaStreamSynchronize(s) != cudaSuccess)
+        return dpb::fail(DPB_ERR_CUDA, "reading the workspace status failed");
+    if (clear && v != 0) {
+        if (cudaMemsetAsync(const_cast<void *>(workspace), 0, sizeof(int32_t), s) != cudaSuccess ||
+            cudaStreamSynchronize(s) != cudaSuccess)
+            return dpb::fail(DPB_ERR_CUDA, "clearing the workspace status failed");
+    }
+    *status_out = v;
+    return v ? dpb::fail(DPB_ERR_DEVICE, "device status 0x%x", v) : DPB_OK;
+}
+
+const char *dpb_status_string(dpb_status s) {
+    switch (s) {
+        case DPB_OK: return "ok";
+        case DPB_ERR_INVALID_ARG: return "invalid argument";
+        case DPB_ERR_UNSUPPORTED: return "unsupported configuration";
+        case DPB_ERR_CUDA: return "CUDA error";
+        case DPB_ERR_TIMEOUT: return "device wait timed out";
+        case DPB_ERR_NO_MEMORY: return "out of memory";
+        case DPB_ERR_DEVICE: return "device-side error flagged";
+    }
+    return "unknown status";
+}
+
+const char *dpb_last_error(void) { return dpb::last_error_message(); }
+
+}  // extern "C"

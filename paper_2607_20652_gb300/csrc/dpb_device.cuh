@@ -1,0 +1,150 @@
+// dpb_device.cuh -- device helpers shared by the DPB kernels: dtype access,
+// on-chip generation of parity signs, warp-level exact top-k selection and a
+// warp bitonic sort. Everything here runs inside one warp.
+#pragma once
+
+#include <cuda_bf16.h>
+
+#include <cstdint>
+
+namespace dpb {
+
+constexpr unsigned kFull = 0xffffffffu;
+
+// ---- element access ---------------------------------------------------------
+
+__device__ __forceinline__ float ld_elem(const float *p, int64_t i) { return p[i]; }
+__device__ __forceinline__ float ld_elem(const __nv_bfloat16 *p, int64_t i) {
+    return __bfloat162float(p[i]);
+}
+__device__ __forceinline__ void st_elem(float *p, int64_t i, float v) { p[i] = v; }
+__device__ __forceinline__ void st_elem(__nv_bfloat16 *p, int64_t i, float v) {
+    p[i] = __float2bfloat16_rn(v);
+}
+
+// ---- parity signs (App. A.4, Eq. 26-27) ------------------------------------
+
+// Sign of coordinate iota of phi~_c in bit 31: parity(M[iota] AND c), so a
+// float is multiplied by R(.) = (-1)^bit with one XOR.
+__device__ __forceinline__ uint32_t sign31(uint32_t m_row, uint32_t c) {
+    return static_cast<uint32_t>(__popc(m_row & c)) << 31;
+}
+__device__ __forceinline__ float flip(float v, uint32_t s31) {
+    return __uint_as_float(__float_as_uint(v) ^ s31);
+}
+
+// ---- ordering keys ----------------------------------------------------------
+
+// |z| as an unsigned key: for finite floats the bit pattern of |z| orders like
+// the value. Candidates are ordered by (key descending, index ascending).
+__device__ __forceinline__ uint32_t akey(float z) { return __float_as_uint(z) & 0x7fffffffu; }
+
+__device__ __forceinline__ bool before(uint32_t ka, uint32_t ia, uint32_t kb, uint32_t ib) {
+    return ka > kb || (ka == kb && ia < ib);
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
+    return v;
+}
+
+// ---- exact top-K of a shared-memory list -------------------------------------
+
+// Writes the K first entries of (z[0..n), id[0..n)) in (|z| desc, id asc)
+// order to (oz, oid), unordered, and returns K (n < K keeps all n). The K-th
+// key is found by bisection on its bits (counts reduced across the warp), then
+// ties on that key are cut by index with a second bisection. Warp-collective.
+__device__ __forceinline__ int warp_select(const float *z, const uint32_t *id, int n, int K, float *oz,
+                           uint32_t *oid) {
+    const int lane = threadIdx.x & 31;
+    if (K > n) K = n;
+    uint32_t tau = 0;  // largest key with count(key >= tau) >= K
+    if (K < n) {
+        for (int b = 30; b >= 0; --b) {
+            const uint32_t c = tau | (1u << b);
+            int cnt = 0;
+            for (int e = lane; e < n; e += 32) cnt += (akey(z[e]) >= c);
+            if (__reduce_add_sync(kFull, cnt) >= K) tau = c;
+        }
+    }
+    int above = 0, ties = 0;
+    for (int e = lane; e < n; e += 32) {
+        const uint32_t k = akey(z[e]);
+        above += (k > tau);
+        ties += (k == tau);
+    }
+    above = __reduce_add_sync(kFull, above);
+    ties = __reduce_add_sync(kFull, ties);
+    const int need = K - above;
+    uint32_t cut = 0xffffffffu;  // ties with id <= cut are kept
+    if (K < n && need < ties) {
+        // cut = need-th smallest id among the ties
+        uint32_t v = 0;
+        for (int b = 31; b >= 0; --b) {
+            const uint32_t c = v | (1u << b);
+            int cnt = 0;
+            for (int e = lane; e < n; e += 32) cnt += (akey(z[e]) == tau && id[e] < c);
+            if (__reduce_add_sync(kFull, cnt) < need) v = c;
+        }
+        cut = v;
+    }
+    int base = 0;
+    for (int e0 = 0; e0 < n; e0 += 32) {
+        const int e = e0 + lane;
+        bool keep = false;
+        if (e < n) {
+            const uint32_t k = akey(z[e]);
+            keep = (K >= n) || k > tau || (k == tau && id[e] <= cut);
+        }
+        const unsigned m = __ballot_sync(kFull, keep);
+        if (keep) {
+            const int pos = base + __popc(m & ((1u << lane) - 1u));
+            oz[pos] = z[e];
+            oid[pos] = id[e];
+        }
+        base += __popc(m);
+    }
+    __syncwarp();
+    return K;
+}
+
+// ---- warp bitonic sort -------------------------------------------------------
+
+// Sorts (z, id)[0..n) in place into (|z| desc, id asc) order. `cap` is a power
+// of two >= n; slots n..cap-1 are filled with a sentinel that sorts last.
+__device__ __forceinline__ void warp_sort(float *z, uint32_t *id, int n, int cap) {
+    const int lane = threadIdx.x & 31;
+    for (int e = n + lane; e < cap; e += 32) {
+        z[e] = 0.f;
+        id[e] = 0xffffffffu;
+    }
+    __syncwarp();
+    for (int size = 2; size <= cap; size <<= 1) {
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            for (int i = lane; i < cap; i += 32) {
+                const int j = i ^ stride;
+                if (j > i) {
+                    const bool up = (i & size) == 0;  // this run ascends in (before) order
+                    const uint32_t ki = akey(z[i]), kj = akey(z[j]);
+                    const bool swap = up ? before(kj, id[j], ki, id[i]) : before(ki, id[i], kj, id[j]);
+                    if (swap) {
+                        const float tz = z[i];
+                        z[i] = z[j];
+                        z[j] = tz;
+                        const uint32_t ti = id[i];
+                        id[i] = id[j];
+                        id[j] = ti;
+                    }
+                }
+            }
+            __syncwarp();
+        }
+    }
+}
+
+__device__ __forceinline__ void set_status(int32_t *status, int32_t bit) {
+    if (status) atomicOr(status, bit);
+}
+
+}  // namespace dpb

@@ -1,0 +1,50 @@
+// dpb_internal.h -- private declarations shared by the library's translation
+// units (plan builder, C-ABI layer, kernel launchers). Not installed.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <cstdint>
+#include <vector>
+
+#include "../../include/dpb.h"
+
+struct dpb_plan {
+    dpb_config cfg;             // resolved: every derived field filled in
+    int device = 0;             // device current at creation; tables live there
+    int t = 0;                  // field GF(2^t)
+    uint32_t poly = 0;          // p(z), bit t set
+    int code_len = 0;           // k (global) or sum of k_per_level
+    uint32_t m_mask = 0;        // 2^N - 1, N = bits[levels-1]
+    float inv_sqrt_d = 0.f;     // fp32(1 / sqrt(d))
+    std::vector<uint32_t> M;    // [d] packed seed-matrix rows
+    std::vector<uint32_t> G;    // [DPB_MAX_LEVELS * DPB_MAX_CHILDREN]
+    uint32_t *dM = nullptr;     // device copy of M
+    uint32_t *dG = nullptr;     // device copy of G
+};
+
+namespace dpb {
+
+// Records a message for dpb_last_error() and returns `s`.
+dpb_status fail(dpb_status s, const char *fmt, ...);
+
+// Builds field, seed matrix and generators on the host (dpb_plan.cu).
+dpb_status resolve_and_build(const dpb_config *in, const uint32_t *generators, dpb_plan *p);
+
+// Kernel launchers (return cudaGetLastError() of the launch).
+cudaError_t launch_encode(const dpb_plan *p, const void *x, int64_t T, const float *mu,
+                          const float *sigma, int32_t *idx, float *val, float *xnorm,
+                          int32_t *status, cudaStream_t stream);
+cudaError_t launch_decode(const dpb_plan *p, const int32_t *idx, const float *val, int64_t T,
+                          const float *xnorm, void *y, int32_t *status, cudaStream_t stream);
+cudaError_t launch_backward(const dpb_plan *p, const void *x, const int32_t *idx,
+                            const float *val, int64_t T, const float *sigma, const void *grad_y,
+                            void *grad_x, float *grad_val, int32_t *status,
+                            cudaStream_t stream);
+
+// Dynamic shared memory (bytes) the encode kernel needs per warp / per block
+// header, used both to pick the launch shape and to reject plans that do not fit.
+size_t encode_smem_per_warp(const dpb_plan *p);
+size_t encode_smem_header(const dpb_plan *p);
+
+}  // namespace dpb

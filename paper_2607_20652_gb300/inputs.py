@@ -71,16 +71,29 @@ class PlantedTree:
     coef: np.ndarray
 
 
+def _distinct_rows(g: np.random.Generator, T: int, n: int, high: int) -> np.ndarray:
+    """[T, n] integers below `high`, distinct within each row: a random
+    permutation prefix when collisions are likely, else redraws of the rows
+    that repeat a value."""
+    if n * n > high // 4:
+        return np.argsort(g.random((T, high)), axis=1)[:, :n]
+    out = g.integers(0, high, size=(T, n))
+    while True:
+        s = np.sort(out, axis=1)
+        bad = np.nonzero(np.any(s[:, 1:] == s[:, :-1], axis=1))[0]
+        if len(bad) == 0:
+            return out
+        out[bad] = g.integers(0, high, size=(len(bad), n))
+
+
 def planted_tree(T: int, d: int, levels: int, children, per_level, seed: int) -> PlantedTree:
     g = rng(seed)
-    n0 = per_level[0]
-    roots = np.stack([g.choice(d, size=n0, replace=False) for _ in range(T)]).astype(np.int64)
+    roots = _distinct_rows(g, T, per_level[0], d).astype(np.int64)
     parent, gen = [None], [None]
     for l in range(1, levels):
         n_prev, n_here = per_level[l - 1], per_level[l]
         # distinct (parent slot, generator slot) pairs per token
-        pairs = np.stack([g.choice(n_prev * children[l], size=n_here, replace=False)
-                          for _ in range(T)])
+        pairs = _distinct_rows(g, T, n_here, n_prev * children[l])
         parent.append(pairs // children[l])
         gen.append(pairs % children[l])
     k = int(sum(per_level[:levels]))

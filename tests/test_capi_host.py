@@ -1,0 +1,106 @@
+"""CPU tests of the C-ABI library: it loads, exports every entry point that
+include/dpb.h declares, and its host-side plan builder (field, seed matrix,
+generators, config resolution) agrees bit-exactly with the oracle's
+independent construction. No compute call is made here."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2607_20652_gb300 import build, dpb
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return dpb.load()
+
+
+def _declared():
+    text = open(os.path.join(ROOT, "include", "dpb.h")).read()
+    return sorted(set(re.findall(r"^\s*(?:const\s+char\s*\*|dpb_status)\s*(dpb_\w+)\s*\(", text, re.M)))
+
+
+def test_library_exports_every_declared_symbol(lib):
+    names = _declared()
+    assert len(names) >= 12
+    for name in names:
+        assert hasattr(lib, name), name
+    out = os.popen(f"nm -D --defined-only {dpb.library_path()}").read()
+    exported = set(re.findall(r" T (dpb_\w+)", out))
+    assert set(names) <= exported
+    assert set(dpb.EXPORTS) == set(names)
+
+
+def test_status_strings(lib):
+    assert lib.dpb_status_string(0) == b"ok"
+    assert lib.dpb_status_string(2) == b"unsupported configuration"
+
+
+CASES = [
+    # name, d, m_bits, levels, beam, k
+    ("tiny", 64, 12, 3, 4, 8),
+    ("gpt2", 768, 16, 4, 8, 32),
+    ("wide", 768, 20, 5, 8, 64),
+    ("sweep_2^18", 768, 18, 5, 16, 128),
+    ("sweep_2^22", 768, 22, 5, 4, 16),
+    ("paper_small_3l", 1024, 17, 3, 8, 64),
+]
+
+
+@pytest.mark.parametrize("name,d,m_bits,levels,beam,k", CASES)
+def test_plan_tables_match_oracle(lib, name, d, m_bits, levels, beam, k):
+    for seed in (0, 12345):
+        plan = dpb.Plan(d=d, levels=levels, m_bits=m_bits, children=16, beam=beam, k=k, seed=seed)
+        ref = oracle.resolve(d=d, m_bits=m_bits, levels=levels, children=16, beam=beam, k=k, seed=seed)
+        cfg = plan.config
+        assert cfg["bits"] == ref.bits
+        assert cfg["field_t"] == ref.t and cfg["field_poly"] == ref.poly
+        M, G = plan.tables()
+        assert np.array_equal(M, ref.M)
+        for l in range(1, levels):
+            assert np.array_equal(G[l, :16], ref.G[l, :16])
+            assert np.all(G[l, 16:] == 0)
+
+
+@pytest.mark.parametrize("t", [6, 7, 8, 9, 12, 13])
+def test_default_polynomials_match_oracle(lib, t):
+    # the library's and the oracle's default-polynomial rules agree
+    d = 1 << min(t, 12)
+    plan = dpb.Plan(d=min(d, 4096), levels=2, m_bits=2 * t, children=4, beam=2, k=4, field_t=t)
+    assert plan.config["field_poly"] == oracle.default_poly(t)
+    M, _ = plan.tables()
+    assert np.array_equal(M, oracle.seed_matrix(plan.d, t, oracle.default_poly(t)))
+
+
+def test_explicit_generators_are_used(lib):
+    G = np.zeros((8, 256), dtype=np.uint32)
+    G[1, :16] = [(h << 6) | s for h in range(1, 9) for s in (0, 1)]
+    plan = dpb.Plan(d=64, levels=2, m_bits=12, children=16, beam=4, k=8, generators=G,
+                    bits=[6, 12], dtype="f32")
+    _, got = plan.tables()
+    assert np.array_equal(got[1, :16], G[1, :16])
+
+
+@pytest.mark.parametrize("kw,status", [
+    (dict(k=65, d=64), 1),                      # k > d
+    (dict(beam=33), 2),                         # beam outside [1, 32]
+    (dict(k=257, d=512), 2),                    # k outside [1, 256]
+    (dict(field_poly=0x41, field_t=6), 1),      # z^6+1 = (z^3+1)^2 is reducible
+    (dict(bits=[6, 6, 12]), 1),                 # bits must increase
+    (dict(children=[0, 300, 16]), 2),           # children outside [1, 256]
+    (dict(d=5000), 2),                          # d outside [2, 4096]
+    (dict(m_bits=40), 2),                       # index space beyond 2^31
+    (dict(children=[0, 65, 16], bits=[6, 7, 12]), 1),  # only 64 valid generators at level 1
+])
+def test_invalid_configs_are_rejected(lib, kw, status):
+    args = dict(d=64, levels=3, m_bits=12, children=16, beam=4, k=8, dtype="f32")
+    args.update(kw)
+    with pytest.raises(dpb.DPBError) as e:
+        dpb.Plan(**args)
+    assert e.value.status == status

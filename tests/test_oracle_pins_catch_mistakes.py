@@ -34,7 +34,7 @@ def test_kloosterman_pin_catches_a_wrong_inverse():
     one_off = M.copy()
     one_off[5] ^= np.uint32(1 << t)                                         # one row's inverse wrong
     assert pins.kloosterman_generation_mismatch(one_off, t, mul, inv, tr, pairs) > 0
-    wrong_poly = oracle.seed_matrix(d, t, 0x49)                             # z^6+z^3+1 (reducible)
+    wrong_poly = oracle.seed_matrix(d, t, 0x49)                             # another field: z^6+z^3+1
     assert pins.kloosterman_generation_mismatch(wrong_poly, t, mul, inv, tr, pairs) > 0
 
 
