@@ -1,0 +1,63 @@
+"""Host logic of the benchmark's multi-rank path, on CPU with gloo ranks:
+each rank gets its own token shard (distinct seeds), the timed region is
+closed by a barrier, the reported time is the max over ranks and the value is
+the whole-job rate. Also the roofline arithmetic on known numbers."""
+import os
+import socket
+
+import pytest
+import torch.multiprocessing as mp
+
+import bench
+
+
+def _free_port():
+    s = socket.socket()
+    s.bind(("127.0.0.1", 0))
+    port = s.getsockname()[1]
+    s.close()
+    return port
+
+
+def _worker(rank, world, port, q):
+    import torch.distributed as dist
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank),
+                      WORLD_SIZE=str(world), LOCAL_RANK=str(rank))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    ws, r, local = bench.dist_env()
+    seed = bench.shard_seed(0, r)
+    bench.barrier(ws)
+    t = bench.max_over_ranks(1.0 + r, ws)
+    q.put((r, ws, local, seed, t))
+    dist.destroy_process_group()
+
+
+def test_two_gloo_ranks_shard_and_take_the_max():
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_worker, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(120)
+        assert p.exitcode == 0
+    out = sorted(q.get(timeout=10) for _ in range(2))
+    assert [o[0] for o in out] == [0, 1] and all(o[1] == 2 for o in out)
+    assert out[0][3] != out[1][3]                       # distinct token shards
+    assert all(o[4] == 2.0 for o in out)                # max over ranks
+    assert bench.whole_job_rate(65536, 2, 10, 2.0) == 65536 * 2 * 10 / 2.0
+
+
+def test_roofline_arithmetic():
+    cfg = {"d": 768, "k": 64, "beam": 8, "levels": 5, "children": [0, 16, 16, 16, 16]}
+    work = bench.algorithmic_work(cfg, 65536, 40.0, 2)
+    assert work["encode"]["bytes"] == 65536 * 2052
+    assert work["encode"]["tensor_flops"] == 65536 * 4 * 2 * 8 * 16 * 768
+    assert work["backward"]["bytes"] == 65536 * 5376
+    peaks = {"hbm_gbs": 6781.4, "bf16_tflops_sustained": 1714.8, "sm_max_mhz": 2070.0}
+    r = bench.roofline_for("encode", work["encode"], 60e-6, peaks, "measured")
+    assert r["bound"] == "tensor"
+    assert abs(r["frac"] - (work["encode"]["tensor_flops"] / 60e-6 / 1714.8e12)) < 1e-3
+    r = bench.roofline_for("decode", work["decode"], 100e-6, peaks, "measured")
+    assert r["bound"] == "alu" and abs(r["peak"] - 152 * 128 * 2070e6 / 1e12) < 1e-3
