@@ -201,6 +201,30 @@ dpb_status dpb_backward(const dpb_plan *plan, const void *x, const int32_t *idx,
 dpb_status dpb_workspace_status(const void *workspace, int clear, int32_t *status_out,
                                 void *stream);
 
+/*
+ * dpb_encode_noalloc -- dpb_encode for callers that cannot allocate device
+ * memory. The paper has no counterpart: this is a deployment convenience.
+ * Some callers cannot call cudaMalloc or hand over a workspace, for example a
+ * plug-in that runs inside another runtime which owns every device
+ * allocation and passes it only its input and output buffers. This entry
+ * point takes the same inputs and outputs as dpb_encode but no workspace: its
+ * scratch (the device status word) lives in a file-scope device array of
+ * 4096 bytes that every GPU which loads the library keeps until the process
+ * exits. It allocates nothing: no cudaMalloc, no cudaFree, no allocating
+ * library routine.
+ *   status_out  device int32 (nullable): receives the DPB_DEV_* bits of this
+ *               call (the scratch word is cleared at the start of each call)
+ * Plans whose scratch need (dpb_workspace_size) exceeds 4096 bytes are
+ * rejected with DPB_ERR_UNSUPPORTED. The first call on a device looks up the
+ * array's device address (cudaGetSymbolAddress); make that first call before
+ * any stream capture. Every call on a device shares the one array, so calls
+ * whose kernels overlap on the GPU (different streams, or several host
+ * threads) race on it and must be serialised by the caller.
+ */
+dpb_status dpb_encode_noalloc(const dpb_plan *plan, const void *x, int64_t T, const float *mu,
+                              const float *sigma, int32_t *idx, float *val, float *xnorm,
+                              int32_t *status_out, void *stream);
+
 /* Static description of a status code. */
 const char *dpb_status_string(dpb_status s);
 

@@ -62,7 +62,7 @@ class Config(ctypes.Structure):
 _lib = None
 EXPORTS = ("dpb_plan_create", "dpb_plan_destroy", "dpb_plan_config", "dpb_plan_tables",
            "dpb_code_length", "dpb_workspace_size", "dpb_encode", "dpb_decode", "dpb_backward",
-           "dpb_workspace_status", "dpb_status_string", "dpb_last_error")
+           "dpb_workspace_status", "dpb_status_string", "dpb_last_error", "dpb_encode_noalloc")
 
 
 def library_path() -> str:
@@ -91,6 +91,7 @@ def load(path: Optional[str] = None):
     lib.dpb_decode.argtypes = [vp, vp, vp, i64, vp, vp, vp, sz, vp]
     lib.dpb_backward.argtypes = [vp, vp, vp, vp, i64, vp, vp, vp, vp, vp, sz, vp]
     lib.dpb_workspace_status.argtypes = [vp, ctypes.c_int, ctypes.POINTER(ctypes.c_int32), vp]
+    lib.dpb_encode_noalloc.argtypes = [vp, vp, i64, vp, vp, vp, vp, vp, vp, vp]
     lib.dpb_status_string.argtypes = [st]
     lib.dpb_status_string.restype = ctypes.c_char_p
     lib.dpb_last_error.argtypes = []
