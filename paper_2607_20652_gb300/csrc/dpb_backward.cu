@@ -1,0 +1,452 @@
+// dpb_backward.cu -- gradients of decode(encode(x)) with the selected set held
+// fixed (the paper trains through the layer end to end but does not write the
+// backward out; it is derived by the chain rule), one warp per token.
+//
+// With g = dL/dy, r = sum_e val_e phi_e, c = |x| / |r| and norm matching:
+//   dL/dr      = c (g - (<g,r> / |r|^2) r)          (g without norm matching)
+//   grad_val_e = <phi_e, dL/dr>
+//   grad_x     = sum_e (grad_val_e / sigma_e) phi_e + (<g,r>/|r|) x / |x|.
+// The table-driven kernel (d <= 1024) evaluates the two sums over phi with the
+// sweeps of dpb_lut.cuh and the inner products <phi_e, dL/dr> with per-token
+// tables of signed sums of dL/dr over 4 coordinates (see analyse()).
+#include <algorithm>
+#include <climits>
+
+#include "dpb_device.cuh"
+#include "dpb_internal.h"
+#include "dpb_lut.cuh"
+
+namespace dpb {
+
+namespace {
+
+struct BackwardArgs {
+    const void *x, *gy;
+    const int32_t *idx;
+    const float *val, *sigma;
+    void *gx;
+    float *gval;
+    int64_t T;
+    int32_t *status;
+    const uint32_t *M, *VH;
+    int d, k, norm_match;
+    uint32_t m_mask;
+    float inv_sqrt_d;
+};
+
+// r (basis part rb, hashed +-sum rh) of one token into shared memory; lane l
+// owns coordinates l, l+32, ... so no two lanes touch the same word.
+__device__ void reconstruct(const int32_t *idx, const float *val, int k, int d, uint32_t m_mask,
+                            const uint32_t *sM, float *rb, float *rh, int32_t *status) {
+    const int lane = threadIdx.x & 31;
+    for (int i = lane; i < d; i += 32) {
+        rb[i] = 0.f;
+        rh[i] = 0.f;
+    }
+    for (int e = 0; e < k; ++e) {
+        const int32_t ci = idx[e];
+        const float a = val[e];
+        if (ci < 0 || (uint32_t)ci > m_mask) {
+            if (lane == 0) set_status(status, DPB_DEV_BAD_INDEX);
+            continue;
+        }
+        const uint32_t c = (uint32_t)ci;
+        if (c < (uint32_t)d) {
+            if ((int)(c & 31) == lane) rb[c] += a;
+        } else {
+            for (int i = lane; i < d; i += 32) rh[i] += flip(a, sign31(sM[i], c));
+        }
+    }
+}
+
+template <typename Tio>
+__global__ void __launch_bounds__(128) backward_warp_kernel(BackwardArgs a) {
+    extern __shared__ __align__(16) uint32_t smem[];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+    const int d = a.d;
+    uint32_t *sM = smem;
+    for (int i = threadIdx.x; i < d; i += blockDim.x) sM[i] = a.M[i];
+    __syncthreads();
+    float *rb = reinterpret_cast<float *>(sM + d) + (size_t)warp * 4 * d;
+    float *rh = rb + d;    // hashed sum, then reused as dL/dr
+    float *xs = rh + d;
+    float *gx = xs + d;
+    const Tio *X = static_cast<const Tio *>(a.x);
+    const Tio *GY = static_cast<const Tio *>(a.gy);
+    Tio *GX = static_cast<Tio *>(a.gx);
+    for (int64_t t = (int64_t)blockIdx.x * nwarps + warp; t < a.T; t += (int64_t)gridDim.x * nwarps) {
+        const int32_t *it = a.idx + t * a.k;
+        const float *vt = a.val + t * a.k;
+        float sxx = 0.f;
+        for (int i = lane; i < d; i += 32) {
+            const float v = ld_elem(X, t * d + i);
+            xs[i] = v;
+            sxx += v * v;
+        }
+        const float nx = sqrtf(warp_sum(sxx));
+        float direct = 0.f;  // coefficient of x/|x| in grad_x
+        if (a.norm_match) {
+            reconstruct(it, vt, a.k, d, a.m_mask, sM, rb, rh, a.status);
+            __syncwarp();
+            float srr = 0.f, sgr = 0.f;
+            for (int i = lane; i < d; i += 32) {
+                const float r = rb[i] + rh[i] * a.inv_sqrt_d;
+                rb[i] = r;
+                srr += r * r;
+                sgr += ld_elem(GY, t * d + i) * r;
+            }
+            srr = warp_sum(srr);
+            sgr = warp_sum(sgr);
+            const float nr = sqrtf(srr);
+            if (nr > 0.f) {
+                const float c = nx / nr, beta = sgr / srr;
+                for (int i = lane; i < d; i += 32) rh[i] = c * (ld_elem(GY, t * d + i) - beta * rb[i]);
+                direct = nx > 0.f ? sgr / nr : 0.f;
+            } else {
+                for (int i = lane; i < d; i += 32) rh[i] = 0.f;
+            }
+        } else {
+            for (int i = lane; i < d; i += 32) rh[i] = ld_elem(GY, t * d + i);
+        }
+        const float dx = nx > 0.f ? direct / nx : 0.f;
+        for (int i = lane; i < d; i += 32) gx[i] = dx * xs[i];
+        __syncwarp();
+        // grad_val_e = <phi_e, dL/dr>; grad_x += (grad_val_e / sigma_e) phi_e
+        for (int e = 0; e < a.k; ++e) {
+            const int32_t ci = it[e];
+            if (ci < 0 || (uint32_t)ci > a.m_mask) {
+                if (lane == 0) {
+                    set_status(a.status, DPB_DEV_BAD_INDEX);
+                    a.gval[t * a.k + e] = 0.f;
+                }
+                continue;
+            }
+            const uint32_t c = (uint32_t)ci;
+            float sd = 1.f;
+            if (a.sigma) {
+                sd = a.sigma[c];
+                if (!(sd > 0.f) && lane == 0) set_status(a.status, DPB_DEV_BAD_SIGMA);
+            }
+            if (c < (uint32_t)d) {
+                const float gv = rh[c];
+                if (lane == 0) a.gval[t * a.k + e] = gv;
+                if ((int)(c & 31) == lane) gx[c] += gv / sd;
+            } else {
+                float acc = 0.f;
+                for (int i = lane; i < d; i += 32) acc += flip(rh[i], sign31(sM[i], c));
+                const float gv = warp_sum(acc) * a.inv_sqrt_d;
+                if (lane == 0) a.gval[t * a.k + e] = gv;
+                const float w = (gv / sd) * a.inv_sqrt_d;
+                for (int i = lane; i < d; i += 32) gx[i] += flip(w, sign31(sM[i], c));
+            }
+            __syncwarp();
+        }
+        for (int i = lane; i < d; i += 32) st_elem(GX, t * d + i, gx[i]);
+        __syncwarp();
+    }
+}
+
+
+// ---- table-driven backward (d <= 1024) ---------------------------------------
+
+constexpr int kChunkBlocks = 8;                       // 32-coordinate blocks per analysis chunk
+constexpr int kTabStride = 17;                        // 16 entries + 1 pad (bank spread)
+constexpr int kChunkTables = kChunkBlocks * 8 * kTabStride;  // nibble tables of a chunk (words)
+
+__host__ __device__ constexpr int bwd_warp_words(int d, int k) {
+    return 2 * pad4(d) /* r then grad_x; dL/dr */ + 6 * pad4(k) /* list, map, sums, offsets */ +
+           (kSweepWords > kChunkTables ? kSweepWords : pad4(kChunkTables));
+}
+
+__host__ __device__ constexpr int bwd_block_words(int d, int nkc) {
+    return pad4(d) /* koff */ + 32 /* W5 */ + 1024 /* PQ */ + nkc * 1024 /* VH */;
+}
+
+struct BwdWarp {
+    float *rg;      // [d] r, later grad_x
+    float *h;       // [d] dL/dr
+    uint32_t *hc;   // [k] hashed indices
+    float *ha;      // [k] hashed coefficients, later grad_val / sigma
+    int *cmap;      // [k] code entry -> hashed position (>= 0) or -(c+1) (basis) or INT_MIN
+    float *gv;      // [k] analysis sums per hashed position
+    uint32_t *o1;   // [k] packed table offsets (W5, PQ, VH_0, VH_1)
+    uint32_t *o2;   // [k] packed table offsets (VH_2, VH_3)
+    uint32_t *scratch;
+};
+
+// Table offsets (bytes) of code c in the sign-word tables of a block:
+// W5[c & 31], PQ[q][(c_lo >> 5) & 31], VH_k[q][(c >> (t + 5k)) & 31].
+__device__ __forceinline__ void code_offsets(uint32_t c, int t, uint32_t &o1, uint32_t &o2) {
+    const uint32_t lo = c & ((1u << t) - 1u);
+    const uint32_t b0 = (c & 31u) * 4u, b1 = ((lo >> 5) & 31u) * 4u;
+    const uint32_t h0 = ((c >> t) & 31u) * 4u, h1 = ((c >> (t + 5)) & 31u) * 4u;
+    const uint32_t h2 = (t + 10 < 32) ? ((c >> (t + 10)) & 31u) * 4u : 0u;
+    const uint32_t h3 = (t + 15 < 32) ? ((c >> (t + 15)) & 31u) * 4u : 0u;
+    o1 = b0 | (b1 << 8) | (h0 << 16) | (h1 << 24);
+    o2 = h2 | (h3 << 8);
+}
+
+// Sign word of code (o1, o2) over block q: bit l = parity(M[32q + l] AND c).
+template <int NKC>
+__device__ __forceinline__ uint32_t block_signs(const uint32_t *w5, const uint32_t *pq, const uint32_t *vh,
+                                                int q, uint32_t o1, uint32_t o2) {
+    const char *W = reinterpret_cast<const char *>(w5);
+    const char *P = reinterpret_cast<const char *>(pq + q * 32);
+    const char *V = reinterpret_cast<const char *>(vh + q * 32);
+    uint32_t s = *reinterpret_cast<const uint32_t *>(W + __byte_perm(o1, 0, 0x4440)) ^
+                 *reinterpret_cast<const uint32_t *>(P + __byte_perm(o1, 0, 0x4441)) ^
+                 *reinterpret_cast<const uint32_t *>(V + __byte_perm(o1, 0, 0x4442));
+    s ^= *reinterpret_cast<const uint32_t *>(V + 4096 + __byte_perm(o1, 0, 0x4443));
+    if (NKC > 2) s ^= *reinterpret_cast<const uint32_t *>(V + 8192 + __byte_perm(o2, 0, 0x4440));
+    if (NKC > 3) s ^= *reinterpret_cast<const uint32_t *>(V + 12288 + __byte_perm(o2, 0, 0x4441));
+    return s;
+}
+
+// gv[p] += sum_i h[i] (-1)^{parity(M[i] AND hc_p)} for the nh hashed codes.
+// Per chunk of 8 blocks: nibble tables TH[b][n][v] = sum_j (-1)^{v_j}
+// h[32b + 4n + j] (16 entries per 4 coordinates), then one (code, block) item
+// per lane: the code's sign word over the block indexes 8 nibble tables.
+// Items of one warp step have distinct codes, so the shared-memory
+// accumulation order is fixed.
+template <int NKC>
+__device__ __forceinline__ void analyse(const BwdWarp &w, int nh, int d, const uint32_t *w5,
+                                        const uint32_t *pq, const uint32_t *vh) {
+    const int lane = threadIdx.x & 31;
+    const int qn = (d + 31) / 32;
+    const int nhp = nh > 32 ? nh : 32;
+    float *TH = reinterpret_cast<float *>(w.scratch);
+    for (int q0 = 0; q0 < qn; q0 += kChunkBlocks) {
+        const int cq = min(kChunkBlocks, qn - q0);
+        for (int tau = lane; tau < cq * 8; tau += 32) {
+            const int i0 = 32 * (q0 + tau / 8) + 4 * (tau % 8);  // = 4 (8 q0 + tau)
+            float4 hv = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (i0 + 3 < d) {
+                hv = *reinterpret_cast<const float4 *>(w.h + i0);
+            } else {
+                if (i0 < d) hv.x = w.h[i0];
+                if (i0 + 1 < d) hv.y = w.h[i0 + 1];
+                if (i0 + 2 < d) hv.z = w.h[i0 + 2];
+            }
+            // entry v = (v3 v2 v1 v0): sum_j (-1)^{v_j} h_j = A[v1 v0] + B[v3 v2]
+            const float a0 = hv.x + hv.y, a1 = hv.x - hv.y;
+            const float b0 = hv.z + hv.w, b1 = hv.z - hv.w;
+            float *T = TH + tau * kTabStride;
+            // v0 = 1 negates h0: A[01] = -h0 + h1 = -a1, A[10] = h0 - h1 = a1
+            const float A[4] = {a0, -a1, a1, -a0};
+            const float B[4] = {b0, -b1, b1, -b0};
+#pragma unroll
+            for (int v = 0; v < 16; ++v) T[v] = A[v & 3] + B[v >> 2];
+        }
+        __syncwarp();
+        for (int it = lane; it < cq * nhp; it += 32) {
+            const int qq = it / nhp, e = it - qq * nhp;
+            if (e < nh) {
+                const uint32_t s = block_signs<NKC>(w5, pq, vh, q0 + qq, w.o1[e], w.o2[e]);
+                const char *T = reinterpret_cast<const char *>(TH + qq * 8 * kTabStride);
+                constexpr int S4 = 4 * kTabStride;  // bytes per table
+                float p0 = *reinterpret_cast<const float *>(T + ((s << 2) & 0x3Cu));
+                float p1 = *reinterpret_cast<const float *>(T + 1 * S4 + ((s >> 2) & 0x3Cu));
+                float p2 = *reinterpret_cast<const float *>(T + 2 * S4 + ((s >> 6) & 0x3Cu));
+                float p3 = *reinterpret_cast<const float *>(T + 3 * S4 + ((s >> 10) & 0x3Cu));
+                float p4 = *reinterpret_cast<const float *>(T + 4 * S4 + ((s >> 14) & 0x3Cu));
+                float p5 = *reinterpret_cast<const float *>(T + 5 * S4 + ((s >> 18) & 0x3Cu));
+                float p6 = *reinterpret_cast<const float *>(T + 6 * S4 + ((s >> 22) & 0x3Cu));
+                float p7 = *reinterpret_cast<const float *>(T + 7 * S4 + ((s >> 26) & 0x3Cu));
+                atomicAdd(&w.gv[e], ((p0 + p1) + (p2 + p3)) + ((p4 + p5) + (p6 + p7)));
+            }
+        }
+        __syncwarp();
+    }
+}
+
+template <typename Tio, int NKC>
+__global__ void __launch_bounds__(128) backward_lut_kernel(BackwardArgs a, int t) {
+    extern __shared__ __align__(16) uint32_t smem[];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+    const int d = a.d, k = a.k;
+    const int dp = pad4(d), kp = pad4(k);
+    uint32_t *koff = smem;
+    uint32_t *w5 = koff + dp;
+    uint32_t *pq = w5 + 32;
+    uint32_t *vh = pq + 1024;
+    for (int v = threadIdx.x; v < 32; v += blockDim.x) {
+        uint32_t word = 0;
+        for (int l = 0; l < 32; ++l) word |= (uint32_t)(__popc(l & v) & 1) << l;
+        w5[v] = word;
+    }
+    for (int i = threadIdx.x; i < 1024; i += blockDim.x) pq[i] = (__popc((i >> 5) & (i & 31)) & 1) ? ~0u : 0u;
+    for (int i = threadIdx.x; i < NKC * 1024; i += blockDim.x) vh[i] = a.VH[i];
+    load_koff(a.M, d, t, koff);  // ends with __syncthreads()
+
+    uint32_t *base = smem + bwd_block_words(d, NKC) + (size_t)warp * bwd_warp_words(d, k);
+    BwdWarp w;
+    w.rg = reinterpret_cast<float *>(base);
+    w.h = w.rg + dp;
+    w.hc = reinterpret_cast<uint32_t *>(w.h + dp);
+    w.ha = reinterpret_cast<float *>(w.hc + kp);
+    w.cmap = reinterpret_cast<int *>(w.ha + kp);
+    w.gv = reinterpret_cast<float *>(w.cmap + kp);
+    w.o1 = reinterpret_cast<uint32_t *>(w.gv + kp);
+    w.o2 = w.o1 + kp;
+    w.scratch = w.o2 + kp;
+    Sweep sw = sweep_at(w.scratch);
+
+    const Tio *X = static_cast<const Tio *>(a.x);
+    const Tio *GY = static_cast<const Tio *>(a.gy);
+    Tio *GX = static_cast<Tio *>(a.gx);
+    for (int64_t tk = (int64_t)blockIdx.x * nwarps + warp; tk < a.T; tk += (int64_t)gridDim.x * nwarps) {
+        const int32_t *it = a.idx + tk * k;
+        const float *vt = a.val + tk * k;
+        // ---- split the code: basis entries into rg, hashed entries listed ----
+        for (int i = lane; i < d; i += 32) w.rg[i] = 0.f;
+        __syncwarp();
+        int nh = 0;
+        for (int e0 = 0; e0 < k; e0 += 32) {
+            const int e = e0 + lane;
+            int32_t ci = -1;
+            float v = 0.f;
+            if (e < k) {
+                ci = it[e];
+                v = vt[e];
+            }
+            const bool valid = e < k && ci >= 0 && (uint32_t)ci <= a.m_mask;
+            const bool hashed = valid && ci >= d;
+            if (e < k && !valid) {
+                set_status(a.status, DPB_DEV_BAD_INDEX);
+                w.cmap[e] = INT_MIN;
+            }
+            if (valid && !hashed) {
+                atomicAdd(&w.rg[ci], v);
+                w.cmap[e] = -(ci + 1);
+            }
+            const unsigned m = __ballot_sync(kFull, hashed);
+            if (hashed) {
+                const int pos = nh + __popc(m & ((1u << lane) - 1u));
+                w.hc[pos] = (uint32_t)ci;
+                w.ha[pos] = v;
+                w.cmap[e] = pos;
+                w.gv[pos] = 0.f;
+                code_offsets((uint32_t)ci, t, w.o1[pos], w.o2[pos]);
+            }
+            nh += __popc(m);
+        }
+        __syncwarp();
+        // ---- |x|, r and dL/dr ----
+        float sxx = 0.f;
+        for (int i = lane; i < d; i += 32) {
+            const float xv = ld_elem(X, tk * d + i);
+            sxx += xv * xv;
+        }
+        const float nx = sqrtf(warp_sum(sxx));
+        float direct = 0.f;
+        if (a.norm_match) {
+            synthesise<NKC>(sw, w.hc, w.ha, nh, t, d, koff, a.inv_sqrt_d, w.rg);
+            float srr = 0.f, sgr = 0.f;
+            for (int i = lane; i < d; i += 32) {
+                const float r = w.rg[i], g = ld_elem(GY, tk * d + i);
+                w.h[i] = g;
+                srr += r * r;
+                sgr += g * r;
+            }
+            srr = warp_sum(srr);
+            sgr = warp_sum(sgr);
+            const float nr = sqrtf(srr);
+            if (nr > 0.f) {
+                const float c = nx / nr, beta = sgr / srr;
+                for (int i = lane; i < d; i += 32) w.h[i] = c * (w.h[i] - beta * w.rg[i]);
+                direct = nx > 0.f ? sgr / nr : 0.f;
+            } else {
+                for (int i = lane; i < d; i += 32) w.h[i] = 0.f;
+            }
+        } else {
+            for (int i = lane; i < d; i += 32) w.h[i] = ld_elem(GY, tk * d + i);
+        }
+        __syncwarp();
+        // ---- grad_val = <phi_e, dL/dr> ----
+        analyse<NKC>(w, nh, d, w5, pq, vh);
+        // ---- grad_x: direct term, basis terms, then the hashed sum ----
+        const float dx = nx > 0.f ? direct / nx : 0.f;
+        for (int i = lane; i < d; i += 32) w.rg[i] = dx * ld_elem(X, tk * d + i);
+        __syncwarp();
+        for (int e = lane; e < k; e += 32) {
+            const int cm = w.cmap[e];
+            float gvv = 0.f;
+            if (cm >= 0) {
+                gvv = w.gv[cm] * a.inv_sqrt_d;
+                float sd = 1.f;
+                if (a.sigma) {
+                    sd = a.sigma[w.hc[cm]];
+                    if (!(sd > 0.f)) set_status(a.status, DPB_DEV_BAD_SIGMA);
+                }
+                w.ha[cm] = gvv / sd;
+            } else if (cm != INT_MIN) {
+                const int c = -cm - 1;
+                gvv = w.h[c];
+                float sd = 1.f;
+                if (a.sigma) {
+                    sd = a.sigma[c];
+                    if (!(sd > 0.f)) set_status(a.status, DPB_DEV_BAD_SIGMA);
+                }
+                atomicAdd(&w.rg[c], gvv / sd);
+            }
+            a.gval[tk * k + e] = gvv;
+        }
+        __syncwarp();
+        synthesise<NKC>(sw, w.hc, w.ha, nh, t, d, koff, a.inv_sqrt_d, w.rg);
+        for (int i = lane; i < d; i += 32) st_elem(GX, tk * d + i, w.rg[i]);
+        __syncwarp();
+    }
+}
+
+int grid_for(const dpb_plan *p, int64_t T, int warps) {
+    int sms = 0;
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, p->device);
+    return (int)std::min<int64_t>((T + warps - 1) / warps, (int64_t)sms * 16);
+}
+
+template <typename Tio, int NKC>
+cudaError_t run_backward_lut(const dpb_plan *p, const BackwardArgs &a, int64_t T, cudaStream_t stream) {
+    const int warps = 4;
+    const size_t smem = sizeof(uint32_t) * ((size_t)bwd_block_words(p->cfg.d, NKC) +
+                                            (size_t)warps * bwd_warp_words(p->cfg.d, p->code_len));
+    cudaFuncSetAttribute(backward_lut_kernel<Tio, NKC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    backward_lut_kernel<Tio, NKC><<<grid_for(p, T, warps), warps * 32, smem, stream>>>(a, p->t);
+    return cudaGetLastError();
+}
+
+template <typename Tio>
+cudaError_t dispatch_backward_lut(const dpb_plan *p, const BackwardArgs &a, int64_t T, cudaStream_t stream) {
+    if (p->kvh <= 2) return run_backward_lut<Tio, 2>(p, a, T, stream);
+    if (p->kvh == 3) return run_backward_lut<Tio, 3>(p, a, T, stream);
+    return run_backward_lut<Tio, 4>(p, a, T, stream);
+}
+
+}  // namespace
+
+cudaError_t launch_backward(const dpb_plan *p, const void *x, const int32_t *idx,
+                            const float *val, int64_t T, const float *sigma, const void *grad_y,
+                            void *grad_x, float *grad_val, int32_t *status,
+                            cudaStream_t stream) {
+    const dpb_config &c = p->cfg;
+    BackwardArgs a{x, grad_y, idx, val, sigma, grad_x, grad_val, T, status, p->dM, p->dVH,
+                   c.d, p->code_len, c.norm_match, p->m_mask, p->inv_sqrt_d};
+    if (c.d <= 1024) {
+        return c.dtype == DPB_BF16 ? dispatch_backward_lut<__nv_bfloat16>(p, a, T, stream)
+                                   : dispatch_backward_lut<float>(p, a, T, stream);
+    }
+    const int warps = 4;
+    const size_t smem = sizeof(uint32_t) * ((size_t)c.d + (size_t)warps * 4 * c.d);
+    const int grid = grid_for(p, T, warps);
+    if (c.dtype == DPB_BF16) {
+        cudaFuncSetAttribute(backward_warp_kernel<__nv_bfloat16>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        backward_warp_kernel<__nv_bfloat16><<<grid, warps * 32, smem, stream>>>(a);
+    } else {
+        cudaFuncSetAttribute(backward_warp_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
+        backward_warp_kernel<float><<<grid, warps * 32, smem, stream>>>(a);
+    }
+    return cudaGetLastError();
+}
+
+}  // namespace dpb

@@ -92,16 +92,21 @@ dpb_status dpb_plan_create(const dpb_config *cfg, const uint32_t *generators, dp
         return dpb::fail(DPB_ERR_CUDA, "cudaGetDevice failed");
     }
     const size_t mb = sizeof(uint32_t) * p->M.size(), gb = sizeof(uint32_t) * p->G.size();
-    if (cudaMalloc(&p->dM, mb) != cudaSuccess || cudaMalloc(&p->dG, gb) != cudaSuccess) {
+    const size_t vb = sizeof(uint32_t) * p->VH.size();
+    if (cudaMalloc(&p->dM, mb) != cudaSuccess || cudaMalloc(&p->dG, gb) != cudaSuccess ||
+        cudaMalloc(&p->dVH, vb) != cudaSuccess) {
         cudaFree(p->dM);
         cudaFree(p->dG);
+        cudaFree(p->dVH);
         delete p;
         return dpb::fail(DPB_ERR_NO_MEMORY, "device table allocation failed");
     }
     if (cudaMemcpy(p->dM, p->M.data(), mb, cudaMemcpyHostToDevice) != cudaSuccess ||
-        cudaMemcpy(p->dG, p->G.data(), gb, cudaMemcpyHostToDevice) != cudaSuccess) {
+        cudaMemcpy(p->dG, p->G.data(), gb, cudaMemcpyHostToDevice) != cudaSuccess ||
+        cudaMemcpy(p->dVH, p->VH.data(), vb, cudaMemcpyHostToDevice) != cudaSuccess) {
         cudaFree(p->dM);
         cudaFree(p->dG);
+        cudaFree(p->dVH);
         delete p;
         return dpb::fail(DPB_ERR_CUDA, "device table upload failed");
     }
@@ -120,6 +125,7 @@ dpb_status dpb_plan_destroy(dpb_plan *plan) {
     if (cur != plan->device) cudaSetDevice(plan->device);
     cudaFree(plan->dM);
     cudaFree(plan->dG);
+    cudaFree(plan->dVH);
     if (cur >= 0 && cur != plan->device) cudaSetDevice(cur);
     delete plan;
     return DPB_OK;

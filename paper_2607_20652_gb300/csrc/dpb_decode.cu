@@ -1,5 +1,4 @@
-// dpb_decode.cu -- the §2.1 parity decoder and the backward of the whole
-// encode-then-decode map, one warp per token.
+// dpb_decode.cu -- the §2.1 parity decoder, one warp per token.
 //
 // r = sum_e val_e phi_{idx_e}: a basis entry (idx < d, Eq. 2) adds to one
 // coordinate; a hashed entry adds +-val to every coordinate with the sign
@@ -10,6 +9,7 @@
 
 #include "dpb_device.cuh"
 #include "dpb_internal.h"
+#include "dpb_lut.cuh"
 
 namespace dpb {
 
@@ -27,19 +27,6 @@ struct DecodeArgs {
     float inv_sqrt_d;
 };
 
-struct BackwardArgs {
-    const void *x, *gy;
-    const int32_t *idx;
-    const float *val, *sigma;
-    void *gx;
-    float *gval;
-    int64_t T;
-    int32_t *status;
-    const uint32_t *M;
-    int d, k, norm_match;
-    uint32_t m_mask;
-    float inv_sqrt_d;
-};
 
 // r (basis part rb, hashed +-sum rh) of one token into shared memory; lane l
 // owns coordinates l, l+32, ... so no two lanes touch the same word.
@@ -97,89 +84,38 @@ __global__ void __launch_bounds__(128) decode_warp_kernel(DecodeArgs a) {
     }
 }
 
-template <typename Tio>
-__global__ void __launch_bounds__(128) backward_warp_kernel(BackwardArgs a) {
+// ---- table-driven decoder (d <= 1024) -----------------------------------------
+
+// Per-warp shared memory of the decoder, in 4-byte words: r (d), the hashed
+// list (indices, coefficients) and one sweep's tables.
+__host__ __device__ constexpr int decode_warp_words(int d, int k) { return pad4(d) + 2 * pad4(k) + kSweepWords; }
+
+template <typename Tio, int NKC>
+__global__ void __launch_bounds__(256) decode_lut_kernel(DecodeArgs a, int t) {
     extern __shared__ __align__(16) uint32_t smem[];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
     const int d = a.d;
-    uint32_t *sM = smem;
-    for (int i = threadIdx.x; i < d; i += blockDim.x) sM[i] = a.M[i];
-    __syncthreads();
-    float *rb = reinterpret_cast<float *>(sM + d) + (size_t)warp * 4 * d;
-    float *rh = rb + d;    // hashed sum, then reused as dL/dr
-    float *xs = rh + d;
-    float *gx = xs + d;
-    const Tio *X = static_cast<const Tio *>(a.x);
-    const Tio *GY = static_cast<const Tio *>(a.gy);
-    Tio *GX = static_cast<Tio *>(a.gx);
-    for (int64_t t = (int64_t)blockIdx.x * nwarps + warp; t < a.T; t += (int64_t)gridDim.x * nwarps) {
-        const int32_t *it = a.idx + t * a.k;
-        const float *vt = a.val + t * a.k;
-        float sxx = 0.f;
-        for (int i = lane; i < d; i += 32) {
-            const float v = ld_elem(X, t * d + i);
-            xs[i] = v;
-            sxx += v * v;
-        }
-        const float nx = sqrtf(warp_sum(sxx));
-        float direct = 0.f;  // coefficient of x/|x| in grad_x
-        if (a.norm_match) {
-            reconstruct(it, vt, a.k, d, a.m_mask, sM, rb, rh, a.status);
-            __syncwarp();
-            float srr = 0.f, sgr = 0.f;
-            for (int i = lane; i < d; i += 32) {
-                const float r = rb[i] + rh[i] * a.inv_sqrt_d;
-                rb[i] = r;
-                srr += r * r;
-                sgr += ld_elem(GY, t * d + i) * r;
-            }
-            srr = warp_sum(srr);
-            sgr = warp_sum(sgr);
-            const float nr = sqrtf(srr);
-            if (nr > 0.f) {
-                const float c = nx / nr, beta = sgr / srr;
-                for (int i = lane; i < d; i += 32) rh[i] = c * (ld_elem(GY, t * d + i) - beta * rb[i]);
-                direct = nx > 0.f ? sgr / nr : 0.f;
-            } else {
-                for (int i = lane; i < d; i += 32) rh[i] = 0.f;
-            }
-        } else {
-            for (int i = lane; i < d; i += 32) rh[i] = ld_elem(GY, t * d + i);
-        }
-        const float dx = nx > 0.f ? direct / nx : 0.f;
-        for (int i = lane; i < d; i += 32) gx[i] = dx * xs[i];
+    uint32_t *koff = smem;
+    load_koff(a.M, d, t, koff);
+    const int dp = pad4(d), kp = pad4(a.k);
+    uint32_t *base = smem + dp + (size_t)warp * decode_warp_words(d, a.k);
+    float *r = reinterpret_cast<float *>(base);
+    HashedList hl{base + dp, reinterpret_cast<float *>(base + dp + kp), nullptr};
+    Sweep sw = sweep_at(base + dp + 2 * kp);
+    Tio *Y = static_cast<Tio *>(a.y);
+    for (int64_t tk = (int64_t)blockIdx.x * nwarps + warp; tk < a.T; tk += (int64_t)gridDim.x * nwarps) {
+        for (int i = lane; i < d; i += 32) r[i] = 0.f;
         __syncwarp();
-        // grad_val_e = <phi_e, dL/dr>; grad_x += (grad_val_e / sigma_e) phi_e
-        for (int e = 0; e < a.k; ++e) {
-            const int32_t ci = it[e];
-            if (ci < 0 || (uint32_t)ci > a.m_mask) {
-                if (lane == 0) {
-                    set_status(a.status, DPB_DEV_BAD_INDEX);
-                    a.gval[t * a.k + e] = 0.f;
-                }
-                continue;
-            }
-            const uint32_t c = (uint32_t)ci;
-            float sd = 1.f;
-            if (a.sigma) {
-                sd = a.sigma[c];
-                if (!(sd > 0.f) && lane == 0) set_status(a.status, DPB_DEV_BAD_SIGMA);
-            }
-            if (c < (uint32_t)d) {
-                const float gv = rh[c];
-                if (lane == 0) a.gval[t * a.k + e] = gv;
-                if ((int)(c & 31) == lane) gx[c] += gv / sd;
-            } else {
-                float acc = 0.f;
-                for (int i = lane; i < d; i += 32) acc += flip(rh[i], sign31(sM[i], c));
-                const float gv = warp_sum(acc) * a.inv_sqrt_d;
-                if (lane == 0) a.gval[t * a.k + e] = gv;
-                const float w = (gv / sd) * a.inv_sqrt_d;
-                for (int i = lane; i < d; i += 32) gx[i] += flip(w, sign31(sM[i], c));
-            }
-            __syncwarp();
+        const int nh = split_code(a.idx + tk * a.k, a.val + tk * a.k, a.k, d, a.m_mask, r, hl, a.status);
+        synthesise<NKC>(sw, hl.c, hl.a, nh, t, d, koff, a.inv_sqrt_d, r);
+        float ss = 0.f;
+        for (int i = lane; i < d; i += 32) ss += r[i] * r[i];
+        float scale = 1.f;
+        if (a.norm_match) {
+            const float nr = sqrtf(warp_sum(ss));
+            scale = nr > 0.f ? a.xnorm[tk] / nr : 0.f;
         }
-        for (int i = lane; i < d; i += 32) st_elem(GX, t * d + i, gx[i]);
+        for (int i = lane; i < d; i += 32) st_elem(Y, tk * d + i, r[i] * scale);
         __syncwarp();
     }
 }
@@ -192,11 +128,36 @@ int grid_for(const dpb_plan *p, int64_t T, int warps) {
 
 }  // namespace
 
+namespace {
+
+template <typename Tio, int NKC>
+cudaError_t run_decode_lut(const dpb_plan *p, const DecodeArgs &a, int64_t T, cudaStream_t stream) {
+    const int warps = 8;
+    const size_t smem = sizeof(uint32_t) * ((size_t)pad4(p->cfg.d) + (size_t)warps * decode_warp_words(p->cfg.d, p->code_len));
+    cudaFuncSetAttribute(decode_lut_kernel<Tio, NKC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    decode_lut_kernel<Tio, NKC><<<grid_for(p, T, warps), warps * 32, smem, stream>>>(a, p->t);
+    return cudaGetLastError();
+}
+
+template <typename Tio>
+cudaError_t dispatch_decode_lut(const dpb_plan *p, const DecodeArgs &a, int64_t T, cudaStream_t stream) {
+    const int nkc = (p->t + 4) / 5;
+    if (nkc <= 2) return run_decode_lut<Tio, 2>(p, a, T, stream);
+    if (nkc == 3) return run_decode_lut<Tio, 3>(p, a, T, stream);
+    return run_decode_lut<Tio, 4>(p, a, T, stream);
+}
+
+}  // namespace
+
 cudaError_t launch_decode(const dpb_plan *p, const int32_t *idx, const float *val, int64_t T,
                           const float *xnorm, void *y, int32_t *status, cudaStream_t stream) {
     const dpb_config &c = p->cfg;
     DecodeArgs a{idx, val, xnorm, y, T, status, p->dM, c.d, p->code_len, c.norm_match, p->m_mask,
                  p->inv_sqrt_d};
+    if (c.d <= 1024) {
+        return c.dtype == DPB_BF16 ? dispatch_decode_lut<__nv_bfloat16>(p, a, T, stream)
+                                   : dispatch_decode_lut<float>(p, a, T, stream);
+    }
     const int warps = 4;
     const size_t smem = sizeof(uint32_t) * ((size_t)c.d + (size_t)warps * 2 * c.d);
     const int grid = grid_for(p, T, warps);
@@ -208,28 +169,6 @@ cudaError_t launch_decode(const dpb_plan *p, const int32_t *idx, const float *va
         cudaFuncSetAttribute(decode_warp_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem);
         decode_warp_kernel<float><<<grid, warps * 32, smem, stream>>>(a);
-    }
-    return cudaGetLastError();
-}
-
-cudaError_t launch_backward(const dpb_plan *p, const void *x, const int32_t *idx,
-                            const float *val, int64_t T, const float *sigma, const void *grad_y,
-                            void *grad_x, float *grad_val, int32_t *status,
-                            cudaStream_t stream) {
-    const dpb_config &c = p->cfg;
-    BackwardArgs a{x, grad_y, idx, val, sigma, grad_x, grad_val, T, status, p->dM,
-                   c.d, p->code_len, c.norm_match, p->m_mask, p->inv_sqrt_d};
-    const int warps = 4;
-    const size_t smem = sizeof(uint32_t) * ((size_t)c.d + (size_t)warps * 4 * c.d);
-    const int grid = grid_for(p, T, warps);
-    if (c.dtype == DPB_BF16) {
-        cudaFuncSetAttribute(backward_warp_kernel<__nv_bfloat16>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        backward_warp_kernel<__nv_bfloat16><<<grid, warps * 32, smem, stream>>>(a);
-    } else {
-        cudaFuncSetAttribute(backward_warp_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)smem);
-        backward_warp_kernel<float><<<grid, warps * 32, smem, stream>>>(a);
     }
     return cudaGetLastError();
 }

@@ -19,8 +19,14 @@ struct dpb_plan {
     float inv_sqrt_d = 0.f;     // fp32(1 / sqrt(d))
     std::vector<uint32_t> M;    // [d] packed seed-matrix rows
     std::vector<uint32_t> G;    // [DPB_MAX_LEVELS * DPB_MAX_CHILDREN]
+    // VH[k][q][v]: bit l = parity(inv(32 q + l) AND (v << 5k)), the part of the
+    // sign word of a 32-coordinate block that the high half of an index
+    // contributes, per 5-bit chunk k of that half (d <= 1024 only).
+    std::vector<uint32_t> VH;   // [kvh][32][32]
+    int kvh = 0;                // chunks of the high half: ceil(t / 5)
     uint32_t *dM = nullptr;     // device copy of M
     uint32_t *dG = nullptr;     // device copy of G
+    uint32_t *dVH = nullptr;    // device copy of VH
 };
 
 namespace dpb {

@@ -1,0 +1,316 @@
+// dpb_lut.cuh -- table-driven sums of generated parity signs (one warp per
+// token, lane l owning coordinates iota = 32 q + l).
+//
+// The decoder's sum r[iota] = sum_e a_e (-1)^{parity(M[iota] AND c_e)}
+// (§2.1 with App. A.4 Eq. 26) is evaluated 64 codes at a time (a "sweep"):
+//
+//  1. Signs, bit-sliced over codes. Z(iota) is a 64-bit word whose bit e is
+//     the sign bit of code e at coordinate iota. The sign is linear in the
+//     bits of M[iota] = iota | inv(iota) << t (App. A.4 Eq. 22), so
+//       Z(iota) = ZL(iota & 31) ^ ZQ(iota >> 5) ^ XOR_k ZH_k(chunk_k(inv iota)),
+//     each term the XOR of the ballots C_b = {bit b of c_e}_e over the set
+//     bits of its argument: ZL is a register per lane, ZQ one word per block,
+//     ZH_k 32-entry tables indexed by 5-bit chunks of inv(iota).
+//  2. Sums, four Russians style. Each run of 5 codes has a 32-entry table of
+//     all its signed sums sum_j (-1)^{v_j} a_j; the run's 5 sign bits in
+//     Z(iota) index it, so one lookup and one add replace 5 sign-adds. Even
+//     runs are held one entry per lane and read with a shuffle (which uses
+//     only the low 5 bits of its index); odd runs live in shared memory (a
+//     32-word table spans all banks: every lookup is conflict-free). The two
+//     kinds of lookup go down different pipes.
+#pragma once
+
+#include <cstdint>
+
+#include "dpb_device.cuh"
+
+namespace dpb {
+
+constexpr int kMaxKChunks = 4;   // ceil(16 / 5) chunks of inv(iota) for t <= 16
+constexpr int kMaxRuns = 13;     // ceil(64 / 5) runs of 5 codes per sweep
+constexpr int kShflRuns = 7;     // even runs 0, 2, ..., 12
+
+// Shared-memory words of one sweep's tables.
+constexpr int kSweepWords = 2 * 32 /* ZQ (uint2 per block, up to 32 blocks) */ +
+                            2 * 32 * kMaxKChunks /* ZH (uint2 entries) */ +
+                            32 * kShflRuns /* odd runs' value tables */ + 64 /* coefficients */;
+
+struct Sweep {
+    uint2 zl;                 // ZL(lane) for codes 0..31 (x) and 32..63 (y)
+    float vt[kShflRuns];      // lane v holds the table of run 2i at v
+    uint2 *zq;                // [32] (shared)
+    uint2 *zh;                // [kMaxKChunks][32] (shared)
+    float *vto;               // [6][32] odd runs (shared)
+    float *coef;              // [64] (shared)
+    int runs;                 // ceil(codes / 5)
+};
+
+__device__ __forceinline__ Sweep sweep_at(uint32_t *base) {
+    Sweep s;
+    s.zq = reinterpret_cast<uint2 *>(base);
+    s.zh = s.zq + 32;
+    s.vto = reinterpret_cast<float *>(s.zh + 32 * kMaxKChunks);
+    s.coef = s.vto + 32 * (kMaxRuns - kShflRuns);
+    return s;
+}
+
+// Byte offsets (x8, for uint2 tables) of the 5-bit chunks of kappa = inv(iota).
+__device__ __forceinline__ uint32_t kappa_offsets8(uint32_t kappa) {
+    uint32_t off = 0;
+#pragma unroll
+    for (int k = 0; k < kMaxKChunks; ++k) off |= (((kappa >> (5 * k)) & 31u) * 8u) << (8 * k);
+    return off;
+}
+
+// Sign tables of a sweep from its codes (lane holds codes lane and 32 + lane;
+// 0 for empty slots). qn = number of 32-coordinate blocks (<= 32).
+__device__ __forceinline__ void sweep_build_signs(uint32_t ca, uint32_t cb, int t, int qn, Sweep &s) {
+    const int lane = threadIdx.x & 31;
+    uint2 zl = make_uint2(0u, 0u);
+#pragma unroll
+    for (int b = 0; b < 5; ++b) {
+        const uint32_t xa = __ballot_sync(kFull, (ca >> b) & 1u), xb = __ballot_sync(kFull, (cb >> b) & 1u);
+        if ((lane >> b) & 1) {
+            zl.x ^= xa;
+            zl.y ^= xb;
+        }
+    }
+    s.zl = zl;
+    uint32_t qa[5], qb[5];  // iota bits 5..9 are the bits of the block index q
+#pragma unroll
+    for (int b = 0; b < 5; ++b) {
+        const bool live = 5 + b < t;
+        qa[b] = live ? __ballot_sync(kFull, (ca >> (5 + b)) & 1u) : 0u;
+        qb[b] = live ? __ballot_sync(kFull, (cb >> (5 + b)) & 1u) : 0u;
+    }
+    if (lane < qn) {
+        uint2 z = make_uint2(0u, 0u);
+#pragma unroll
+        for (int b = 0; b < 5; ++b)
+            if ((lane >> b) & 1) {
+                z.x ^= qa[b];
+                z.y ^= qb[b];
+            }
+        s.zq[lane] = z;
+    }
+#pragma unroll
+    for (int k = 0; k < kMaxKChunks; ++k) {
+        uint2 acc = make_uint2(0u, 0u);
+#pragma unroll
+        for (int bb = 0; bb < 5; ++bb) {
+            const int b = t + 5 * k + bb;
+            const bool live = b < 2 * t && b < 32;
+            const uint32_t xa = live ? __ballot_sync(kFull, (ca >> b) & 1u) : 0u;
+            const uint32_t xb = live ? __ballot_sync(kFull, (cb >> b) & 1u) : 0u;
+            if ((lane >> bb) & 1) {
+                acc.x ^= xa;
+                acc.y ^= xb;
+            }
+        }
+        s.zh[k * 32 + lane] = acc;
+    }
+}
+
+// Value tables of a sweep from its 64 coefficients (already in s.coef, zero
+// beyond the sweep's codes).
+__device__ __forceinline__ void sweep_build_values(Sweep &s) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int g = 0; g < kMaxRuns; ++g) {
+        float v = 0.f;
+        if (g < s.runs) {
+#pragma unroll
+            for (int j = 0; j < 5; ++j) {
+                const int e = 5 * g + j;
+                const float a = e < 64 ? s.coef[e] : 0.f;
+                v += ((lane >> j) & 1) ? -a : a;
+            }
+        }
+        if (g % 2 == 0)
+            s.vt[g / 2] = v;
+        else
+            s.vto[(g / 2) * 32 + lane] = v;
+    }
+}
+
+// Z(iota) of a sweep; koff = kappa_offsets8(inv iota), zq = ZQ(iota >> 5).
+template <int NKC>
+__device__ __forceinline__ uint2 sweep_signs(const Sweep &s, uint2 zq, uint32_t koff) {
+    const char *zh = reinterpret_cast<const char *>(s.zh);
+    uint2 z = make_uint2(s.zl.x ^ zq.x, s.zl.y ^ zq.y);
+#pragma unroll
+    for (int k = 0; k < NKC; ++k) {
+        const uint2 h = *reinterpret_cast<const uint2 *>(zh + k * 256 + __byte_perm(koff, 0, 0x4440 + k));
+        z.x ^= h.x;
+        z.y ^= h.y;
+    }
+    return z;
+}
+
+// Bits 5G..5G+4 of the 64-bit z in the low bits (high bits unspecified).
+template <int G>
+__device__ __forceinline__ uint32_t run_field(uint2 z) {
+    constexpr int lo = 5 * G;
+    if constexpr (lo + 5 <= 32) {
+        return z.x >> lo;
+    } else if constexpr (lo >= 32) {
+        return z.y >> (lo - 32);
+    } else {
+        return __funnelshift_r(z.x, z.y, lo);
+    }
+}
+
+// The same field times 4 (a byte offset into a 32-float table), G >= 1.
+template <int G>
+__device__ __forceinline__ uint32_t run_offset(uint2 z) {
+    constexpr int lo = 5 * G - 2;
+    uint32_t v;
+    if constexpr (lo + 7 <= 32) {
+        v = z.x >> lo;
+    } else if constexpr (lo >= 32) {
+        v = z.y >> (lo - 32);
+    } else {
+        v = __funnelshift_r(z.x, z.y, lo);
+    }
+    return v & 0x7Cu;
+}
+
+template <int G, int RUNS>
+__device__ __forceinline__ void run_lookups(const Sweep &s, uint2 z, const char *vto, float *p) {
+    if constexpr (G < RUNS) {
+        if constexpr (G % 2 == 0) {
+            p[G] = __shfl_sync(kFull, s.vt[G / 2], run_field<G>(z));
+        } else {
+            p[G] = *reinterpret_cast<const float *>(vto + (G / 2) * 128 + run_offset<G>(z));
+        }
+        run_lookups<G + 1, RUNS>(s, z, vto, p);
+    }
+}
+
+// sum_e coef_e (-1)^{bit e of z} over the sweep's RUNS runs of 5 codes.
+template <int RUNS>
+__device__ __forceinline__ float sweep_sum(const Sweep &s, uint2 z) {
+    float p[RUNS];
+    run_lookups<0, RUNS>(s, z, reinterpret_cast<const char *>(s.vto), p);
+#pragma unroll
+    for (int w = 1; w < RUNS; w *= 2)
+#pragma unroll
+        for (int g = 0; g + w < RUNS; g += 2 * w) p[g] += p[g + w];
+    return p[0];
+}
+
+// Sizes rounded up to 4 words, so that every per-warp array of the kernels'
+// shared-memory layouts starts 16-byte aligned.
+__host__ __device__ constexpr int pad4(int v) { return (v + 3) & ~3; }
+
+// ---- a token's code -----------------------------------------------------------
+
+// Compact list of a token's hashed entries (index >= d).
+struct HashedList {
+    uint32_t *c;    // [k] indices
+    float *a;       // [k] coefficients
+    int *pos;       // [k] position in the code (nullable)
+};
+
+// Adds the basis entries of a token's code (index < d) into `basis` (at
+// their coordinate) and compacts the hashed entries into `hl`; entries
+// outside [0, m_mask] are skipped and flagged. Returns the hashed count.
+__device__ __forceinline__ int split_code(const int32_t *idx, const float *val, int k, int d,
+                                          uint32_t m_mask, float *basis, HashedList &hl,
+                                          int32_t *status) {
+    const int lane = threadIdx.x & 31;
+    int nh = 0;
+    for (int e0 = 0; e0 < k; e0 += 32) {
+        const int e = e0 + lane;
+        int32_t ci = -1;
+        float a = 0.f;
+        if (e < k) {
+            ci = idx[e];
+            a = val[e];
+        }
+        const bool valid = e < k && ci >= 0 && (uint32_t)ci <= m_mask;
+        if (e < k && !valid) set_status(status, DPB_DEV_BAD_INDEX);
+        const bool hashed = valid && ci >= d;
+        if (valid && !hashed && basis) atomicAdd(&basis[ci], a);
+        const unsigned m = __ballot_sync(kFull, hashed);
+        if (hashed) {
+            const int pos = nh + __popc(m & ((1u << lane) - 1u));
+            hl.c[pos] = (uint32_t)ci;
+            hl.a[pos] = a;
+            if (hl.pos) hl.pos[pos] = e;
+        }
+        nh += __popc(m);
+    }
+    __syncwarp();
+    return nh;
+}
+
+// ---- synthesis over a hashed list ---------------------------------------------
+
+// out[i] += scale * sum over one sweep, for every coordinate of the token.
+template <int NKC, int RUNS>
+__device__ __forceinline__ void sweep_accumulate(const Sweep &s, float *out, const uint32_t *koff, int d,
+                                                 float scale) {
+    const int lane = threadIdx.x & 31;
+    const int qn = (d + 31) / 32;
+#pragma unroll 2
+    for (int q = 0; q < qn; ++q) {
+        const int i = 32 * q + lane;
+        const bool in = i < d;
+        const uint2 z = sweep_signs<NKC>(s, s.zq[q], in ? koff[i] : 0u);
+        const float v = sweep_sum<RUNS>(s, z);
+        if (in) out[i] += scale * v;
+    }
+}
+
+template <int NKC>
+__device__ __forceinline__ void sweep_accumulate_runs(const Sweep &s, float *out, const uint32_t *koff,
+                                                      int d, float scale) {
+    switch (s.runs) {
+        case 1: sweep_accumulate<NKC, 1>(s, out, koff, d, scale); break;
+        case 2: sweep_accumulate<NKC, 2>(s, out, koff, d, scale); break;
+        case 3: sweep_accumulate<NKC, 3>(s, out, koff, d, scale); break;
+        case 4: sweep_accumulate<NKC, 4>(s, out, koff, d, scale); break;
+        case 5: sweep_accumulate<NKC, 5>(s, out, koff, d, scale); break;
+        case 6: sweep_accumulate<NKC, 6>(s, out, koff, d, scale); break;
+        case 7: sweep_accumulate<NKC, 7>(s, out, koff, d, scale); break;
+        case 8: sweep_accumulate<NKC, 8>(s, out, koff, d, scale); break;
+        case 9: sweep_accumulate<NKC, 9>(s, out, koff, d, scale); break;
+        case 10: sweep_accumulate<NKC, 10>(s, out, koff, d, scale); break;
+        case 11: sweep_accumulate<NKC, 11>(s, out, koff, d, scale); break;
+        case 12: sweep_accumulate<NKC, 12>(s, out, koff, d, scale); break;
+        default: sweep_accumulate<NKC, 13>(s, out, koff, d, scale); break;
+    }
+}
+
+// out[i] += scale * sum_e coef_e (-1)^{parity(M[i] AND c_e)} over n codes
+// (indices c, coefficients coef), 64 codes per sweep. koff[i] holds the
+// packed chunk offsets of inv(i) (kappa_offsets8).
+template <int NKC>
+__device__ __forceinline__ void synthesise(Sweep &s, const uint32_t *c, const float *coef, int n, int t,
+                                           int d, const uint32_t *koff, float scale, float *out) {
+    const int lane = threadIdx.x & 31;
+    const int qn = (d + 31) / 32;
+    for (int g0 = 0; g0 < n; g0 += 64) {
+        const int m = min(64, n - g0);
+        const uint32_t ca = lane < m ? c[g0 + lane] : 0u;
+        const uint32_t cb = lane + 32 < m ? c[g0 + 32 + lane] : 0u;
+        s.coef[lane] = lane < m ? coef[g0 + lane] : 0.f;
+        s.coef[32 + lane] = lane + 32 < m ? coef[g0 + 32 + lane] : 0.f;
+        sweep_build_signs(ca, cb, t, qn, s);
+        s.runs = (m + 4) / 5;
+        __syncwarp();
+        sweep_build_values(s);
+        __syncwarp();
+        sweep_accumulate_runs<NKC>(s, out, koff, d, scale);
+        __syncwarp();
+    }
+}
+
+// Packed chunk offsets of inv(i) = M[i] >> t for the block's coordinates.
+__device__ __forceinline__ void load_koff(const uint32_t *M, int d, int t, uint32_t *koff) {
+    for (int i = threadIdx.x; i < d; i += blockDim.x) koff[i] = kappa_offsets8(M[i] >> t);
+    __syncthreads();
+}
+
+}  // namespace dpb

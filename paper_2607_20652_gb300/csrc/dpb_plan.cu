@@ -7,6 +7,7 @@
 // primitive element, which give the same unique inverse xi^{2^t-2} of Eq. 25.
 // The seed-matrix row packing is App. A.4 Eq. 22 with the low t bits meeting
 // coord(xi) and the next t bits meeting coord(xi^{-1}).
+#include <algorithm>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -242,6 +243,25 @@ dpb_status resolve_and_build(const dpb_config *in, const uint32_t *generators, d
             for (int m = 0; m < n; ++m) dup |= (row[m] == g);
             if (!dup) row[n++] = g;
         }
+    }
+    // high-half sign tables for the table-driven backward
+    p->kvh = (c.field_t + 4) / 5;
+    // at least two chunks: the kernels for t <= 10 read chunks 0 and 1
+    p->VH.assign((size_t)std::max(p->kvh, 2) * 32 * 32, 0u);
+    if (c.d <= 1024) {
+        for (int k = 0; k < p->kvh; ++k)
+            for (int q = 0; q < 32; ++q)
+                for (int v = 0; v < 32; ++v) {
+                    uint32_t w = 0;
+                    const uint32_t mask = (uint32_t)v << (5 * k);
+                    for (int l = 0; l < 32; ++l) {
+                        const int iota = 32 * q + l;
+                        if (iota >= c.d) continue;
+                        const uint32_t kappa = p->M[iota] >> c.field_t;
+                        w |= (uint32_t)(__builtin_popcount(kappa & mask) & 1) << l;
+                    }
+                    p->VH[((size_t)k * 32 + q) * 32 + v] = w;
+                }
     }
     p->cfg = c;
     p->t = c.field_t;
