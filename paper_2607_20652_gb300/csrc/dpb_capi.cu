@@ -92,23 +92,23 @@ dpb_status dpb_plan_create(const dpb_config *cfg, const uint32_t *generators, dp
         return dpb::fail(DPB_ERR_CUDA, "cudaGetDevice failed");
     }
     const size_t mb = sizeof(uint32_t) * p->M.size(), gb = sizeof(uint32_t) * p->G.size();
-    const size_t vb = sizeof(uint32_t) * p->VH.size();
-    if (cudaMalloc(&p->dM, mb) != cudaSuccess || cudaMalloc(&p->dG, gb) != cudaSuccess ||
-        cudaMalloc(&p->dVH, vb) != cudaSuccess) {
-        cudaFree(p->dM);
-        cudaFree(p->dG);
-        cudaFree(p->dVH);
-        delete p;
-        return dpb::fail(DPB_ERR_NO_MEMORY, "device table allocation failed");
-    }
-    if (cudaMemcpy(p->dM, p->M.data(), mb, cudaMemcpyHostToDevice) != cudaSuccess ||
-        cudaMemcpy(p->dG, p->G.data(), gb, cudaMemcpyHostToDevice) != cudaSuccess ||
-        cudaMemcpy(p->dVH, p->VH.data(), vb, cudaMemcpyHostToDevice) != cudaSuccess) {
-        cudaFree(p->dM);
-        cudaFree(p->dG);
-        cudaFree(p->dVH);
-        delete p;
-        return dpb::fail(DPB_ERR_CUDA, "device table upload failed");
+    struct Up {
+        uint32_t **dst;
+        const std::vector<uint32_t> *src;
+    } ups[] = {{&p->dM, &p->M}, {&p->dG, &p->G}, {&p->dVH, &p->VH}, {&p->dFRAG, &p->FRAG}, {&p->dDD, &p->DD}};
+    for (const Up &u : ups) {
+        if (u.src->empty()) continue;
+        const size_t bytes = sizeof(uint32_t) * u.src->size();
+        if (cudaMalloc(u.dst, bytes) != cudaSuccess) {
+            for (const Up &v : ups) cudaFree(*v.dst);
+            delete p;
+            return dpb::fail(DPB_ERR_NO_MEMORY, "device table allocation failed");
+        }
+        if (cudaMemcpy(*u.dst, u.src->data(), bytes, cudaMemcpyHostToDevice) != cudaSuccess) {
+            for (const Up &v : ups) cudaFree(*v.dst);
+            delete p;
+            return dpb::fail(DPB_ERR_CUDA, "device table upload failed");
+        }
     }
     *out = p;
     return DPB_OK;
@@ -126,6 +126,8 @@ dpb_status dpb_plan_destroy(dpb_plan *plan) {
     cudaFree(plan->dM);
     cudaFree(plan->dG);
     cudaFree(plan->dVH);
+    cudaFree(plan->dFRAG);
+    cudaFree(plan->dDD);
     if (cur >= 0 && cur != plan->device) cudaSetDevice(cur);
     delete plan;
     return DPB_OK;

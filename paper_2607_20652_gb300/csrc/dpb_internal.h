@@ -24,12 +24,40 @@ struct dpb_plan {
     // contributes, per 5-bit chunk k of that half (d <= 1024 only).
     std::vector<uint32_t> VH;   // [kvh][32][32]
     int kvh = 0;                // chunks of the high half: ceil(t / 5)
+    // Tensor-core encoder tables (built when mma_encode is set):
+    //  FRAG[l-1][m][lane][8]: the generator signs gamma_j of level l over
+    //    32-coordinate block m, as bf16 +-1 pairs in mma.sync B-fragment order;
+    //  DD[l-1][kDedupSlots][2]: open-addressing table of the differences
+    //    g_j ^ g_j' (j != j') of level l, value (j | j' << 8), key + 1 (0 = empty).
+    bool mma_encode = false;
+    std::vector<uint32_t> FRAG;
+    std::vector<uint32_t> DD;
     uint32_t *dM = nullptr;     // device copy of M
     uint32_t *dG = nullptr;     // device copy of G
     uint32_t *dVH = nullptr;    // device copy of VH
+    uint32_t *dFRAG = nullptr;  // device copy of FRAG
+    uint32_t *dDD = nullptr;    // device copy of DD
 };
 
 namespace dpb {
+
+constexpr int kDedupSlots = 512;
+
+__host__ __device__ inline uint32_t dedup_hash(uint32_t delta) {
+    return (delta * 2654435761u) >> (32 - 9);
+}
+
+// The K-permuted coordinate of pair slot `pair` (0..3), half `half` (0..1) of
+// lane quarter q4 in a 32-coordinate block: the tensor-core encoder gives the
+// lane with q4 = lane % 4 the coordinates q4 + 4 j (j < 8), paired (j, j + 4).
+__host__ __device__ inline int frag_coord(int q4, int pair, int half) { return q4 + 4 * (pair + 4 * half); }
+
+// Builds the tensor-core encoder tables when the plan qualifies (dpb_plan.cu).
+void build_mma_tables(dpb_plan *p);
+
+// Dynamic shared memory (bytes) of the tensor-core encoder for this plan.
+size_t encode_mma_smem(const dpb_plan *p);
+constexpr size_t kMaxSmemPerBlock = 227 * 1024;
 
 // Records a message for dpb_last_error() and returns `s`.
 dpb_status fail(dpb_status s, const char *fmt, ...);
@@ -38,6 +66,9 @@ dpb_status fail(dpb_status s, const char *fmt, ...);
 dpb_status resolve_and_build(const dpb_config *in, const uint32_t *generators, dpb_plan *p);
 
 // Kernel launchers (return cudaGetLastError() of the launch).
+cudaError_t launch_encode_mma(const dpb_plan *p, const void *x, int64_t T, const float *mu,
+                              const float *sigma, int32_t *idx, float *val, float *xnorm,
+                              int32_t *status, cudaStream_t stream);
 cudaError_t launch_encode(const dpb_plan *p, const void *x, int64_t T, const float *mu,
                           const float *sigma, int32_t *idx, float *val, float *xnorm,
                           int32_t *status, cudaStream_t stream);

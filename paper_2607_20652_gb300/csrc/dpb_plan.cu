@@ -149,6 +149,46 @@ int ceil_log2(int v) {
 
 }  // namespace
 
+void build_mma_tables(dpb_plan *p) {
+    const dpb_config &c = p->cfg;
+    bool ok = c.dtype == DPB_BF16 && c.d % 32 == 0 && c.d >= 32 && c.d <= 1024 && c.levels >= 2 &&
+              c.select_mode == DPB_SELECT_GLOBAL && c.beam == 8 && c.k >= c.beam && c.k <= 256;
+    for (int l = 1; l < c.levels && ok; ++l) ok = c.children[l] == 16;
+    const int nblk = c.d / 32;
+    // every level's fragments, the tables and the warps' pools share one block
+    if (ok && encode_mma_smem(p) > kMaxSmemPerBlock) ok = false;
+    p->mma_encode = ok;
+    if (!ok) return;
+    p->FRAG.assign((size_t)(c.levels - 1) * nblk * 256, 0u);
+    auto sign_bf16 = [&](uint32_t g, int iota) -> uint32_t {
+        return (__builtin_popcount(p->M[iota] & g) & 1) ? 0xBF80u : 0x3F80u;
+    };
+    for (int l = 1; l < c.levels; ++l)
+        for (int m = 0; m < nblk; ++m)
+            for (int lane = 0; lane < 32; ++lane)
+                for (int w = 0; w < 8; ++w) {
+                    const int chunk = w / 4, half = (w / 2) % 2, reg = w % 2;
+                    const int n = 8 * half + lane / 4, q4 = lane % 4, pair = 2 * chunk + reg;
+                    const uint32_t g = p->G[(size_t)l * DPB_MAX_CHILDREN + n];
+                    const int ia = 32 * m + frag_coord(q4, pair, 0), ib = 32 * m + frag_coord(q4, pair, 1);
+                    p->FRAG[(((size_t)(l - 1) * nblk + m) * 32 + lane) * 8 + w] = sign_bf16(g, ia) | (sign_bf16(g, ib) << 16);
+                }
+    p->DD.assign((size_t)(c.levels - 1) * kDedupSlots * 2, 0u);
+    for (int l = 1; l < c.levels; ++l) {
+        uint32_t *tab = &p->DD[(size_t)(l - 1) * kDedupSlots * 2];
+        const uint32_t *g = &p->G[(size_t)l * DPB_MAX_CHILDREN];
+        for (int j = 0; j < 16; ++j)
+            for (int jj = 0; jj < 16; ++jj) {
+                if (j == jj) continue;
+                const uint32_t delta = g[j] ^ g[jj];
+                uint32_t h = dedup_hash(delta);
+                while (tab[2 * h] != 0) h = (h + 1) & (kDedupSlots - 1);
+                tab[2 * h] = delta + 1;
+                tab[2 * h + 1] = (uint32_t)j | ((uint32_t)jj << 8);
+            }
+    }
+}
+
 dpb_status fail(dpb_status s, const char *fmt, ...) {
     va_list ap;
     va_start(ap, fmt);
@@ -264,6 +304,7 @@ dpb_status resolve_and_build(const dpb_config *in, const uint32_t *generators, d
                 }
     }
     p->cfg = c;
+    build_mma_tables(p);
     p->t = c.field_t;
     p->poly = c.field_poly;
     p->m_mask = (N >= 32) ? 0xffffffffu : ((1u << N) - 1u);
