@@ -1,0 +1,738 @@
+// dpb_encode_mma.cuh -- the §2.2 encoder with the child scoring of Eq. 6 on the
+// tensor cores (bf16 inputs, beam 8, 16 children per parent). Instantiated
+// per count of inverse-coordinate sign tables (dpb_encode_mma_n*.cu).
+//
+// Scoring. A warp owns two tokens at a time. At level l its 16 tensor-core
+// rows are the (token, beam slot) pairs and the contraction is
+//     score[row][j] = sum_iota (x_token (.) phi~_parent)[iota] * gamma_j[iota],
+// rows x (.) phi~_p times the universal matrix Gamma_l (Eq. 6), by mma.sync
+// m16n8k16 (bf16 x bf16 -> fp32). The A operand is never staged: each lane
+// builds its fragment in registers as the bf16 bits of x XOR a sign mask. The
+// K order is permuted so that the lane with q4 = lane % 4 holds coordinates
+// q4 + 4j of every 32-coordinate block, paired (j, j+4): the two sign bits of
+// a pair sit 16 apart in the parent's sign word over the block, and one shift
+// moves both to the bf16 sign positions 15 and 31. The sign word of parent p
+// over block m is
+//     W5[p & 31] ^ PQ[m][(p_lo >> 5) & 31] ^ XOR_k VH_k[m][chunk_k(p_hi)],
+// the Walsh, block-parity and inverse-coordinate parts of parity(M[iota] & p)
+// (App. A.4 Eq. 26). Gamma_l lives in shared memory in B-fragment order.
+//
+// Selection (global mode, readings R8-R10). Every candidate is one 64-bit
+// word, |z| bits above (2^31 - 1 - index) and the sign of z, so that larger
+// words come first in the order (|z| descending, index ascending). Each token
+// keeps its code as a sorted list of k words in shared memory:
+//   level 0  the exact top k of the d coordinates: each lane keeps its best R
+//            32-bit words (|x| bf16 bits, index, sign), the warp sorts the
+//            union of 32 R and takes its k-th word tau; if exactly k
+//            coordinates reach tau the union's first k are the top k
+//            (otherwise, and with standardisation, a bisection path);
+//   level l  the distinct children ahead of the list's k-th word are merged
+//            in by rank (each entrant's place = entrants ahead of it + list
+//            words ahead of it); the beam is the first 8 children, read from
+//            those ranks, or from a warp tournament when fewer than 8 or more
+//            than 32 children enter.
+// The list after the last level is the code.
+#pragma once
+
+#include <algorithm>
+
+#include "dpb_device.cuh"
+#include "dpb_internal.h"
+#include "dpb_select.cuh"
+
+namespace dpb {
+namespace mmaenc {
+
+constexpr int kMaxWarps = 16;
+constexpr int kBeam = 8;
+
+struct Args {
+    const __nv_bfloat16 *x;
+    int64_t T;
+    const float *mu, *sigma;
+    int32_t *idx;
+    float *val, *xnorm;
+    int32_t *status;
+    const uint32_t *frag, *G, *VH, *DD;
+    int d, nblk, levels, k, t, ecap;
+    float inv_sqrt_d;
+};
+
+// ---- shared-memory layout (32-bit words) ------------------------------------------
+
+__host__ __device__ inline int block_words(int levels, int nblk, int nkc) {
+    // frag [(L-1)][nblk][32][8], W5 [32], PQ [32][32], VH [nkc][32][32],
+    // DD [(L-1)][kDedupSlots][2], G [L][16]
+    return (levels - 1) * nblk * 256 + 32 + 1024 + nkc * 1024 + (levels - 1) * kDedupSlots * 2 + 8 * 16;
+}
+
+// 64-bit entries of the per-warp scratch buffer: the entrants of a merge, the
+// lists of the bisection path, and the parents' sign words of a level
+// (16 rows x nblk blocks).
+__host__ __device__ inline int entrant_cap(int k, int nblk) {
+    int c = 128;
+    while (c < k) c <<= 1;
+    return c > 8 * nblk ? c : 8 * nblk;
+}
+
+__host__ __device__ inline int warp_words(int nblk, int k) {
+    // x tile [2][nblk * 16], code lists [2][k] (64-bit), scratch [ecap]
+    // (64-bit), beams [2][8], duplicate bits [8], spare [8]
+    return 2 * nblk * 16 + 4 * k + 2 * entrant_cap(k, nblk) + 16 + 8 + 8;
+}
+
+// ---- candidate words ------------------------------------------------------------------
+
+__device__ __forceinline__ uint64_t cword(float z, uint32_t idx) {
+    const uint32_t b = __float_as_uint(z);
+    return ((uint64_t)(b & 0x7fffffffu) << 32) | ((uint64_t)(0x7fffffffu - idx) << 1) | (b >> 31);
+}
+__device__ __forceinline__ uint32_t cword_idx(uint64_t c) { return 0x7fffffffu - ((uint32_t)c >> 1); }
+__device__ __forceinline__ float cword_z(uint64_t c) {
+    return __uint_as_float((uint32_t)(c >> 32) | ((uint32_t)c << 31));
+}
+
+// Level-0 word of bf16 coordinate i (< 2^15) with bits b: the same order in 32 bits.
+__device__ __forceinline__ uint32_t cword0(uint32_t b, uint32_t i) {
+    return ((b & 0x7fffu) << 16) | ((0x7fffu - i) << 1) | ((b >> 15) & 1u);
+}
+__device__ __forceinline__ uint64_t widen0(uint32_t c) {
+    const uint32_t i = 0x7fffu - ((c >> 1) & 0x7fffu);
+    return ((uint64_t)((c >> 16) << 16) << 32) | ((uint64_t)(0x7fffffffu - i) << 1) | (c & 1u);
+}
+
+// ---- helpers ----------------------------------------------------------------------
+
+__device__ __forceinline__ void mma_bf16(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                         uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+        "{%0,%1,%2,%3};\n"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// Byte offsets of parent p into PQ[m] and VH_k[m], packed four to a word.
+struct ParentOff {
+    uint32_t w5;  // the Walsh word (the same for every block)
+    uint32_t o;   // PQ, VH_0, VH_1, VH_2 byte offsets
+    uint32_t o3;  // VH_3 byte offset
+};
+
+__device__ __forceinline__ ParentOff parent_offsets(uint32_t p, int t, const uint32_t *w5) {
+    ParentOff po;
+    po.w5 = w5[p & 31u];  // t >= 5: bits 0..4 belong to p_lo
+    const uint32_t b1 = (((p & ((1u << t) - 1u)) >> 5) & 31u) * 4u;
+    const uint32_t h0 = ((p >> t) & 31u) * 4u, h1 = ((p >> (t + 5)) & 31u) * 4u;
+    const uint32_t h2 = ((p >> min(t + 10, 31)) & 31u) * 4u;
+    const uint32_t h3 = ((p >> min(t + 15, 31)) & 31u) * 4u;
+    po.o = b1 | (h0 << 8) | (h1 << 16) | (h2 << 24);
+    po.o3 = h3;
+    return po;
+}
+
+// Sign word of a parent over 32-coordinate block m (bit l = 1: coordinate
+// 32 m + l of phi~_p is negative).
+template <int NKC>
+__device__ __forceinline__ uint32_t parent_signs(const ParentOff &po, const uint32_t *pq, const uint32_t *vh, int m) {
+    const char *P = reinterpret_cast<const char *>(pq + m * 32);
+    const char *V = reinterpret_cast<const char *>(vh + m * 32);
+    uint32_t s = po.w5 ^ *reinterpret_cast<const uint32_t *>(P + __byte_perm(po.o, 0, 0x4440)) ^
+                 *reinterpret_cast<const uint32_t *>(V + __byte_perm(po.o, 0, 0x4441));
+    s ^= *reinterpret_cast<const uint32_t *>(V + 4096 + __byte_perm(po.o, 0, 0x4442));
+    if (NKC > 2) s ^= *reinterpret_cast<const uint32_t *>(V + 8192 + __byte_perm(po.o, 0, 0x4443));
+    if (NKC > 3) s ^= *reinterpret_cast<const uint32_t *>(V + 12288 + po.o3);
+    return s;
+}
+
+// Coordinate i of one token's row, read back from the permuted tile.
+__device__ __forceinline__ float x_at(const uint16_t *xh, int i) {
+    const int m = i >> 5, l = i & 31;
+    return __uint_as_float((uint32_t)xh[(m * 16 + (l & 3) * 4 + ((l >> 2) & 3)) * 2 + (l >> 4)] << 16);
+}
+
+// z = (s - mu_c) / sigma_c (§2.2 score standardisation); identity without tables.
+__device__ __forceinline__ float standardise(float s, uint32_t c, const float *mu, const float *sigma,
+                                             int32_t *status) {
+    if (!mu) return s;
+    const float sd = sigma[c];
+    if (status && !(sd > 0.f)) set_status(status, DPB_DEV_BAD_SIGMA);
+    return (s - mu[c]) / sd;
+}
+
+// bf16 element e (0..7) of a 16-byte chunk.
+__device__ __forceinline__ uint32_t elem16(const uint4 &v, int e) {
+    const uint32_t w = (e >> 1) == 0 ? v.x : (e >> 1) == 1 ? v.y : (e >> 1) == 2 ? v.z : v.w;
+    return (w >> (16 * (e & 1))) & 0xffffu;
+}
+
+__device__ __forceinline__ unsigned lanes_below() { return (1u << (threadIdx.x & 31)) - 1u; }
+
+// Appends the lane-distributed (z, id) entries with `take` set to a shared list
+// at position n; returns the new length (warp-uniform).
+__device__ __forceinline__ int warp_append(float *z, uint32_t *id, int n, bool take, float zv, uint32_t iv) {
+    const unsigned mb = __ballot_sync(kFull, take);
+    if (take) {
+        const int pos = n + __popc(mb & lanes_below());
+        z[pos] = zv;
+        id[pos] = iv;
+    }
+    return n + __popc(mb);
+}
+
+// Warp bitonic sort, descending, of 32 R words held R per lane (element
+// lane * R + r).
+template <int R>
+__device__ __forceinline__ void warp_sort_desc(uint32_t (&v)[R]) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int size = 2; size <= 32 * R; size <<= 1) {
+#pragma unroll
+        for (int stride = size / 2; stride > 0; stride >>= 1) {
+            if (stride >= R) {
+                const bool lower = (lane & (stride / R)) == 0;
+#pragma unroll
+                for (int r = 0; r < R; ++r) {
+                    const bool desc = (((lane * R + r) & size) == 0);
+                    const uint32_t o = __shfl_xor_sync(kFull, v[r], stride / R);
+                    v[r] = (lower == desc) ? max(v[r], o) : min(v[r], o);
+                }
+            } else {
+#pragma unroll
+                for (int r = 0; r < R; ++r) {
+                    const int q = r ^ stride;
+                    if (q > r) {
+                        const bool desc = (((lane * R + r) & size) == 0);
+                        const uint32_t hi = max(v[r], v[q]), lo = min(v[r], v[q]);
+                        v[r] = desc ? hi : lo;
+                        v[q] = desc ? lo : hi;
+                    }
+                }
+            }
+        }
+    }
+}
+
+__device__ __forceinline__ void cas_desc(uint64_t &a, uint64_t &b) {
+    const uint64_t hi = a > b ? a : b, lo = a > b ? b : a;
+    a = hi;
+    b = lo;
+}
+
+// The first kBeam of up to 128 distinct candidate words held 4 per lane (0 =
+// none), by kBeam rounds of a warp tournament over the lanes' sorted heads.
+__device__ __forceinline__ void beam_tournament(uint64_t (&c)[4], uint32_t *beam) {
+    cas_desc(c[0], c[1]);
+    cas_desc(c[2], c[3]);
+    cas_desc(c[0], c[2]);
+    cas_desc(c[1], c[3]);
+    cas_desc(c[1], c[2]);
+#pragma unroll 1
+    for (int r = 0; r < kBeam; ++r) {
+        const uint32_t hi = (uint32_t)(c[0] >> 32), lo = (uint32_t)c[0];
+        const uint32_t mh = __reduce_max_sync(kFull, hi);
+        const uint32_t ml = __reduce_max_sync(kFull, hi == mh ? lo : 0u);
+        if (hi == mh && lo == ml && (mh | ml) != 0u) {
+            beam[r] = cword_idx(c[0]);
+            c[0] = c[1];
+            c[1] = c[2];
+            c[2] = c[3];
+            c[3] = 0ull;
+        }
+    }
+    __syncwarp();
+}
+
+// ---- merging entrants into a code list -------------------------------------------
+
+// Merges the m entrant words E[0..m) (each ahead of L[k-1], any order) into
+// the sorted list L of k words, 32 entrants at a time: an entrant's place is
+// the entrants of its chunk ahead of it plus the list words ahead of it (a
+// prefix of L, found by bisection); a list word moves down by the entrants
+// ahead of it; whatever lands at k or beyond drops out. When 8..32 words enter
+// and `beam` is given, the first 8 entrants become the beam.
+template <int KPL>
+__device__ __forceinline__ void merge_sorted(uint64_t *L, int k, const uint64_t *E, int m, uint32_t *beam) {
+    const int lane = threadIdx.x & 31;
+    int top = 1;
+    while (2 * top <= k) top <<= 1;
+    for (int q0 = 0; q0 < m; q0 += 32) {
+        const int mq = min(32, m - q0);
+        const uint64_t mine = lane < mq ? E[q0 + lane] : 0ull;
+        uint64_t lv[KPL];
+        int rl[KPL];
+#pragma unroll
+        for (int r = 0; r < KPL; ++r) {
+            const int e = lane + 32 * r;
+            lv[r] = e < k ? L[e] : 0ull;
+            rl[r] = 0;
+        }
+        int rs = 0;  // entrants of this chunk ahead of mine
+        for (int i = 0; i < mq; ++i) {
+            const uint64_t s = E[q0 + i];
+            rs += s > mine;
+#pragma unroll
+            for (int r = 0; r < KPL; ++r) rl[r] += s > lv[r];
+        }
+        int pos = 0;  // list words ahead of mine
+        for (int step = top; step > 0; step >>= 1) {
+            const int np = pos + step;
+            if (np <= k && L[np - 1] > mine) pos = np;
+        }
+        __syncwarp();
+        if (lane < mq && rs + pos < k) L[rs + pos] = mine;
+#pragma unroll
+        for (int r = 0; r < KPL; ++r) {
+            const int e = lane + 32 * r;
+            if (e < k && e + rl[r] < k) L[e + rl[r]] = lv[r];
+        }
+        if (beam && m >= kBeam && m <= 32 && lane < mq && rs < kBeam) beam[rs] = cword_idx(mine);
+        __syncwarp();
+    }
+}
+
+// Gathers the candidate words c[] (4 per lane, 0 = none) that are ahead of the
+// list's k-th word into E (capacity >= 128) and merges them into L. Returns
+// the number of entrants.
+template <int KPL>
+__device__ __forceinline__ int merge_entrants(uint64_t *L, int k, uint64_t *E, const uint64_t (&c)[4],
+                                              uint32_t *beam) {
+    const uint64_t tau = L[k - 1];
+    int m = 0;
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        const bool take = c[e] > tau;
+        const unsigned mb = __ballot_sync(kFull, take);
+        if (take) E[m + __popc(mb & lanes_below())] = c[e];
+        m += __popc(mb);
+    }
+    __syncwarp();
+    merge_sorted<KPL>(L, k, E, m, beam);
+    return m;
+}
+
+// ---- level 0 ----------------------------------------------------------------------
+
+// Fast path (no standardisation, k <= 16 R): see the header comment. `wv`
+// holds the words of this lane's coordinates (16-byte chunk lane + 32 j,
+// element e; 0 where the chunk lies past the row). The union's first k go to
+// the list; coordinates that reach its k-th word without being among their
+// lane's R kept words are merged in afterwards. Returns false, with nothing
+// written, when more of them arrive than the scratch holds.
+template <int R, int KPL>
+__device__ __forceinline__ bool level0_union(const uint32_t (&wv)[4][8], int nch, int k, uint64_t *E, int ecap,
+                                             uint64_t *L, uint32_t *beam) {
+    const int lane = threadIdx.x & 31;
+    uint32_t top[R];
+#pragma unroll
+    for (int r = 0; r < R; ++r) top[r] = 0u;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        if (lane + 32 * j < nch) {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                uint32_t c = wv[j][e];
+#pragma unroll
+                for (int r = 0; r < R; ++r) {
+                    const uint32_t hi = max(top[r], c);
+                    c = min(top[r], c);
+                    top[r] = hi;
+                }
+            }
+        }
+    }
+    const uint32_t kept_min = top[R - 1];  // every word of this lane below it was not kept
+    warp_sort_desc<R>(top);
+    uint32_t mine = 0u;
+#pragma unroll
+    for (int r = 0; r < R; ++r)
+        if (r == (k - 1) % R) mine = top[r];
+    const uint32_t tau = __shfl_sync(kFull, mine, (k - 1) / R);
+    int nx = 0;
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+        if (lane + 32 * j < nch)
+#pragma unroll
+            for (int e = 0; e < 8; ++e) nx += (wv[j][e] >= tau) & (wv[j][e] < kept_min);
+    const int total = __reduce_add_sync(kFull, nx);
+    if (total > ecap) return false;
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+        const int e = lane * R + r;
+        if (e < k) L[e] = widen0(top[r]);
+    }
+    if (total > 0) {
+        int off = nx;  // exclusive prefix of the extras over the lanes
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int v = __shfl_up_sync(kFull, off, o);
+            if (lane >= o) off += v;
+        }
+        off -= nx;
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+            if (lane + 32 * j < nch)
+#pragma unroll
+                for (int e = 0; e < 8; ++e)
+                    if (wv[j][e] >= tau && wv[j][e] < kept_min) E[off++] = widen0(wv[j][e]);
+        __syncwarp();
+        merge_sorted<KPL>(L, k, E, total, nullptr);
+        if (lane < kBeam) beam[lane] = cword_idx(L[lane]);
+    } else {
+#pragma unroll
+        for (int r = 0; r < R; ++r)
+            if (lane * R + r < kBeam) beam[lane * R + r] = 0x7fffu - ((top[r] >> 1) & 0x7fffu);
+    }
+    __syncwarp();
+    return true;
+}
+
+// General path: every coordinate (standardised if tables are given) is a
+// candidate; a per-lane threshold keeps at least k of them in the scratch
+// (z, id) lists of capacity `cap`, the k-th is found by bisection, and the
+// first k, sorted, become the code list; its first 8 are the beam.
+__device__ __forceinline__ void level0_bisect(const Args &a, const uint16_t *xh, float *pz, uint32_t *pid, int cap,
+                                              uint64_t *L, uint32_t *beam) {
+    const int lane = threadIdx.x & 31, d = a.d, k = a.k;
+    const int lowbit = a.mu ? 0 : 16;  // keys of unstandardised bf16 values have 16 zero bits
+    // Each lane's R-th best key: at least 32 R >= k candidates are at or above
+    // the smallest of them.
+    const int R = (k + 31) >> 5;
+    uint32_t best[8];
+#pragma unroll
+    for (int r = 0; r < 8; ++r) best[r] = 0u;
+    for (int i = lane; i < d; i += 32) {
+        uint32_t kv = akey(standardise(x_at(xh, i), (uint32_t)i, a.mu, a.sigma, a.status)) + 1u;
+#pragma unroll
+        for (int r = 0; r < 8; ++r) {
+            if (r < R && kv > best[r]) {
+                const uint32_t tmp = best[r];
+                best[r] = kv;
+                kv = tmp;
+            }
+        }
+    }
+    uint32_t mine = 0;
+#pragma unroll
+    for (int r = 0; r < 8; ++r)
+        if (r == R - 1) mine = best[r];
+    const uint32_t tau_low = __reduce_min_sync(kFull, mine);
+    int n = 0;
+    bool overflow = false;
+    for (int i0 = 0; i0 < d && !overflow; i0 += 32) {
+        const int i = i0 + lane;
+        float z = 0.f;
+        bool take = false;
+        if (i < d) {
+            z = standardise(x_at(xh, i), (uint32_t)i, a.mu, a.sigma, nullptr);
+            take = akey(z) + 1u >= tau_low;
+        }
+        if (n + __popc(__ballot_sync(kFull, take)) > cap) {
+            overflow = true;  // many equal keys at the threshold
+        } else {
+            n = warp_append(pz, pid, n, take, z, (uint32_t)i);
+        }
+    }
+    __syncwarp();
+    if (overflow) {
+        // exact k-th key over the whole row, then every entry above it and the
+        // first ties by index
+        uint32_t tau = 0;
+        for (int b = 30; b >= lowbit; --b) {
+            const uint32_t c = tau | (1u << b);
+            int cnt = 0;
+            for (int i = lane; i < d; i += 32)
+                cnt += akey(standardise(x_at(xh, i), (uint32_t)i, a.mu, a.sigma, nullptr)) >= c;
+            if (__reduce_add_sync(kFull, cnt) >= k) tau = c;
+        }
+        n = 0;
+        for (int i0 = 0; i0 < d; i0 += 32) {
+            const int i = i0 + lane;
+            float z = 0.f;
+            if (i < d) z = standardise(x_at(xh, i), (uint32_t)i, a.mu, a.sigma, nullptr);
+            n = warp_append(pz, pid, n, i < d && akey(z) > tau, z, (uint32_t)i);
+        }
+        for (int i0 = 0; i0 < d && n < k; i0 += 32) {
+            const int i = i0 + lane;
+            float z = 0.f;
+            bool tie = false;
+            if (i < d) {
+                z = standardise(x_at(xh, i), (uint32_t)i, a.mu, a.sigma, nullptr);
+                tie = akey(z) == tau;
+            }
+            const unsigned mb = __ballot_sync(kFull, tie);
+            const int rank = __popc(mb & lanes_below());
+            if (tie && n + rank < k) {
+                pz[n + rank] = z;
+                pid[n + rank] = (uint32_t)i;
+            }
+            n = min(k, n + __popc(mb));
+        }
+        __syncwarp();
+    }
+    uint32_t tk, ti;
+    warp_kth(pz, pid, n, k, lowbit, tk, ti);
+    n = warp_compact_keep(pz, pid, n, tk, ti);
+    int sc = 32;
+    while (sc < n) sc <<= 1;
+    warp_sort(pz, pid, n, sc);
+    for (int e = lane; e < k; e += 32) L[e] = cword(pz[e], pid[e]);
+    if (lane < kBeam) beam[lane] = pid[lane];
+    __syncwarp();
+}
+
+// ---- the kernel ---------------------------------------------------------------------
+
+template <int NKC, int KPL>
+__global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
+    extern __shared__ __align__(16) uint32_t smem[];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+    const int d = a.d, nblk = a.nblk, L = a.levels, k = a.k, t = a.t;
+    const int q4 = lane & 3, slot = lane >> 2;
+
+    uint32_t *s_frag = smem;
+    uint32_t *s_w5 = s_frag + (L - 1) * nblk * 256;
+    uint32_t *s_pq = s_w5 + 32;
+    uint32_t *s_vh = s_pq + 1024;
+    uint32_t *s_dd = s_vh + NKC * 1024;
+    uint32_t *s_g = s_dd + (L - 1) * kDedupSlots * 2;
+    {
+        const uint4 *src = reinterpret_cast<const uint4 *>(a.frag);
+        uint4 *dst = reinterpret_cast<uint4 *>(s_frag);
+        for (int i = threadIdx.x; i < (L - 1) * nblk * 64; i += blockDim.x) dst[i] = src[i];
+        for (int v = threadIdx.x; v < 32; v += blockDim.x) {
+            uint32_t word = 0;
+            for (int l = 0; l < 32; ++l) word |= (uint32_t)(__popc(l & v) & 1) << l;
+            s_w5[v] = word;
+        }
+        for (int i = threadIdx.x; i < 1024; i += blockDim.x) s_pq[i] = (__popc((i >> 5) & i & 31) & 1) ? ~0u : 0u;
+        for (int i = threadIdx.x; i < NKC * 1024; i += blockDim.x) s_vh[i] = a.VH[i];
+        for (int i = threadIdx.x; i < (L - 1) * kDedupSlots * 2; i += blockDim.x) s_dd[i] = a.DD[i];
+        for (int i = threadIdx.x; i < L * 16; i += blockDim.x) s_g[i] = a.G[(i >> 4) * DPB_MAX_CHILDREN + (i & 15)];
+    }
+    __syncthreads();
+
+    uint32_t *xt = smem + block_words(L, nblk, NKC) + warp * warp_words(nblk, k);
+    uint64_t *codes = reinterpret_cast<uint64_t *>(xt + 2 * nblk * 16);  // [2][k]
+    uint64_t *E = codes + 2 * k;                                          // [ecap]
+    uint32_t *beams = reinterpret_cast<uint32_t *>(E + a.ecap);           // [2][8]
+    uint32_t *dup = beams + 16;                                           // [4]
+    uint16_t *xh = reinterpret_cast<uint16_t *>(xt);
+    const int nch = d / 8;  // 16-byte chunks of a row
+    // the lane-th slot pair (sp, s), sp < s, of the beam
+    const int ps = 1 + (lane >= 1) + (lane >= 3) + (lane >= 6) + (lane >= 10) + (lane >= 15) + (lane >= 21);
+    const int psp = lane - ps * (ps - 1) / 2;
+    const int64_t npairs = (a.T + 1) / 2;
+
+    for (int64_t pr = (int64_t)blockIdx.x * nwarps + warp; pr < npairs; pr += (int64_t)gridDim.x * nwarps) {
+        const int64_t t0 = 2 * pr;
+        const int ntok = t0 + 1 < a.T ? 2 : 1;
+
+        // ---- each row into the permuted tile; |x|; level 0 ----
+        for (int tk = 0; tk < ntok; ++tk) {
+            const uint4 *row = reinterpret_cast<const uint4 *>(a.x + (t0 + tk) * d);
+            uint32_t wv[4][8];  // level-0 words of this lane's coordinates
+            float ss = 0.f;
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const int ch = lane + 32 * j;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) wv[j][e] = 0u;
+                if (ch < nch) {
+                    const uint4 v = row[ch];
+                    const int m = ch >> 2, l0 = (ch & 3) * 8, half = l0 >> 4, pb = (l0 & 15) >> 2;
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        const uint32_t bits = elem16(v, e);
+                        xh[(tk * nblk * 16 + m * 16 + (e & 3) * 4 + pb + (e >> 2)) * 2 + half] = (uint16_t)bits;
+                        const float xf = __uint_as_float(bits << 16);
+                        ss = fmaf(xf, xf, ss);
+                        wv[j][e] = cword0(bits, (uint32_t)(8 * ch + e));
+                    }
+                }
+            }
+            ss = warp_sum(ss);
+            if (lane == 0 && a.xnorm) a.xnorm[t0 + tk] = sqrtf(ss);
+            __syncwarp();
+            uint64_t *Lt = codes + tk * k;
+            uint32_t *bt = beams + tk * kBeam;
+            bool done = false;
+            if (!a.mu && KPL <= 4) done = level0_union<(KPL <= 2 ? 4 : 8), KPL>(wv, nch, k, E, a.ecap, Lt, bt);
+            if (!done)
+                level0_bisect(a, xh + tk * nblk * 32, reinterpret_cast<float *>(E),
+                              reinterpret_cast<uint32_t *>(E) + a.ecap, a.ecap, Lt, bt);
+        }
+
+        // ---- levels 1 .. L-1 ----
+        for (int l = 1; l < L; ++l) {
+            const uint32_t *frag = s_frag + (l - 1) * nblk * 256;
+            // this lane's tensor-core rows: (token 0, slot) and (token 1, slot)
+            const uint32_t p0 = beams[slot];
+            const uint32_t p1 = ntok > 1 ? beams[kBeam + slot] : 0u;
+            // sign words of the 16 rows' parents over every block, row 2 slot + token
+            uint2 *sgn = reinterpret_cast<uint2 *>(E);  // [nblk][8] (token 0, token 1)
+            {
+                const int row = lane & 15;
+                const uint32_t pr = (row & 1) && ntok < 2 ? 0u : beams[(row & 1) * kBeam + (row >> 1)];
+                const ParentOff po = parent_offsets(pr, t, s_w5);
+                uint32_t *sw = reinterpret_cast<uint32_t *>(E);
+                for (int m = lane >> 4; m < nblk; m += 2) sw[m * 16 + row] = parent_signs<NKC>(po, s_pq, s_vh, m);
+            }
+            __syncwarp();
+            float acc[2][2][2][4];  // [m & 1][chunk][n-half][reg]
+#pragma unroll
+            for (int u = 0; u < 2; ++u)
+#pragma unroll
+                for (int c = 0; c < 2; ++c)
+#pragma unroll
+                    for (int h = 0; h < 2; ++h)
+#pragma unroll
+                        for (int r = 0; r < 4; ++r) acc[u][c][h][r] = 0.f;
+            const uint4 *xa = reinterpret_cast<const uint4 *>(xt) + q4;
+            const uint4 *xb = reinterpret_cast<const uint4 *>(xt + nblk * 16) + q4;
+            const uint4 *fr = reinterpret_cast<const uint4 *>(frag) + lane * 2;
+            const int sh = 15 - q4;
+#pragma unroll 2
+            for (int m = 0; m < nblk; ++m) {
+                const uint4 va = xa[m * 4], vb = xb[m * 4];
+                const uint2 sg = sgn[m * 8 + slot];
+                const uint32_t s0 = sg.x, s1 = sg.y;
+                const uint4 f0 = fr[m * 64], f1 = fr[m * 64 + 1];
+                // chunk 0 holds pairs 0 and 1 of the block, chunk 1 pairs 2 and 3
+                const uint32_t a00 = va.x ^ ((s0 << sh) & 0x80008000u);
+                const uint32_t a01 = vb.x ^ ((s1 << sh) & 0x80008000u);
+                const uint32_t a02 = va.y ^ ((s0 << (sh - 4)) & 0x80008000u);
+                const uint32_t a03 = vb.y ^ ((s1 << (sh - 4)) & 0x80008000u);
+                const uint32_t a10 = va.z ^ ((s0 << (sh - 8)) & 0x80008000u);
+                const uint32_t a11 = vb.z ^ ((s1 << (sh - 8)) & 0x80008000u);
+                const uint32_t a12 = va.w ^ ((s0 << (sh - 12)) & 0x80008000u);
+                const uint32_t a13 = vb.w ^ ((s1 << (sh - 12)) & 0x80008000u);
+                float(&cc)[2][2][4] = acc[m & 1];
+                mma_bf16(cc[0][0], a00, a01, a02, a03, f0.x, f0.y);
+                mma_bf16(cc[0][1], a00, a01, a02, a03, f0.z, f0.w);
+                mma_bf16(cc[1][0], a10, a11, a12, a13, f1.x, f1.y);
+                mma_bf16(cc[1][1], a10, a11, a12, a13, f1.z, f1.w);
+            }
+            // accumulator (n-half h, register r): row slot (r < 2) or slot + 8
+            // (r >= 2), child 8 h + 2 q4 + (r & 1)
+            float sc[2][4];  // [token][2 h + (r & 1)]
+#pragma unroll
+            for (int h = 0; h < 2; ++h)
+#pragma unroll
+                for (int r = 0; r < 4; ++r)
+                    sc[r >> 1][2 * h + (r & 1)] =
+                        ((acc[0][0][h][r] + acc[0][1][h][r]) + (acc[1][0][h][r] + acc[1][1][h][r])) * a.inv_sqrt_d;
+            const uint32_t *gl = s_g + l * 16;
+            const uint32_t *ddl = s_dd + (l - 1) * kDedupSlots * 2;
+            uint32_t pcur = p0;
+            for (int tk = 0; tk < ntok; ++tk) {
+                uint32_t *bt = beams + tk * kBeam;
+                uint64_t *Lt = codes + tk * k;
+                // ---- duplicate children (R8): p_s ^ g_j' == p_s' ^ g_j with s' < s
+                // exactly when p_s ^ p_s' == g_j ^ g_j'; slot s's copy is dropped
+                uint32_t dmask = 0u;
+                {
+                    uint32_t delta = 0u;
+                    bool hit = false;
+                    if (lane < 28) {
+                        delta = bt[ps] ^ bt[psp];
+                        uint32_t h = dedup_hash(delta);
+                        for (int probe = 0; probe < kDedupSlots; ++probe) {
+                            const uint32_t key = ddl[2 * h];
+                            if (key == 0u) break;
+                            if (key == delta + 1u) {
+                                hit = true;
+                                break;
+                            }
+                            h = (h + 1u) & (kDedupSlots - 1);
+                        }
+                    }
+                    if (__any_sync(kFull, hit)) {
+                        if (lane < 4) dup[lane] = 0u;
+                        __syncwarp();
+                        if (hit) {
+                            uint32_t h = dedup_hash(delta);
+                            for (int probe = 0; probe < kDedupSlots; ++probe) {
+                                const uint32_t key = ddl[2 * h];
+                                if (key == 0u) break;
+                                if (key == delta + 1u) {
+                                    const uint32_t bit = (uint32_t)ps * 16u + (ddl[2 * h + 1] & 0xffu);
+                                    atomicOr(&dup[bit >> 5], 1u << (bit & 31u));
+                                }
+                                h = (h + 1u) & (kDedupSlots - 1);
+                            }
+                        }
+                        __syncwarp();
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            const uint32_t bit = (uint32_t)slot * 16u + (uint32_t)(8 * (e >> 1) + 2 * q4 + (e & 1));
+                            dmask |= ((dup[bit >> 5] >> (bit & 31u)) & 1u) << e;
+                        }
+                        __syncwarp();
+                    }
+                }
+                // ---- this lane's 4 children of token tk as candidate words
+                // (token 1's parent and scores move to token 0's registers after it)
+                uint64_t c[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const uint32_t ci = pcur ^ gl[8 * (e >> 1) + 2 * q4 + (e & 1)];
+                    const float z = standardise(sc[0][e], ci, a.mu, a.sigma, a.status);
+                    c[e] = ((dmask >> e) & 1u) ? 0ull : cword(z, ci);
+                    sc[0][e] = sc[1][e];
+                }
+                pcur = p1;
+                const bool next = l + 1 < L;
+                const int m = merge_entrants<KPL>(Lt, k, E, c, next ? bt : nullptr);
+                if (next && (m < kBeam || m > 32)) beam_tournament(c, bt);
+                __syncwarp();
+            }
+        }
+
+        // ---- the code of each token ----
+        for (int tk = 0; tk < ntok; ++tk) {
+            const uint64_t *Lt = codes + tk * k;
+            const int64_t row = t0 + tk;
+#pragma unroll
+            for (int r = 0; r < KPL; ++r) {
+                const int e = lane + 32 * r;
+                if (e < k) {
+                    const uint64_t w = Lt[e];
+                    a.idx[row * k + e] = (int32_t)cword_idx(w);
+                    a.val[row * k + e] = cword_z(w);
+                }
+            }
+        }
+        __syncwarp();
+    }
+}
+
+template <int NKC, int KPL>
+cudaError_t launch_kpl(const dpb_plan *p, const Args &a, int warps, cudaStream_t stream) {
+    const size_t smem = encode_mma_smem(p, warps);
+    const cudaError_t e =
+        cudaFuncSetAttribute(encode_kernel<NKC, KPL>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    int sms = 0;
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, p->device);
+    const int64_t pairs = (a.T + 1) / 2;
+    const int grid = (int)std::min<int64_t>((pairs + warps - 1) / warps, (int64_t)std::max(sms, 1));
+    encode_kernel<NKC, KPL><<<grid, warps * 32, smem, stream>>>(a);
+    return cudaGetLastError();
+}
+
+template <int NKC>
+cudaError_t launch_nkc(const dpb_plan *p, const Args &a, int warps, cudaStream_t stream) {
+    if (a.k <= 32) return launch_kpl<NKC, 1>(p, a, warps, stream);
+    if (a.k <= 64) return launch_kpl<NKC, 2>(p, a, warps, stream);
+    if (a.k <= 128) return launch_kpl<NKC, 4>(p, a, warps, stream);
+    return launch_kpl<NKC, 8>(p, a, warps, stream);
+}
+
+// One per table count, each in its own translation unit.
+cudaError_t launch_nkc2(const dpb_plan *p, const Args &a, int warps, cudaStream_t stream);
+cudaError_t launch_nkc3(const dpb_plan *p, const Args &a, int warps, cudaStream_t stream);
+cudaError_t launch_nkc4(const dpb_plan *p, const Args &a, int warps, cudaStream_t stream);
+
+}  // namespace mmaenc
+}  // namespace dpb

@@ -1,0 +1,13 @@
+// dpb_encode_mma_n2.cu -- the tensor-core encoder for fields whose inverse
+// coordinates take 2 five-bit sign tables (see dpb_encode_mma.cuh).
+#include "dpb_encode_mma.cuh"
+
+namespace dpb {
+namespace mmaenc {
+
+cudaError_t launch_nkc2(const dpb_plan *p, const Args &a, int warps, cudaStream_t stream) {
+    return launch_nkc<2>(p, a, warps, stream);
+}
+
+}  // namespace mmaenc
+}  // namespace dpb

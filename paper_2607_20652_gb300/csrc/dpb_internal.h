@@ -55,8 +55,10 @@ __host__ __device__ inline int frag_coord(int q4, int pair, int half) { return q
 // Builds the tensor-core encoder tables when the plan qualifies (dpb_plan.cu).
 void build_mma_tables(dpb_plan *p);
 
-// Dynamic shared memory (bytes) of the tensor-core encoder for this plan.
-size_t encode_mma_smem(const dpb_plan *p);
+// Launch shape of the tensor-core encoder: the most warps per block (16, 12,
+// 8 or 4) whose shared memory fits, or 0 if none does; and that memory.
+int encode_mma_warps(const dpb_plan *p);
+size_t encode_mma_smem(const dpb_plan *p, int warps);
 constexpr size_t kMaxSmemPerBlock = 227 * 1024;
 
 // Records a message for dpb_last_error() and returns `s`.

@@ -155,9 +155,9 @@ void build_mma_tables(dpb_plan *p) {
               c.select_mode == DPB_SELECT_GLOBAL && c.beam == 8 && c.k >= c.beam && c.k <= 256;
     for (int l = 1; l < c.levels && ok; ++l) ok = c.children[l] == 16;
     const int nblk = c.d / 32;
-    // every level's fragments, the tables and the warps' pools share one block
-    if (ok && encode_mma_smem(p) > kMaxSmemPerBlock) ok = false;
+    // every level's fragments, the tables and the warps' lists share one block
     p->mma_encode = ok;
+    if (ok && encode_mma_warps(p) == 0) p->mma_encode = ok = false;
     if (!ok) return;
     p->FRAG.assign((size_t)(c.levels - 1) * nblk * 256, 0u);
     auto sign_bf16 = [&](uint32_t g, int iota) -> uint32_t {
@@ -177,10 +177,14 @@ void build_mma_tables(dpb_plan *p) {
     for (int l = 1; l < c.levels; ++l) {
         uint32_t *tab = &p->DD[(size_t)(l - 1) * kDedupSlots * 2];
         const uint32_t *g = &p->G[(size_t)l * DPB_MAX_CHILDREN];
+        // parents of level l lie below 2^bits[l-1], so only differences below
+        // that bound can make two parents share a child
+        const uint32_t bound = 1u << c.bits[l - 1];
         for (int j = 0; j < 16; ++j)
             for (int jj = 0; jj < 16; ++jj) {
                 if (j == jj) continue;
                 const uint32_t delta = g[j] ^ g[jj];
+                if (delta >= bound) continue;
                 uint32_t h = dedup_hash(delta);
                 while (tab[2 * h] != 0) h = (h + 1) & (kDedupSlots - 1);
                 tab[2 * h] = delta + 1;
@@ -270,6 +274,8 @@ dpb_status resolve_and_build(const dpb_config *in, const uint32_t *generators, d
                 uint32_t g = generators[(size_t)l * DPB_MAX_CHILDREN + j];
                 if ((g >> c.bits[l]) != 0 || (g >> c.bits[l - 1]) == 0)
                     return fail(DPB_ERR_INVALID_ARG, "generator %u of level %d breaks the level rule", g, l);
+                for (int jj = 0; jj < j; ++jj)
+                    if (row[jj] == g) return fail(DPB_ERR_INVALID_ARG, "generator %u repeats at level %d", g, l);
                 row[j] = g;
             }
             continue;
