@@ -149,12 +149,13 @@ __global__ void __launch_bounds__(128) backward_warp_kernel(BackwardArgs a) {
 
 // ---- table-driven backward (d <= 1024) ---------------------------------------
 
-constexpr int kChunkBlocks = 8;                       // 32-coordinate blocks per analysis chunk
+constexpr int kChunkBlocks = 4;                       // 32-coordinate blocks per analysis chunk
 constexpr int kTabStride = 17;                        // 16 entries + 1 pad (bank spread)
 constexpr int kChunkTables = kChunkBlocks * 8 * kTabStride;  // nibble tables of a chunk (words)
+constexpr int kBwdWarps = 8;
 
 __host__ __device__ constexpr int bwd_warp_words(int d, int k) {
-    return 2 * pad4(d) /* r then grad_x; dL/dr */ + 6 * pad4(k) /* list, map, sums, offsets */ +
+    return pad4(d) /* r, then dL/dr, then grad_x */ + 6 * pad4(k) /* list, map, sums, offsets */ +
            (kSweepWords > kChunkTables ? kSweepWords : pad4(kChunkTables));
 }
 
@@ -163,14 +164,13 @@ __host__ __device__ constexpr int bwd_block_words(int d, int nkc) {
 }
 
 struct BwdWarp {
-    float *rg;      // [d] r, later grad_x
-    float *h;       // [d] dL/dr
+    float *buf;     // [d] r, then dL/dr, then grad_x
     uint32_t *hc;   // [k] hashed indices
     float *ha;      // [k] hashed coefficients, later grad_val / sigma
     int *cmap;      // [k] code entry -> hashed position (>= 0) or -(c+1) (basis) or INT_MIN
     float *gv;      // [k] analysis sums per hashed position
     uint32_t *o1;   // [k] packed table offsets (W5, PQ, VH_0, VH_1)
-    uint32_t *o2;   // [k] packed table offsets (VH_2, VH_3)
+    uint32_t *o2;   // [k] packed table offsets (VH_2, VH_3); later basis grad_x terms
     uint32_t *scratch;
 };
 
@@ -221,11 +221,11 @@ __device__ __forceinline__ void analyse(const BwdWarp &w, int nh, int d, const u
             const int i0 = 32 * (q0 + tau / 8) + 4 * (tau % 8);  // = 4 (8 q0 + tau)
             float4 hv = make_float4(0.f, 0.f, 0.f, 0.f);
             if (i0 + 3 < d) {
-                hv = *reinterpret_cast<const float4 *>(w.h + i0);
+                hv = *reinterpret_cast<const float4 *>(w.buf + i0);
             } else {
-                if (i0 < d) hv.x = w.h[i0];
-                if (i0 + 1 < d) hv.y = w.h[i0 + 1];
-                if (i0 + 2 < d) hv.z = w.h[i0 + 2];
+                if (i0 < d) hv.x = w.buf[i0];
+                if (i0 + 1 < d) hv.y = w.buf[i0 + 1];
+                if (i0 + 2 < d) hv.z = w.buf[i0 + 2];
             }
             // entry v = (v3 v2 v1 v0): sum_j (-1)^{v_j} h_j = A[v1 v0] + B[v3 v2]
             const float a0 = hv.x + hv.y, a1 = hv.x - hv.y;
@@ -260,7 +260,7 @@ __device__ __forceinline__ void analyse(const BwdWarp &w, int nh, int d, const u
 }
 
 template <typename Tio, int NKC>
-__global__ void __launch_bounds__(128) backward_lut_kernel(BackwardArgs a, int t) {
+__global__ void __launch_bounds__(kBwdWarps * 32, 3) backward_lut_kernel(BackwardArgs a, int t) {
     extern __shared__ __align__(16) uint32_t smem[];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
     const int d = a.d, k = a.k;
@@ -280,15 +280,15 @@ __global__ void __launch_bounds__(128) backward_lut_kernel(BackwardArgs a, int t
 
     uint32_t *base = smem + bwd_block_words(d, NKC) + (size_t)warp * bwd_warp_words(d, k);
     BwdWarp w;
-    w.rg = reinterpret_cast<float *>(base);
-    w.h = w.rg + dp;
-    w.hc = reinterpret_cast<uint32_t *>(w.h + dp);
+    w.buf = reinterpret_cast<float *>(base);
+    w.hc = reinterpret_cast<uint32_t *>(w.buf + dp);
     w.ha = reinterpret_cast<float *>(w.hc + kp);
     w.cmap = reinterpret_cast<int *>(w.ha + kp);
     w.gv = reinterpret_cast<float *>(w.cmap + kp);
     w.o1 = reinterpret_cast<uint32_t *>(w.gv + kp);
     w.o2 = w.o1 + kp;
     w.scratch = w.o2 + kp;
+    float *bterm = reinterpret_cast<float *>(w.o2);  // basis grad_x terms, after the analysis
     Sweep sw = sweep_at(w.scratch);
 
     const Tio *X = static_cast<const Tio *>(a.x);
@@ -297,8 +297,8 @@ __global__ void __launch_bounds__(128) backward_lut_kernel(BackwardArgs a, int t
     for (int64_t tk = (int64_t)blockIdx.x * nwarps + warp; tk < a.T; tk += (int64_t)gridDim.x * nwarps) {
         const int32_t *it = a.idx + tk * k;
         const float *vt = a.val + tk * k;
-        // ---- split the code: basis entries into rg, hashed entries listed ----
-        for (int i = lane; i < d; i += 32) w.rg[i] = 0.f;
+        // ---- split the code: basis entries into buf (r), hashed entries listed ----
+        for (int i = lane; i < d; i += 32) w.buf[i] = 0.f;
         __syncwarp();
         int nh = 0;
         for (int e0 = 0; e0 < k; e0 += 32) {
@@ -316,7 +316,7 @@ __global__ void __launch_bounds__(128) backward_lut_kernel(BackwardArgs a, int t
                 w.cmap[e] = INT_MIN;
             }
             if (valid && !hashed) {
-                atomicAdd(&w.rg[ci], v);
+                atomicAdd(&w.buf[ci], v);
                 w.cmap[e] = -(ci + 1);
             }
             const unsigned m = __ballot_sync(kFull, hashed);
@@ -331,7 +331,7 @@ __global__ void __launch_bounds__(128) backward_lut_kernel(BackwardArgs a, int t
             nh += __popc(m);
         }
         __syncwarp();
-        // ---- |x|, r and dL/dr ----
+        // ---- |x|, r and dL/dr (in place of r) ----
         float sxx = 0.f;
         for (int i = lane; i < d; i += 32) {
             const float xv = ld_elem(X, tk * d + i);
@@ -340,11 +340,10 @@ __global__ void __launch_bounds__(128) backward_lut_kernel(BackwardArgs a, int t
         const float nx = sqrtf(warp_sum(sxx));
         float direct = 0.f;
         if (a.norm_match) {
-            synthesise<NKC>(sw, w.hc, w.ha, nh, t, d, koff, a.inv_sqrt_d, w.rg);
+            synthesise<NKC>(sw, w.hc, w.ha, nh, t, d, koff, a.inv_sqrt_d, w.buf);
             float srr = 0.f, sgr = 0.f;
             for (int i = lane; i < d; i += 32) {
-                const float r = w.rg[i], g = ld_elem(GY, tk * d + i);
-                w.h[i] = g;
+                const float r = w.buf[i], g = ld_elem(GY, tk * d + i);
                 srr += r * r;
                 sgr += g * r;
             }
@@ -353,24 +352,21 @@ __global__ void __launch_bounds__(128) backward_lut_kernel(BackwardArgs a, int t
             const float nr = sqrtf(srr);
             if (nr > 0.f) {
                 const float c = nx / nr, beta = sgr / srr;
-                for (int i = lane; i < d; i += 32) w.h[i] = c * (w.h[i] - beta * w.rg[i]);
+                for (int i = lane; i < d; i += 32) w.buf[i] = c * (ld_elem(GY, tk * d + i) - beta * w.buf[i]);
                 direct = nx > 0.f ? sgr / nr : 0.f;
             } else {
-                for (int i = lane; i < d; i += 32) w.h[i] = 0.f;
+                for (int i = lane; i < d; i += 32) w.buf[i] = 0.f;
             }
         } else {
-            for (int i = lane; i < d; i += 32) w.h[i] = ld_elem(GY, tk * d + i);
+            for (int i = lane; i < d; i += 32) w.buf[i] = ld_elem(GY, tk * d + i);
         }
         __syncwarp();
         // ---- grad_val = <phi_e, dL/dr> ----
         analyse<NKC>(w, nh, d, w5, pq, vh);
-        // ---- grad_x: direct term, basis terms, then the hashed sum ----
-        const float dx = nx > 0.f ? direct / nx : 0.f;
-        for (int i = lane; i < d; i += 32) w.rg[i] = dx * ld_elem(X, tk * d + i);
-        __syncwarp();
+        // ---- grad_val of every entry; the grad_x coefficients ----
         for (int e = lane; e < k; e += 32) {
             const int cm = w.cmap[e];
-            float gvv = 0.f;
+            float gvv = 0.f, term = 0.f;
             if (cm >= 0) {
                 gvv = w.gv[cm] * a.inv_sqrt_d;
                 float sd = 1.f;
@@ -381,19 +377,29 @@ __global__ void __launch_bounds__(128) backward_lut_kernel(BackwardArgs a, int t
                 w.ha[cm] = gvv / sd;
             } else if (cm != INT_MIN) {
                 const int c = -cm - 1;
-                gvv = w.h[c];
+                gvv = w.buf[c];
                 float sd = 1.f;
                 if (a.sigma) {
                     sd = a.sigma[c];
                     if (!(sd > 0.f)) set_status(a.status, DPB_DEV_BAD_SIGMA);
                 }
-                atomicAdd(&w.rg[c], gvv / sd);
+                term = gvv / sd;
             }
+            bterm[e] = term;
             a.gval[tk * k + e] = gvv;
         }
         __syncwarp();
-        synthesise<NKC>(sw, w.hc, w.ha, nh, t, d, koff, a.inv_sqrt_d, w.rg);
-        for (int i = lane; i < d; i += 32) st_elem(GX, tk * d + i, w.rg[i]);
+        // ---- grad_x: direct term, basis terms, then the hashed sum ----
+        const float dx = nx > 0.f ? direct / nx : 0.f;
+        for (int i = lane; i < d; i += 32) w.buf[i] = dx * ld_elem(X, tk * d + i);
+        __syncwarp();
+        for (int e = lane; e < k; e += 32) {
+            const int cm = w.cmap[e];
+            if (cm < 0 && cm != INT_MIN) w.buf[-cm - 1] += bterm[e];  // indices are distinct
+        }
+        __syncwarp();
+        synthesise<NKC>(sw, w.hc, w.ha, nh, t, d, koff, a.inv_sqrt_d, w.buf);
+        for (int i = lane; i < d; i += 32) st_elem(GX, tk * d + i, w.buf[i]);
         __syncwarp();
     }
 }
@@ -406,10 +412,12 @@ int grid_for(const dpb_plan *p, int64_t T, int warps) {
 
 template <typename Tio, int NKC>
 cudaError_t run_backward_lut(const dpb_plan *p, const BackwardArgs &a, int64_t T, cudaStream_t stream) {
-    const int warps = 4;
+    const int warps = kBwdWarps;
     const size_t smem = sizeof(uint32_t) * ((size_t)bwd_block_words(p->cfg.d, NKC) +
                                             (size_t)warps * bwd_warp_words(p->cfg.d, p->code_len));
-    cudaFuncSetAttribute(backward_lut_kernel<Tio, NKC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    const cudaError_t e =
+        cudaFuncSetAttribute(backward_lut_kernel<Tio, NKC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
     backward_lut_kernel<Tio, NKC><<<grid_for(p, T, warps), warps * 32, smem, stream>>>(a, p->t);
     return cudaGetLastError();
 }
