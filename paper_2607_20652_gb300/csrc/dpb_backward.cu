@@ -331,16 +331,64 @@ __global__ void __launch_bounds__(kBwdWarps * 32, 3) backward_lut_kernel(Backwar
             nh += __popc(m);
         }
         __syncwarp();
-        // ---- |x|, r and dL/dr (in place of r) ----
         float sxx = 0.f;
         for (int i = lane; i < d; i += 32) {
             const float xv = ld_elem(X, tk * d + i);
             sxx += xv * xv;
         }
         const float nx = sqrtf(warp_sum(sxx));
-        float direct = 0.f;
-        if (a.norm_match) {
-            synthesise<NKC>(sw, w.hc, w.ha, nh, t, d, koff, a.inv_sqrt_d, w.buf);
+        float direct = 0.f;  // coefficient of x / |x| in grad_x
+        if (!a.norm_match) {
+            for (int i = lane; i < d; i += 32) w.buf[i] = ld_elem(GY, tk * d + i);
+            __syncwarp();
+        }
+        // Two synthesis passes share one call site: pass 0 builds r (norm
+        // matching only) and turns it into dL/dr; pass 1 adds the hashed
+        // entries' sum to grad_x.
+#pragma unroll 1
+        for (int pass = a.norm_match ? 0 : 1;; ++pass) {
+            if (pass == 1) {
+                // ---- grad_val = <phi_e, dL/dr> ----
+                analyse<NKC>(w, nh, d, w5, pq, vh);
+                // ---- grad_val of every entry; the grad_x coefficients ----
+                for (int e = lane; e < k; e += 32) {
+                    const int cm = w.cmap[e];
+                    float gvv = 0.f, term = 0.f;
+                    if (cm >= 0) {
+                        gvv = w.gv[cm] * a.inv_sqrt_d;
+                        float sd = 1.f;
+                        if (a.sigma) {
+                            sd = a.sigma[w.hc[cm]];
+                            if (!(sd > 0.f)) set_status(a.status, DPB_DEV_BAD_SIGMA);
+                        }
+                        w.ha[cm] = gvv / sd;
+                    } else if (cm != INT_MIN) {
+                        const int c = -cm - 1;
+                        gvv = w.buf[c];
+                        float sd = 1.f;
+                        if (a.sigma) {
+                            sd = a.sigma[c];
+                            if (!(sd > 0.f)) set_status(a.status, DPB_DEV_BAD_SIGMA);
+                        }
+                        term = gvv / sd;
+                    }
+                    bterm[e] = term;
+                    a.gval[tk * k + e] = gvv;
+                }
+                __syncwarp();
+                // ---- grad_x: direct term and basis terms, then the hashed sum ----
+                const float dx = nx > 0.f ? direct / nx : 0.f;
+                for (int i = lane; i < d; i += 32) w.buf[i] = dx * ld_elem(X, tk * d + i);
+                __syncwarp();
+                for (int e = lane; e < k; e += 32) {
+                    const int cm = w.cmap[e];
+                    if (cm < 0 && cm != INT_MIN) w.buf[-cm - 1] += bterm[e];  // indices are distinct
+                }
+                __syncwarp();
+            }
+            synthesise<NKC, kSweepCompact>(sw, w.hc, w.ha, nh, t, d, koff, a.inv_sqrt_d, w.buf);
+            if (pass == 1) break;
+            // ---- dL/dr = c (g - (<g,r>/|r|^2) r) in place of r ----
             float srr = 0.f, sgr = 0.f;
             for (int i = lane; i < d; i += 32) {
                 const float r = w.buf[i], g = ld_elem(GY, tk * d + i);
@@ -357,48 +405,8 @@ __global__ void __launch_bounds__(kBwdWarps * 32, 3) backward_lut_kernel(Backwar
             } else {
                 for (int i = lane; i < d; i += 32) w.buf[i] = 0.f;
             }
-        } else {
-            for (int i = lane; i < d; i += 32) w.buf[i] = ld_elem(GY, tk * d + i);
+            __syncwarp();
         }
-        __syncwarp();
-        // ---- grad_val = <phi_e, dL/dr> ----
-        analyse<NKC>(w, nh, d, w5, pq, vh);
-        // ---- grad_val of every entry; the grad_x coefficients ----
-        for (int e = lane; e < k; e += 32) {
-            const int cm = w.cmap[e];
-            float gvv = 0.f, term = 0.f;
-            if (cm >= 0) {
-                gvv = w.gv[cm] * a.inv_sqrt_d;
-                float sd = 1.f;
-                if (a.sigma) {
-                    sd = a.sigma[w.hc[cm]];
-                    if (!(sd > 0.f)) set_status(a.status, DPB_DEV_BAD_SIGMA);
-                }
-                w.ha[cm] = gvv / sd;
-            } else if (cm != INT_MIN) {
-                const int c = -cm - 1;
-                gvv = w.buf[c];
-                float sd = 1.f;
-                if (a.sigma) {
-                    sd = a.sigma[c];
-                    if (!(sd > 0.f)) set_status(a.status, DPB_DEV_BAD_SIGMA);
-                }
-                term = gvv / sd;
-            }
-            bterm[e] = term;
-            a.gval[tk * k + e] = gvv;
-        }
-        __syncwarp();
-        // ---- grad_x: direct term, basis terms, then the hashed sum ----
-        const float dx = nx > 0.f ? direct / nx : 0.f;
-        for (int i = lane; i < d; i += 32) w.buf[i] = dx * ld_elem(X, tk * d + i);
-        __syncwarp();
-        for (int e = lane; e < k; e += 32) {
-            const int cm = w.cmap[e];
-            if (cm < 0 && cm != INT_MIN) w.buf[-cm - 1] += bterm[e];  // indices are distinct
-        }
-        __syncwarp();
-        synthesise<NKC>(sw, w.hc, w.ha, nh, t, d, koff, a.inv_sqrt_d, w.buf);
         for (int i = lane; i < d; i += 32) st_elem(GX, tk * d + i, w.buf[i]);
         __syncwarp();
     }

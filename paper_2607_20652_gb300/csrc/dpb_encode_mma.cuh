@@ -185,9 +185,11 @@ __device__ __forceinline__ int warp_append(float *z, uint32_t *id, int n, bool t
 template <int R>
 __device__ __forceinline__ void warp_sort_desc(uint32_t (&v)[R]) {
     const int lane = threadIdx.x & 31;
-#pragma unroll
+    // stages are looped, not unrolled: the encoder's other phases already
+    // fill the instruction caches
+#pragma unroll 1
     for (int size = 2; size <= 32 * R; size <<= 1) {
-#pragma unroll
+#pragma unroll 1
         for (int stride = size / 2; stride > 0; stride >>= 1) {
             if (stride >= R) {
                 const bool lower = (lane & (stride / R)) == 0;
@@ -199,13 +201,18 @@ __device__ __forceinline__ void warp_sort_desc(uint32_t (&v)[R]) {
                 }
             } else {
 #pragma unroll
-                for (int r = 0; r < R; ++r) {
-                    const int q = r ^ stride;
-                    if (q > r) {
-                        const bool desc = (((lane * R + r) & size) == 0);
-                        const uint32_t hi = max(v[r], v[q]), lo = min(v[r], v[q]);
-                        v[r] = desc ? hi : lo;
-                        v[q] = desc ? lo : hi;
+                for (int cs = 1; cs < R; cs <<= 1) {
+                    if (stride == cs) {
+#pragma unroll
+                        for (int r = 0; r < R; ++r) {
+                            const int q = r ^ cs;
+                            if (q > r) {
+                                const bool desc = (((lane * R + r) & size) == 0);
+                                const uint32_t hi = max(v[r], v[q]), lo = min(v[r], v[q]);
+                                v[r] = desc ? hi : lo;
+                                v[q] = desc ? lo : hi;
+                            }
+                        }
                     }
                 }
             }
@@ -252,7 +259,7 @@ __device__ __forceinline__ void beam_tournament(uint64_t (&c)[4], uint32_t *beam
 // ahead of it; whatever lands at k or beyond drops out. When 8..32 words enter
 // and `beam` is given, the first 8 entrants become the beam.
 template <int KPL>
-__device__ __forceinline__ void merge_sorted(uint64_t *L, int k, const uint64_t *E, int m, uint32_t *beam) {
+__device__ __noinline__ void merge_sorted(uint64_t *L, int k, const uint64_t *E, int m, uint32_t *beam) {
     const int lane = threadIdx.x & 31;
     int top = 1;
     while (2 * top <= k) top <<= 1;

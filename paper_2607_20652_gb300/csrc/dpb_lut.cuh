@@ -248,12 +248,13 @@ __device__ __forceinline__ int split_code(const int32_t *idx, const float *val, 
 // ---- synthesis over a hashed list ---------------------------------------------
 
 // out[i] += scale * sum over one sweep, for every coordinate of the token.
-template <int NKC, int RUNS>
+// UNROLL coordinates blocks per loop trip.
+template <int NKC, int RUNS, int UNROLL>
 __device__ __forceinline__ void sweep_accumulate(const Sweep &s, float *out, const uint32_t *koff, int d,
                                                  float scale) {
     const int lane = threadIdx.x & 31;
     const int qn = (d + 31) / 32;
-#pragma unroll 2
+#pragma unroll UNROLL
     for (int q = 0; q < qn; ++q) {
         const int i = 32 * q + lane;
         const bool in = i < d;
@@ -263,32 +264,37 @@ __device__ __forceinline__ void sweep_accumulate(const Sweep &s, float *out, con
     }
 }
 
-template <int NKC>
+// Code shape of a sweep. kSweepWide rounds the runs up to one of five
+// unrolled widths (the extra runs read all-zero tables) and does two blocks
+// per trip: the fewest instructions. kSweepCompact always does all 13 runs,
+// one block per trip: the least code, for kernels whose other phases already
+// fill the instruction caches.
+enum SweepShape { kSweepWide, kSweepCompact };
+
+template <int NKC, SweepShape SHAPE>
 __device__ __forceinline__ void sweep_accumulate_runs(const Sweep &s, float *out, const uint32_t *koff,
                                                       int d, float scale) {
-    switch (s.runs) {
-        case 1: sweep_accumulate<NKC, 1>(s, out, koff, d, scale); break;
-        case 2: sweep_accumulate<NKC, 2>(s, out, koff, d, scale); break;
-        case 3: sweep_accumulate<NKC, 3>(s, out, koff, d, scale); break;
-        case 4: sweep_accumulate<NKC, 4>(s, out, koff, d, scale); break;
-        case 5: sweep_accumulate<NKC, 5>(s, out, koff, d, scale); break;
-        case 6: sweep_accumulate<NKC, 6>(s, out, koff, d, scale); break;
-        case 7: sweep_accumulate<NKC, 7>(s, out, koff, d, scale); break;
-        case 8: sweep_accumulate<NKC, 8>(s, out, koff, d, scale); break;
-        case 9: sweep_accumulate<NKC, 9>(s, out, koff, d, scale); break;
-        case 10: sweep_accumulate<NKC, 10>(s, out, koff, d, scale); break;
-        case 11: sweep_accumulate<NKC, 11>(s, out, koff, d, scale); break;
-        case 12: sweep_accumulate<NKC, 12>(s, out, koff, d, scale); break;
-        default: sweep_accumulate<NKC, 13>(s, out, koff, d, scale); break;
+    if constexpr (SHAPE == kSweepCompact) {
+        sweep_accumulate<NKC, kMaxRuns, 1>(s, out, koff, d, scale);
+    } else if (s.runs <= 4) {
+        sweep_accumulate<NKC, 4, 2>(s, out, koff, d, scale);
+    } else if (s.runs <= 6) {
+        sweep_accumulate<NKC, 6, 2>(s, out, koff, d, scale);
+    } else if (s.runs <= 8) {
+        sweep_accumulate<NKC, 8, 2>(s, out, koff, d, scale);
+    } else if (s.runs <= 10) {
+        sweep_accumulate<NKC, 10, 2>(s, out, koff, d, scale);
+    } else {
+        sweep_accumulate<NKC, kMaxRuns, 2>(s, out, koff, d, scale);
     }
 }
 
 // out[i] += scale * sum_e coef_e (-1)^{parity(M[i] AND c_e)} over n codes
 // (indices c, coefficients coef), 64 codes per sweep. koff[i] holds the
 // packed chunk offsets of inv(i) (kappa_offsets8).
-template <int NKC>
-__device__ __forceinline__ void synthesise(Sweep &s, const uint32_t *c, const float *coef, int n, int t,
-                                           int d, const uint32_t *koff, float scale, float *out) {
+template <int NKC, SweepShape SHAPE = kSweepWide>
+__device__ __forceinline__ void synthesise(Sweep &s, const uint32_t *c, const float *coef, int n, int t, int d,
+                                           const uint32_t *koff, float scale, float *out) {
     const int lane = threadIdx.x & 31;
     const int qn = (d + 31) / 32;
     for (int g0 = 0; g0 < n; g0 += 64) {
@@ -302,7 +308,7 @@ __device__ __forceinline__ void synthesise(Sweep &s, const uint32_t *c, const fl
         __syncwarp();
         sweep_build_values(s);
         __syncwarp();
-        sweep_accumulate_runs<NKC>(s, out, koff, d, scale);
+        sweep_accumulate_runs<NKC, SHAPE>(s, out, koff, d, scale);
         __syncwarp();
     }
 }
