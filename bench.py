@@ -35,7 +35,17 @@ WORKLOAD = "wide"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
                   "sm_max_mhz": 2070.0}
 GB300_SMS = 152
-FP32_LANES_PER_SM = 128
+FP32_LANES_PER_SM = 128   # FADD/FFMA per SM per clock (measured; packed f32x2 gave no more)
+INT_LOGIC_PER_SM = 64     # LOP3 per SM per clock (measured)
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic_wide_T65536.txt")
+# files whose contents define each timed kernel (traffic figures are dropped
+# when any of them changed after the counters were taken)
+KERNEL_SOURCES = {
+    "encode": ["dpb_encode_mma.cuh", "dpb_encode_mma.cu", "dpb_encode_mma_n2.cu", "dpb_select.cuh",
+               "dpb_device.cuh", "dpb_internal.h", "dpb_plan.cu"],
+    "decode": ["dpb_decode.cu", "dpb_lut.cuh", "dpb_device.cuh", "dpb_internal.h", "dpb_plan.cu"],
+    "backward": ["dpb_backward.cu", "dpb_lut.cuh", "dpb_device.cuh", "dpb_internal.h", "dpb_plan.cu"],
+}
 
 
 # ---------------------------------------------------------------------------
@@ -90,36 +100,73 @@ def load_peaks():
 
 def algorithmic_work(cfg: dict, T: int, k_hash: float, s: int):
     """Per-launch algorithmic bytes and operations of each call (the method's
-    own sums, not implementation overhead). s = bytes per stored element."""
+    own sums, not implementation overhead). s = bytes per stored element;
+    k_hash = mean number of code entries that are hashed directions."""
     d, k, B = cfg["d"], cfg["k"], cfg["beam"]
     mma = sum(2 * B * cfg["children"][l] * d for l in range(1, cfg["levels"]))
+    signs = (cfg["levels"] - 1) * B * d  # the x (.) phi~_p products of Eq. 6
     return {
-        "encode": {"bytes": T * (d * s + 8 * k + 4), "tensor_flops": T * mma},
-        "decode": {"bytes": T * (8 * k + 4 + d * s), "fp_ops": T * k_hash * d},
-        "backward": {"bytes": T * (3 * d * s + 12 * k), "fp_ops": T * 2 * k_hash * d},
+        "encode": {"bytes": T * (d * s + 8 * k + 4), "tensor_flops": T * mma, "int_ops": T * signs},
+        "decode": {"bytes": T * (8 * k + 4 + d * s), "fp_ops": T * (k_hash * d + 3 * d)},
+        "backward": {"bytes": T * (3 * d * s + 12 * k), "fp_ops": T * (2 * k_hash * d + 6 * d)},
     }
 
 
-def roofline_for(name: str, work: dict, seconds: float, peaks: dict, src: str):
-    hbm = peaks["hbm_gbs"] * 1e9
-    tc = peaks["bf16_tflops_sustained"] * 1e12
-    alu = GB300_SMS * FP32_LANES_PER_SM * peaks.get("sm_max_mhz", 2070.0) * 1e6
-    terms = {"hbm": work["bytes"] / hbm}
-    if "tensor_flops" in work:
-        terms["tensor"] = work["tensor_flops"] / tc
-    if "fp_ops" in work:
-        terms["alu"] = work["fp_ops"] / alu
+def peak_rates(peaks: dict):
+    mhz = peaks.get("sm_max_mhz", 2070.0)
+    return {"hbm": peaks["hbm_gbs"] * 1e9, "tensor": peaks["bf16_tflops_sustained"] * 1e12,
+            "alu": GB300_SMS * FP32_LANES_PER_SM * mhz * 1e6, "int": GB300_SMS * INT_LOGIC_PER_SM * mhz * 1e6}
+
+
+def roofline_for(name: str, work: dict, seconds: float, peaks: dict, src: str, traffic=None):
+    """The slowest of the call's terms at peak (HBM bytes, tensor flops, FP32
+    adds, integer logic ops) is its roofline; achieved = that term's work / time."""
+    rate = peak_rates(peaks)
+    keys = {"hbm": "bytes", "tensor": "tensor_flops", "alu": "fp_ops", "int": "int_ops"}
+    terms = {b: work[kk] / rate[b] for b, kk in keys.items() if kk in work}
     bound = max(terms, key=terms.get)
+    achieved = work[keys[bound]] / seconds
     if bound == "hbm":
-        achieved, peak, unit = work["bytes"] / seconds / 1e9, peaks["hbm_gbs"], "GB/s"
+        achieved, peak, unit = achieved / 1e9, peaks["hbm_gbs"], "GB/s"
+        psrc = "copy"
     elif bound == "tensor":
-        achieved, peak, unit = work["tensor_flops"] / seconds / 1e12, peaks["bf16_tflops_sustained"], "TFLOP/s"
+        achieved, peak, unit = achieved / 1e12, peaks["bf16_tflops_sustained"], "TFLOP/s"
+        psrc = "bf16 sustained"
+    elif bound == "alu":
+        achieved, peak, unit = achieved / 1e12, rate["alu"] / 1e12, "TFLOP/s"
+        psrc = "152 SMs x 128 FP32 adds/clock x max SM clock"
     else:
-        achieved, peak, unit = work["fp_ops"] / seconds / 1e12, alu / 1e12, "TFLOP/s"
+        achieved, peak, unit = achieved / 1e12, rate["int"] / 1e12, "Tops/s"
+        psrc = "152 SMs x 64 LOP3/clock x max SM clock"
     return {"kernel": name, "bound": bound, "achieved": round(achieved, 3), "peak": round(peak, 3),
-            "unit": unit, "frac": round(achieved / peak, 4), "traffic": None,
-            "peak_source": f"{src} ({'bf16 sustained' if bound == 'tensor' else 'copy' if bound == 'hbm' else '152 SMs x 128 FP32 lanes x max SM clock'})",
+            "unit": unit, "frac": round(achieved / peak, 4), "traffic": traffic,
+            "algorithmic_bytes": int(work["bytes"]),
+            "peak_source": f"{src} ({psrc})",
             "t_roofline_us": round(terms[bound] * 1e6, 2), "t_measured_us": round(seconds * 1e6, 2)}
+
+
+def kernel_source_hash(name: str) -> str:
+    import hashlib
+    h = hashlib.sha256()
+    for f in KERNEL_SOURCES[name]:
+        with open(os.path.join(ROOT, "paper_2607_20652_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def measured_traffic(name: str, T: int):
+    """DRAM bytes per launch of `name` from the committed ncu figures, or None
+    when absent, taken at another size, or the kernel changed since."""
+    try:
+        with open(TRAFFIC_FILE) as f:
+            for line in f:
+                parts = line.split()
+                if len(parts) == 4 and not line.startswith("#") and parts[0] == name:
+                    if int(parts[1]) == T and parts[3] == kernel_source_hash(name):
+                        return int(parts[2])
+    except (OSError, ValueError):
+        pass
+    return None
 
 
 class ClockSampler:
@@ -267,9 +314,10 @@ def run_reference(args, world, rank):
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(1e3 * total / args.steps, 3), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": config_block(w, world, n_tokens=n),
+        "config": config_block(w, world),
         "cpu_baseline": {"kind": "oracle", "cores": 1, "value": round(value, 2), "unit": "tokens/s",
-                         "sample": f"{n} tokens of the {WORKLOAD} workload per step, single-threaded C oracle (fp64)"},
+                         "sample": f"each step: the first {n} of the {w['T']} tokens of the {WORKLOAD} workload "
+                                   f"(planted, seed 0), encode+decode+backward, single-threaded C oracle (fp64)"},
         "e2e": {"value": round(value, 2), "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -363,7 +411,7 @@ def run_ours(args, world, rank, local):
     peaks, src = load_peaks()
     work = algorithmic_work(plan.config, T, k_hash, 2)
     dom = max(kern_ms, key=kern_ms.get)
-    roof = roofline_for(dom, work[dom], kern_ms[dom] / 1e3, peaks, src)
+    roof = roofline_for(dom, work[dom], kern_ms[dom] / 1e3, peaks, src, measured_traffic(dom, T))
     kernels = {n: {"ms": round(v, 4), **{kk: vv for kk, vv in roofline_for(n, work[n], v / 1e3, peaks, src).items()
                                           if kk in ("bound", "frac", "t_roofline_us")}}
                for n, v in kern_ms.items()}
