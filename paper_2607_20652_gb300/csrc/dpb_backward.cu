@@ -11,6 +11,8 @@
 // tables of signed sums of dL/dr over 4 coordinates (see analyse()).
 #include <algorithm>
 #include <climits>
+#include <cstdint>
+#include <initializer_list>
 
 #include "dpb_device.cuh"
 #include "dpb_internal.h"
@@ -153,6 +155,7 @@ constexpr int kChunkBlocks = 4;                       // 32-coordinate blocks pe
 constexpr int kTabStride = 17;                        // 16 entries + 1 pad (bank spread)
 constexpr int kChunkTables = kChunkBlocks * 8 * kTabStride;  // nibble tables of a chunk (words)
 constexpr int kBwdWarps = 8;
+static_assert(kChunkBlocks == 4, "analyse() maps items to blocks with three compares");
 
 __host__ __device__ constexpr int bwd_warp_words(int d, int k) {
     return pad4(d) /* r, then dL/dr, then grad_x */ + 6 * pad4(k) /* list, map, sums, offsets */ +
@@ -239,7 +242,8 @@ __device__ __forceinline__ void analyse(const BwdWarp &w, int nh, int d, const u
         }
         __syncwarp();
         for (int it = lane; it < cq * nhp; it += 32) {
-            const int qq = it / nhp, e = it - qq * nhp;
+            // block of the chunk and code of this item (cq <= 4 blocks)
+            const int qq = (it >= nhp) + (it >= 2 * nhp) + (it >= 3 * nhp), e = it - qq * nhp;
             if (e < nh) {
                 const uint32_t s = block_signs<NKC>(w5, pq, vh, q0 + qq, w.o1[e], w.o2[e]);
                 const char *T = reinterpret_cast<const char *>(TH + qq * 8 * kTabStride);
@@ -259,7 +263,7 @@ __device__ __forceinline__ void analyse(const BwdWarp &w, int nh, int d, const u
     }
 }
 
-template <typename Tio, int NKC>
+template <typename Tio, int NKC, bool VEC>
 __global__ void __launch_bounds__(kBwdWarps * 32, 3) backward_lut_kernel(BackwardArgs a, int t) {
     extern __shared__ __align__(16) uint32_t smem[];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
@@ -298,7 +302,8 @@ __global__ void __launch_bounds__(kBwdWarps * 32, 3) backward_lut_kernel(Backwar
         const int32_t *it = a.idx + tk * k;
         const float *vt = a.val + tk * k;
         // ---- split the code: basis entries into buf (r), hashed entries listed ----
-        for (int i = lane; i < d; i += 32) w.buf[i] = 0.f;
+        const Tio *xr = X + tk * d, *gr = GY + tk * d;
+        RowOps<VEC>::fill(w.buf, d, 0.f);
         __syncwarp();
         int nh = 0;
         for (int e0 = 0; e0 < k; e0 += 32) {
@@ -331,15 +336,10 @@ __global__ void __launch_bounds__(kBwdWarps * 32, 3) backward_lut_kernel(Backwar
             nh += __popc(m);
         }
         __syncwarp();
-        float sxx = 0.f;
-        for (int i = lane; i < d; i += 32) {
-            const float xv = ld_elem(X, tk * d + i);
-            sxx += xv * xv;
-        }
-        const float nx = sqrtf(warp_sum(sxx));
+        const float nx = sqrtf(warp_sum(RowOps<VEC>::sumsq(xr, d)));
         float direct = 0.f;  // coefficient of x / |x| in grad_x
         if (!a.norm_match) {
-            for (int i = lane; i < d; i += 32) w.buf[i] = ld_elem(GY, tk * d + i);
+            RowOps<VEC>::scale_in(w.buf, gr, d, 1.f);
             __syncwarp();
         }
         // Two synthesis passes share one call site: pass 0 builds r (norm
@@ -378,7 +378,7 @@ __global__ void __launch_bounds__(kBwdWarps * 32, 3) backward_lut_kernel(Backwar
                 __syncwarp();
                 // ---- grad_x: direct term and basis terms, then the hashed sum ----
                 const float dx = nx > 0.f ? direct / nx : 0.f;
-                for (int i = lane; i < d; i += 32) w.buf[i] = dx * ld_elem(X, tk * d + i);
+                RowOps<VEC>::scale_in(w.buf, xr, d, dx);
                 __syncwarp();
                 for (int e = lane; e < k; e += 32) {
                     const int cm = w.cmap[e];
@@ -390,24 +390,19 @@ __global__ void __launch_bounds__(kBwdWarps * 32, 3) backward_lut_kernel(Backwar
             if (pass == 1) break;
             // ---- dL/dr = c (g - (<g,r>/|r|^2) r) in place of r ----
             float srr = 0.f, sgr = 0.f;
-            for (int i = lane; i < d; i += 32) {
-                const float r = w.buf[i], g = ld_elem(GY, tk * d + i);
-                srr += r * r;
-                sgr += g * r;
-            }
+            RowOps<VEC>::dots(w.buf, gr, d, srr, sgr);
             srr = warp_sum(srr);
             sgr = warp_sum(sgr);
             const float nr = sqrtf(srr);
             if (nr > 0.f) {
-                const float c = nx / nr, beta = sgr / srr;
-                for (int i = lane; i < d; i += 32) w.buf[i] = c * (ld_elem(GY, tk * d + i) - beta * w.buf[i]);
+                RowOps<VEC>::project(w.buf, gr, d, nx / nr, sgr / srr);
                 direct = nx > 0.f ? sgr / nr : 0.f;
             } else {
-                for (int i = lane; i < d; i += 32) w.buf[i] = 0.f;
+                RowOps<VEC>::fill(w.buf, d, 0.f);
             }
             __syncwarp();
         }
-        for (int i = lane; i < d; i += 32) st_elem(GX, tk * d + i, w.buf[i]);
+        RowOps<VEC>::store(GX + tk * d, w.buf, d, 1.f);
         __syncwarp();
     }
 }
@@ -418,16 +413,32 @@ int grid_for(const dpb_plan *p, int64_t T, int warps) {
     return (int)std::min<int64_t>((T + warps - 1) / warps, (int64_t)sms * 16);
 }
 
-template <typename Tio, int NKC>
+template <typename Tio, int NKC, bool VEC>
 cudaError_t run_backward_lut(const dpb_plan *p, const BackwardArgs &a, int64_t T, cudaStream_t stream) {
     const int warps = kBwdWarps;
     const size_t smem = sizeof(uint32_t) * ((size_t)bwd_block_words(p->cfg.d, NKC) +
                                             (size_t)warps * bwd_warp_words(p->cfg.d, p->code_len));
-    const cudaError_t e =
-        cudaFuncSetAttribute(backward_lut_kernel<Tio, NKC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    const cudaError_t e = cudaFuncSetAttribute(backward_lut_kernel<Tio, NKC, VEC>,
+                                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    backward_lut_kernel<Tio, NKC><<<grid_for(p, T, warps), warps * 32, smem, stream>>>(a, p->t);
+    backward_lut_kernel<Tio, NKC, VEC><<<grid_for(p, T, warps), warps * 32, smem, stream>>>(a, p->t);
     return cudaGetLastError();
+}
+
+// Rows can be read 4 elements at a time: d % 4 == 0 and every row pointer
+// aligned to 4 elements.
+template <typename Tio>
+bool rows_vec(int d, std::initializer_list<const void *> ptrs) {
+    if (d % 4 != 0) return false;
+    for (const void *q : ptrs)
+        if (reinterpret_cast<uintptr_t>(q) % (4 * sizeof(Tio)) != 0) return false;
+    return true;
+}
+
+template <typename Tio, int NKC>
+cudaError_t run_backward_lut(const dpb_plan *p, const BackwardArgs &a, int64_t T, cudaStream_t stream) {
+    if (rows_vec<Tio>(p->cfg.d, {a.x, a.gy, a.gx})) return run_backward_lut<Tio, NKC, true>(p, a, T, stream);
+    return run_backward_lut<Tio, NKC, false>(p, a, T, stream);
 }
 
 template <typename Tio>

@@ -90,7 +90,7 @@ __global__ void __launch_bounds__(128) decode_warp_kernel(DecodeArgs a) {
 // list (indices, coefficients) and one sweep's tables.
 __host__ __device__ constexpr int decode_warp_words(int d, int k) { return pad4(d) + 2 * pad4(k) + kSweepWords; }
 
-template <typename Tio, int NKC>
+template <typename Tio, int NKC, bool VEC>
 __global__ void __launch_bounds__(256) decode_lut_kernel(DecodeArgs a, int t) {
     extern __shared__ __align__(16) uint32_t smem[];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
@@ -104,18 +104,18 @@ __global__ void __launch_bounds__(256) decode_lut_kernel(DecodeArgs a, int t) {
     Sweep sw = sweep_at(base + dp + 2 * kp);
     Tio *Y = static_cast<Tio *>(a.y);
     for (int64_t tk = (int64_t)blockIdx.x * nwarps + warp; tk < a.T; tk += (int64_t)gridDim.x * nwarps) {
-        for (int i = lane; i < d; i += 32) r[i] = 0.f;
+        RowOps<VEC>::fill(r, d, 0.f);
         __syncwarp();
         const int nh = split_code(a.idx + tk * a.k, a.val + tk * a.k, a.k, d, a.m_mask, r, hl, a.status);
         synthesise<NKC>(sw, hl.c, hl.a, nh, t, d, koff, a.inv_sqrt_d, r);
-        float ss = 0.f;
-        for (int i = lane; i < d; i += 32) ss += r[i] * r[i];
         float scale = 1.f;
         if (a.norm_match) {
+            float ss = 0.f, unused = 0.f;
+            RowOps<VEC>::dots(r, r, d, ss, unused);
             const float nr = sqrtf(warp_sum(ss));
             scale = nr > 0.f ? a.xnorm[tk] / nr : 0.f;
         }
-        for (int i = lane; i < d; i += 32) st_elem(Y, tk * d + i, r[i] * scale);
+        RowOps<VEC>::store(Y + tk * d, r, d, scale);
         __syncwarp();
     }
 }
@@ -130,13 +130,23 @@ int grid_for(const dpb_plan *p, int64_t T, int warps) {
 
 namespace {
 
-template <typename Tio, int NKC>
+template <typename Tio, int NKC, bool VEC>
 cudaError_t run_decode_lut(const dpb_plan *p, const DecodeArgs &a, int64_t T, cudaStream_t stream) {
     const int warps = 8;
     const size_t smem = sizeof(uint32_t) * ((size_t)pad4(p->cfg.d) + (size_t)warps * decode_warp_words(p->cfg.d, p->code_len));
-    cudaFuncSetAttribute(decode_lut_kernel<Tio, NKC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    decode_lut_kernel<Tio, NKC><<<grid_for(p, T, warps), warps * 32, smem, stream>>>(a, p->t);
+    const cudaError_t e = cudaFuncSetAttribute(decode_lut_kernel<Tio, NKC, VEC>,
+                                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    decode_lut_kernel<Tio, NKC, VEC><<<grid_for(p, T, warps), warps * 32, smem, stream>>>(a, p->t);
     return cudaGetLastError();
+}
+
+template <typename Tio, int NKC>
+cudaError_t run_decode_lut(const dpb_plan *p, const DecodeArgs &a, int64_t T, cudaStream_t stream) {
+    // y can be written 4 elements at a time: d % 4 == 0 and y aligned to 4 elements
+    if (p->cfg.d % 4 == 0 && reinterpret_cast<uintptr_t>(a.y) % (4 * sizeof(Tio)) == 0)
+        return run_decode_lut<Tio, NKC, true>(p, a, T, stream);
+    return run_decode_lut<Tio, NKC, false>(p, a, T, stream);
 }
 
 template <typename Tio>

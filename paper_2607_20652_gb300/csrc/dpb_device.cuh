@@ -22,6 +22,118 @@ __device__ __forceinline__ void st_elem(__nv_bfloat16 *p, int64_t i, float v) {
     p[i] = __float2bfloat16_rn(v);
 }
 
+// ---- one warp over the d elements of a row ----------------------------------
+//
+// Rows of x, y, grad_y, grad_x against a float row `buf` in shared memory.
+// With VEC the lane takes 4 consecutive elements at a time (8-byte bf16 or
+// 16-byte fp32 accesses; the caller guarantees d % 4 == 0 and aligned rows),
+// otherwise one element at a time.
+
+__device__ __forceinline__ float4 ld4(const __nv_bfloat16 *p) {
+    const uint2 u = *reinterpret_cast<const uint2 *>(p);
+    return make_float4(__uint_as_float(u.x << 16), __uint_as_float(u.x & 0xffff0000u), __uint_as_float(u.y << 16),
+                       __uint_as_float(u.y & 0xffff0000u));
+}
+__device__ __forceinline__ float4 ld4(const float *p) { return *reinterpret_cast<const float4 *>(p); }
+__device__ __forceinline__ void st4(__nv_bfloat16 *p, float4 v) {
+    const __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y), b = __floats2bfloat162_rn(v.z, v.w);
+    uint2 u;
+    u.x = *reinterpret_cast<const uint32_t *>(&a);
+    u.y = *reinterpret_cast<const uint32_t *>(&b);
+    *reinterpret_cast<uint2 *>(p) = u;
+}
+__device__ __forceinline__ void st4(float *p, float4 v) { *reinterpret_cast<float4 *>(p) = v; }
+
+template <bool VEC>
+struct RowOps {
+    // buf[i] = v
+    __device__ __forceinline__ static void fill(float *buf, int d, float v) {
+        const int lane = threadIdx.x & 31;
+        if (VEC) {
+            for (int i = 4 * lane; i < d; i += 128) *reinterpret_cast<float4 *>(buf + i) = make_float4(v, v, v, v);
+        } else {
+            for (int i = lane; i < d; i += 32) buf[i] = v;
+        }
+    }
+    // sum over the row of row[i]^2 (this lane's share)
+    template <typename T>
+    __device__ __forceinline__ static float sumsq(const T *row, int d) {
+        const int lane = threadIdx.x & 31;
+        float s = 0.f;
+        if (VEC) {
+            for (int i = 4 * lane; i < d; i += 128) {
+                const float4 v = ld4(row + i);
+                s += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+            }
+        } else {
+            for (int i = lane; i < d; i += 32) {
+                const float v = ld_elem(row, i);
+                s += v * v;
+            }
+        }
+        return s;
+    }
+    // buf[i] = c * row[i]
+    template <typename T>
+    __device__ __forceinline__ static void scale_in(float *buf, const T *row, int d, float c) {
+        const int lane = threadIdx.x & 31;
+        if (VEC) {
+            for (int i = 4 * lane; i < d; i += 128) {
+                const float4 v = ld4(row + i);
+                *reinterpret_cast<float4 *>(buf + i) = make_float4(c * v.x, c * v.y, c * v.z, c * v.w);
+            }
+        } else {
+            for (int i = lane; i < d; i += 32) buf[i] = c * ld_elem(row, i);
+        }
+    }
+    // srr += buf[i]^2, sgr += row[i] buf[i] (this lane's share)
+    template <typename T>
+    __device__ __forceinline__ static void dots(const float *buf, const T *row, int d, float &srr, float &sgr) {
+        const int lane = threadIdx.x & 31;
+        if (VEC) {
+            for (int i = 4 * lane; i < d; i += 128) {
+                const float4 r = *reinterpret_cast<const float4 *>(buf + i), g = ld4(row + i);
+                srr += r.x * r.x + r.y * r.y + r.z * r.z + r.w * r.w;
+                sgr += g.x * r.x + g.y * r.y + g.z * r.z + g.w * r.w;
+            }
+        } else {
+            for (int i = lane; i < d; i += 32) {
+                const float r = buf[i], g = ld_elem(row, i);
+                srr += r * r;
+                sgr += g * r;
+            }
+        }
+    }
+    // buf[i] = c (row[i] - beta buf[i])
+    template <typename T>
+    __device__ __forceinline__ static void project(float *buf, const T *row, int d, float c, float beta) {
+        const int lane = threadIdx.x & 31;
+        if (VEC) {
+            for (int i = 4 * lane; i < d; i += 128) {
+                const float4 r = *reinterpret_cast<const float4 *>(buf + i), g = ld4(row + i);
+                *reinterpret_cast<float4 *>(buf + i) =
+                    make_float4(c * (g.x - beta * r.x), c * (g.y - beta * r.y), c * (g.z - beta * r.z),
+                                c * (g.w - beta * r.w));
+            }
+        } else {
+            for (int i = lane; i < d; i += 32) buf[i] = c * (ld_elem(row, i) - beta * buf[i]);
+        }
+    }
+    // row[i] = c * buf[i]
+    template <typename T>
+    __device__ __forceinline__ static void store(T *row, const float *buf, int d, float c) {
+        const int lane = threadIdx.x & 31;
+        if (VEC) {
+            for (int i = 4 * lane; i < d; i += 128) {
+                const float4 r = *reinterpret_cast<const float4 *>(buf + i);
+                st4(row + i, make_float4(c * r.x, c * r.y, c * r.z, c * r.w));
+            }
+        } else {
+            for (int i = lane; i < d; i += 32) st_elem(row, i, c * buf[i]);
+        }
+    }
+};
+
 // ---- parity signs (App. A.4, Eq. 26-27) ------------------------------------
 
 // Sign of coordinate iota of phi~_c in bit 31: parity(M[iota] AND c), so a
