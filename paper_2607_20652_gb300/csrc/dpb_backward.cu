@@ -220,6 +220,8 @@ __device__ __forceinline__ void analyse(const BwdWarp &w, int nh, int d, const u
     float *TH = reinterpret_cast<float *>(w.scratch);
     for (int q0 = 0; q0 < qn; q0 += kChunkBlocks) {
         const int cq = min(kChunkBlocks, qn - q0);
+        // both loops stay rolled: this kernel's hot code is at the instruction caches' size
+#pragma unroll 1
         for (int tau = lane; tau < cq * 8; tau += 32) {
             const int i0 = 32 * (q0 + tau / 8) + 4 * (tau % 8);  // = 4 (8 q0 + tau)
             float4 hv = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -241,6 +243,7 @@ __device__ __forceinline__ void analyse(const BwdWarp &w, int nh, int d, const u
             for (int v = 0; v < 16; ++v) T[v] = A[v & 3] + B[v >> 2];
         }
         __syncwarp();
+#pragma unroll 1
         for (int it = lane; it < cq * nhp; it += 32) {
             // block of the chunk and code of this item (cq <= 4 blocks)
             const int qq = (it >= nhp) + (it >= 2 * nhp) + (it >= 3 * nhp), e = it - qq * nhp;

@@ -180,44 +180,46 @@ __device__ __forceinline__ int warp_append(float *z, uint32_t *id, int n, bool t
     return n + __popc(mb);
 }
 
-// Warp bitonic sort, descending, of 32 R words held R per lane (element
-// lane * R + r).
+// One compare-exchange stage (size, stride) of a warp bitonic sort,
+// descending, of 32 R words held R per lane (element lane * R + r).
 template <int R>
-__device__ __forceinline__ void warp_sort_desc(uint32_t (&v)[R]) {
+__device__ __forceinline__ void sort_stage(uint32_t (&v)[R], int size, int stride) {
     const int lane = threadIdx.x & 31;
-    // stages are looped, not unrolled: the encoder's other phases already
-    // fill the instruction caches
-#pragma unroll 1
-    for (int size = 2; size <= 32 * R; size <<= 1) {
-#pragma unroll 1
-        for (int stride = size / 2; stride > 0; stride >>= 1) {
-            if (stride >= R) {
-                const bool lower = (lane & (stride / R)) == 0;
+    if (stride >= R) {
+        const bool lower = (lane & (stride / R)) == 0;
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+            const bool desc = (((lane * R + r) & size) == 0);
+            const uint32_t o = __shfl_xor_sync(kFull, v[r], stride / R);
+            v[r] = (lower == desc) ? max(v[r], o) : min(v[r], o);
+        }
+    } else {
+#pragma unroll
+        for (int cs = 1; cs < R; cs <<= 1) {
+            if (stride == cs) {
 #pragma unroll
                 for (int r = 0; r < R; ++r) {
-                    const bool desc = (((lane * R + r) & size) == 0);
-                    const uint32_t o = __shfl_xor_sync(kFull, v[r], stride / R);
-                    v[r] = (lower == desc) ? max(v[r], o) : min(v[r], o);
-                }
-            } else {
-#pragma unroll
-                for (int cs = 1; cs < R; cs <<= 1) {
-                    if (stride == cs) {
-#pragma unroll
-                        for (int r = 0; r < R; ++r) {
-                            const int q = r ^ cs;
-                            if (q > r) {
-                                const bool desc = (((lane * R + r) & size) == 0);
-                                const uint32_t hi = max(v[r], v[q]), lo = min(v[r], v[q]);
-                                v[r] = desc ? hi : lo;
-                                v[q] = desc ? lo : hi;
-                            }
-                        }
+                    const int q = r ^ cs;
+                    if (q > r) {
+                        const bool desc = (((lane * R + r) & size) == 0);
+                        const uint32_t hi = max(v[r], v[q]), lo = min(v[r], v[q]);
+                        v[r] = desc ? hi : lo;
+                        v[q] = desc ? lo : hi;
                     }
                 }
             }
         }
     }
+}
+
+// Warp bitonic sort, descending. The stages are looped, not unrolled: the
+// encoder's other phases already fill the instruction caches.
+template <int R>
+__device__ __forceinline__ void warp_sort_desc(uint32_t (&v)[R]) {
+#pragma unroll 1
+    for (int size = 2; size <= 32 * R; size <<= 1)
+#pragma unroll 1
+        for (int stride = size / 2; stride > 0; stride >>= 1) sort_stage<R>(v, size, stride);
 }
 
 __device__ __forceinline__ void cas_desc(uint64_t &a, uint64_t &b) {
@@ -564,6 +566,7 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
             uint64_t *Lt = codes + tk * k;
             uint32_t *bt = beams + tk * kBeam;
             bool done = false;
+            // each lane keeps R words, so the union of 32 R holds at least 2 k
             if (!a.mu && KPL <= 4) done = level0_union<(KPL <= 2 ? 4 : 8), KPL>(wv, nch, k, E, a.ecap, Lt, bt);
             if (!done)
                 level0_bisect(a, xh + tk * nblk * 32, reinterpret_cast<float *>(E),
