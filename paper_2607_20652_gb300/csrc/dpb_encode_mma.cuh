@@ -322,31 +322,30 @@ __device__ __forceinline__ int merge_entrants(uint64_t *L, int k, uint64_t *E, c
 
 // ---- level 0 ----------------------------------------------------------------------
 
-// Fast path (no standardisation, k <= 16 R): see the header comment. `wv`
-// holds the words of this lane's coordinates (16-byte chunk lane + 32 j,
-// element e; 0 where the chunk lies past the row). The union's first k go to
-// the list; coordinates that reach its k-th word without being among their
-// lane's R kept words are merged in afterwards. Returns false, with nothing
-// written, when more of them arrive than the scratch holds.
+// Fast path (no standardisation, k <= 16 R): see the header comment. `row`
+// is the token's row as 16-byte chunks (8 coordinates each); this lane reads
+// chunks lane + 32 j (again from L1 in the later passes). The union's first k
+// go to the list; coordinates that reach its k-th word without being among
+// their lane's R kept words are merged in afterwards. Returns false, with
+// nothing written, when more of them arrive than the scratch holds.
 template <int R, int KPL>
-__device__ __forceinline__ bool level0_union(const uint32_t (&wv)[4][8], int nch, int k, uint64_t *E, int ecap,
-                                             uint64_t *L, uint32_t *beam) {
+__device__ __forceinline__ bool level0_union(const uint4 *row, int nch, int k, uint64_t *E, int ecap, uint64_t *L,
+                                             uint32_t *beam) {
     const int lane = threadIdx.x & 31;
     uint32_t top[R];
 #pragma unroll
     for (int r = 0; r < R; ++r) top[r] = 0u;
+#pragma unroll 1
+    for (int ch = lane; ch < nch; ch += 32) {
+        const uint4 v = row[ch];
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-        if (lane + 32 * j < nch) {
+        for (int e = 0; e < 8; ++e) {
+            uint32_t c = cword0(elem16(v, e), (uint32_t)(8 * ch + e));
 #pragma unroll
-            for (int e = 0; e < 8; ++e) {
-                uint32_t c = wv[j][e];
-#pragma unroll
-                for (int r = 0; r < R; ++r) {
-                    const uint32_t hi = max(top[r], c);
-                    c = min(top[r], c);
-                    top[r] = hi;
-                }
+            for (int r = 0; r < R; ++r) {
+                const uint32_t hi = max(top[r], c);
+                c = min(top[r], c);
+                top[r] = hi;
             }
         }
     }
@@ -358,11 +357,15 @@ __device__ __forceinline__ bool level0_union(const uint32_t (&wv)[4][8], int nch
         if (r == (k - 1) % R) mine = top[r];
     const uint32_t tau = __shfl_sync(kFull, mine, (k - 1) / R);
     int nx = 0;
+#pragma unroll 1
+    for (int ch = lane; ch < nch; ch += 32) {
+        const uint4 v = row[ch];
 #pragma unroll
-    for (int j = 0; j < 4; ++j)
-        if (lane + 32 * j < nch)
-#pragma unroll
-            for (int e = 0; e < 8; ++e) nx += (wv[j][e] >= tau) & (wv[j][e] < kept_min);
+        for (int e = 0; e < 8; ++e) {
+            const uint32_t w = cword0(elem16(v, e), (uint32_t)(8 * ch + e));
+            nx += (w >= tau) & (w < kept_min);
+        }
+    }
     const int total = __reduce_add_sync(kFull, nx);
     if (total > ecap) return false;
 #pragma unroll
@@ -378,12 +381,15 @@ __device__ __forceinline__ bool level0_union(const uint32_t (&wv)[4][8], int nch
             if (lane >= o) off += v;
         }
         off -= nx;
+#pragma unroll 1
+        for (int ch = lane; ch < nch; ch += 32) {
+            const uint4 v = row[ch];
 #pragma unroll
-        for (int j = 0; j < 4; ++j)
-            if (lane + 32 * j < nch)
-#pragma unroll
-                for (int e = 0; e < 8; ++e)
-                    if (wv[j][e] >= tau && wv[j][e] < kept_min) E[off++] = widen0(wv[j][e]);
+            for (int e = 0; e < 8; ++e) {
+                const uint32_t w = cword0(elem16(v, e), (uint32_t)(8 * ch + e));
+                if (w >= tau && w < kept_min) E[off++] = widen0(w);
+            }
+        }
         __syncwarp();
         merge_sorted<KPL>(L, k, E, total, nullptr);
         if (lane < kBeam) beam[lane] = cword_idx(L[lane]);
@@ -540,24 +546,17 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
         // ---- each row into the permuted tile; |x|; level 0 ----
         for (int tk = 0; tk < ntok; ++tk) {
             const uint4 *row = reinterpret_cast<const uint4 *>(a.x + (t0 + tk) * d);
-            uint32_t wv[4][8];  // level-0 words of this lane's coordinates
             float ss = 0.f;
+#pragma unroll 1
+            for (int ch = lane; ch < nch; ch += 32) {
+                const uint4 v = row[ch];
+                const int m = ch >> 2, l0 = (ch & 3) * 8, half = l0 >> 4, pb = (l0 & 15) >> 2;
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                const int ch = lane + 32 * j;
-#pragma unroll
-                for (int e = 0; e < 8; ++e) wv[j][e] = 0u;
-                if (ch < nch) {
-                    const uint4 v = row[ch];
-                    const int m = ch >> 2, l0 = (ch & 3) * 8, half = l0 >> 4, pb = (l0 & 15) >> 2;
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        const uint32_t bits = elem16(v, e);
-                        xh[(tk * nblk * 16 + m * 16 + (e & 3) * 4 + pb + (e >> 2)) * 2 + half] = (uint16_t)bits;
-                        const float xf = __uint_as_float(bits << 16);
-                        ss = fmaf(xf, xf, ss);
-                        wv[j][e] = cword0(bits, (uint32_t)(8 * ch + e));
-                    }
+                for (int e = 0; e < 8; ++e) {
+                    const uint32_t bits = elem16(v, e);
+                    xh[(tk * nblk * 16 + m * 16 + (e & 3) * 4 + pb + (e >> 2)) * 2 + half] = (uint16_t)bits;
+                    const float xf = __uint_as_float(bits << 16);
+                    ss = fmaf(xf, xf, ss);
                 }
             }
             ss = warp_sum(ss);
@@ -567,7 +566,7 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
             uint32_t *bt = beams + tk * kBeam;
             bool done = false;
             // each lane keeps R words, so the union of 32 R holds at least 2 k
-            if (!a.mu && KPL <= 4) done = level0_union<(KPL <= 2 ? 4 : 8), KPL>(wv, nch, k, E, a.ecap, Lt, bt);
+            if (!a.mu && KPL <= 4) done = level0_union<(KPL <= 2 ? 4 : 8), KPL>(row, nch, k, E, a.ecap, Lt, bt);
             if (!done)
                 level0_bisect(a, xh + tk * nblk * 32, reinterpret_cast<float *>(E),
                               reinterpret_cast<uint32_t *>(E) + a.ecap, a.ecap, Lt, bt);
