@@ -71,6 +71,7 @@ typedef enum { DPB_SELECT_GLOBAL = 0, DPB_SELECT_PER_LEVEL = 1 } dpb_select;
 #define DPB_DEV_BAD_INDEX 0x1   /* an idx outside [0, 2^N) was skipped        */
 #define DPB_DEV_BAD_SIGMA 0x2   /* a sigma <= 0 or non-finite was met         */
 #define DPB_DEV_SHORT_CODE 0x4  /* fewer than k distinct candidates were seen */
+#define DPB_DEV_TIMEOUT 0x8     /* a bounded wait inside a kernel gave up      */
 
 /*
  * Configuration (§2.2 and App. G). Zero-valued optional fields are derived:

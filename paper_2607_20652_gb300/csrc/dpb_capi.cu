@@ -75,7 +75,9 @@ dpb_status dpb_plan_create(const dpb_config *cfg, const uint32_t *generators, dp
         delete p;
         return s;
     }
-    const size_t smem = dpb::encode_smem_header(p) + dpb::encode_smem_per_warp(p);
+    const size_t smem = p->cfg.select_mode == DPB_SELECT_GLOBAL
+                            ? dpb::encode_smem_header(p) + dpb::encode_smem_per_warp(p)
+                            : dpb::encode_pl_smem(p);
     if (smem > 200 * 1024) {
         delete p;
         return dpb::fail(DPB_ERR_UNSUPPORTED, "encoder needs %zu bytes of shared memory per warp", smem);
@@ -95,7 +97,8 @@ dpb_status dpb_plan_create(const dpb_config *cfg, const uint32_t *generators, dp
     struct Up {
         uint32_t **dst;
         const std::vector<uint32_t> *src;
-    } ups[] = {{&p->dM, &p->M}, {&p->dG, &p->G}, {&p->dVH, &p->VH}, {&p->dFRAG, &p->FRAG}, {&p->dDD, &p->DD}};
+    } ups[] = {{&p->dM, &p->M}, {&p->dG, &p->G}, {&p->dVH, &p->VH}, {&p->dFRAG, &p->FRAG}, {&p->dDD, &p->DD},
+                {&p->dGT, &p->GT},     {&p->dVH2, &p->VH2}};
     for (const Up &u : ups) {
         if (u.src->empty()) continue;
         const size_t bytes = sizeof(uint32_t) * u.src->size();
@@ -128,6 +131,8 @@ dpb_status dpb_plan_destroy(dpb_plan *plan) {
     cudaFree(plan->dVH);
     cudaFree(plan->dFRAG);
     cudaFree(plan->dDD);
+    cudaFree(plan->dGT);
+    cudaFree(plan->dVH2);
     if (cur >= 0 && cur != plan->device) cudaSetDevice(cur);
     delete plan;
     return DPB_OK;

@@ -213,6 +213,9 @@ size_t encode_smem_per_warp(const dpb_plan *p) {
 cudaError_t launch_encode(const dpb_plan *p, const void *x, int64_t T, const float *mu,
                           const float *sigma, int32_t *idx, float *val, float *xnorm,
                           int32_t *status, cudaStream_t stream) {
+    // the paper's per-level selection: tcgen05 scoring
+    if (p->cfg.select_mode == DPB_SELECT_PER_LEVEL)
+        return launch_encode_pl(p, x, T, mu, sigma, idx, val, xnorm, status, stream);
     // bf16 rows on 16-byte boundaries, beam 8, 16 children: tensor-core scoring
     if (p->mma_encode && (reinterpret_cast<uintptr_t>(x) & 15u) == 0)
         return launch_encode_mma(p, x, T, mu, sigma, idx, val, xnorm, status, stream);

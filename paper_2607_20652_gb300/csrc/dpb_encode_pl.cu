@@ -1,0 +1,562 @@
+// dpb_encode_pl.cu -- the paper's per-level encoder (§2.2 and the per-level
+// configuration table of App. G): level 0 keeps its top K_0 coordinates;
+// level l scores the Delta_l children p ^ g_j of every index kept at level
+// l-1 and keeps its top K_l distinct children; the code is every level's kept
+// set, level by level, each in (|z| descending, index ascending) order.
+//
+// Child scoring (Eq. 6) runs on the tcgen05 tensor cores. A block of 4 warps
+// owns 4 tokens. At level l its 128 tensor-core rows are (token, parent
+// slot), 32 slots per token, and its Delta_l columns the level's generators,
+// so one tcgen05.mma of M = 128, N = Delta_l, K = 16 scores 128 x Delta_l
+// children at once; K runs over d in chunks of 64 coordinates, double
+// buffered:
+//  - A (128 x 64 bf16) is built in shared memory by the block's threads,
+//    each writing its row x (.) phi~_parent: the token's x pairs XOR the
+//    parent's sign bits (App. A.4 Eq. 26 tables), in the K-major core-matrix
+//    layout with the K order permuted so that K positions (2i, 2i+1) of a
+//    32-coordinate block hold coordinates (i, i + 16), whose sign bits one
+//    shift moves to the bf16 sign positions;
+//  - B (Delta_l x 64 bf16, the generators' +-1 signs in the same order) is
+//    one bulk copy of the plan's precomputed tile;
+//  - one thread issues the 4 MMAs of the chunk and commits them to an
+//    mbarrier that frees the chunk's buffers; scores accumulate in TMEM.
+// Every mbarrier wait is bounded; a wait that gives up sets
+// DPB_DEV_TIMEOUT, and the block drains its MMAs and frees its TMEM.
+//
+// Selection of a level (one warp per token, lane = parent slot): each lane
+// keeps the 4 largest keys |z| of its row, the warp sorts the union and takes
+// a threshold tau at rank K + K/2 of it; every candidate at or above tau is
+// gathered (a count pass, a prefix sum and a write pass), sorted, and its
+// repeated indices (two parents can share a child) are dropped. When K
+// distinct candidates reach tau they are exactly the level's top K.
+#include <algorithm>
+
+#include "dpb_encode_mma.cuh"
+#include "dpb_internal.h"
+
+namespace dpb {
+
+namespace {
+
+constexpr int kTokens = 4;      // tokens per block, one per warp
+constexpr int kRows = 32;       // tensor-core rows per token (parent slots)
+constexpr int kChunk = 64;      // coordinates per K chunk
+constexpr int kATile = 128 * kChunk * 2;
+constexpr int kSelCap = 256;    // gathered candidates per token and level
+constexpr int kMaxK = 64;       // K_l per level
+constexpr uint32_t kSpin = 1u << 20;  // bound of every mbarrier wait
+// at least this much shared memory per block, so that at most two blocks (2 x
+// 256 TMEM columns) share an SM
+constexpr int kMinSmem = 80 * 1024;
+
+struct Args {
+    const __nv_bfloat16 *x;
+    int64_t T;
+    const float *mu, *sigma;
+    int32_t *idx;
+    float *val, *xnorm;
+    int32_t *status;
+    const uint32_t *GT, *G, *VH2;
+    int d, nblk, levels, t, kvh, code_len, dmax;
+    int kl[DPB_MAX_LEVELS], delta[DPB_MAX_LEVELS], off[DPB_MAX_LEVELS];
+    int64_t gt_off[DPB_MAX_LEVELS];
+    float inv_sqrt_d;
+};
+
+// ---- layout --------------------------------------------------------------------
+
+constexpr int kWarpBytes = 4 * kRows /* parents */ + 4 * kSelCap /* z */ + 4 * kSelCap /* index */;
+
+struct Layout {
+    int a, b, xw, vh, g, w5, warps, mbar, total;
+};
+
+__host__ __device__ inline Layout layout(int d, int levels, int kvh, int dmax) {
+    const int nblk = d / 32;
+    Layout l;
+    l.a = 0;
+    l.b = l.a + 2 * kATile;
+    l.xw = l.b + 2 * dmax * 128;
+    l.vh = l.xw + kTokens * nblk * 16 * 4;
+    l.g = l.vh + kvh * nblk * 32 * 4;
+    l.w5 = l.g + levels * 256 * 4;
+    l.warps = l.w5 + 32 * 4;
+    l.mbar = l.warps + kTokens * kWarpBytes;
+    l.total = l.mbar + 4 * 8 + 16;
+    return l;
+}
+
+// ---- PTX wrappers ----------------------------------------------------------------
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ bool mbar_wait(uint32_t mbar, uint32_t parity) {
+    for (uint32_t i = 0; i < kSpin; ++i) {
+        uint32_t done;
+        asm volatile(
+            "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+            : "=r"(done)
+            : "r"(mbar), "r"(parity)
+            : "memory");
+        if (done) return true;
+    }
+    return false;
+}
+
+// Shared-memory matrix descriptor: K-major, no swizzle, 16-byte core-matrix
+// rows, 128 bytes between core matrices along K, 1024 between 8-row groups.
+__device__ __forceinline__ uint64_t tile_desc(uint32_t saddr) {
+    return (uint64_t)((saddr >> 4) & 0x3FFFu) | ((uint64_t)(128 >> 4) << 16) | ((uint64_t)(1024 >> 4) << 32) |
+           ((uint64_t)1 << 46);
+}
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,"
+        "%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
+          "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15]),
+          "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]),
+          "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// ---- selection ---------------------------------------------------------------------
+
+struct WarpBufs {
+    uint32_t *par;   // [32] parents of the next level
+    float *z;        // [kSelCap]
+    uint32_t *id;    // [kSelCap]
+};
+
+// The top K distinct candidates of one token, as explained in the header.
+// `scan(f)` calls f(z, index, live) for every candidate of this lane, in the
+// same order each time. Writes code columns [col, col + K) of row `tok` and,
+// when `par_out`, the K indices as the next level's parents. Returns the
+// number of distinct candidates written (< K only with the status bit set).
+template <class Scan>
+__device__ __forceinline__ int select_level(Scan scan, int nlive, int K, const WarpBufs &w, const Args &a,
+                                            int64_t tok, int col, bool par_out) {
+    const int lane = threadIdx.x & 31;
+    uint32_t top[4] = {0u, 0u, 0u, 0u};
+    scan([&](float z, uint32_t, bool live) {
+        uint32_t c = live ? akey(z) + 1u : 0u;
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+            const uint32_t hi = max(top[r], c);
+            c = min(top[r], c);
+            top[r] = hi;
+        }
+    });
+    mmaenc::warp_sort_desc<4>(top);
+    const int nunion = min(4 * nlive, 128);
+    int n = 0, distinct = 0;
+    // the threshold's rank in the union: K + K/2 first; K when too many
+    // candidates reach it; the union's last when repeats leave fewer than K
+    int rank = min(K + K / 2, nunion);
+    for (int attempt = 0; attempt < 3; ++attempt) {
+        uint32_t mine = 0u;
+#pragma unroll
+        for (int r = 0; r < 4; ++r)
+            if (r == (rank - 1) % 4) mine = top[r];
+        uint32_t tau = __shfl_sync(kFull, mine, (rank - 1) / 4);
+        if (tau == 0u) tau = 1u;
+        int cnt = 0;
+        scan([&](float z, uint32_t, bool live) { cnt += live && akey(z) + 1u >= tau; });
+        n = __reduce_add_sync(kFull, cnt);
+        if (n > kSelCap) {
+            if (rank > K) {  // a tighter threshold
+                rank = min(K, nunion);
+                continue;
+            }
+            set_status(a.status, DPB_DEV_SHORT_CODE);
+            n = kSelCap;
+        }
+        int off = cnt;  // exclusive prefix over the lanes
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int v = __shfl_up_sync(kFull, off, o);
+            if (lane >= o) off += v;
+        }
+        off -= cnt;
+        scan([&](float z, uint32_t ci, bool live) {
+            if (live && akey(z) + 1u >= tau) {
+                if (off < kSelCap) {
+                    w.z[off] = z;
+                    w.id[off] = ci;
+                }
+                ++off;
+            }
+        });
+        __syncwarp();
+        int cap = 32;
+        while (cap < n) cap <<= 1;
+        warp_sort(w.z, w.id, n, cap);
+        // repeated indices are adjacent (equal candidates score equally)
+        distinct = 0;
+        for (int e0 = 0; e0 < n; e0 += 32) {
+            const int e = e0 + lane;
+            const bool keep = e < n && (e == 0 || w.id[e] != w.id[e - 1]);
+            const unsigned mb = __ballot_sync(kFull, keep);
+            const float zv = keep ? w.z[e] : 0.f;
+            const uint32_t iv = keep ? w.id[e] : 0u;
+            __syncwarp();
+            if (keep) {
+                const int pos = distinct + __popc(mb & mmaenc::lanes_below());
+                w.z[pos] = zv;
+                w.id[pos] = iv;
+            }
+            distinct += __popc(mb);
+            __syncwarp();
+        }
+        if (distinct >= K || rank >= nunion) break;
+        rank = nunion;  // repeats took the margin: the loosest threshold
+    }
+    if (distinct < K) set_status(a.status, DPB_DEV_SHORT_CODE);
+    for (int e = lane; e < K; e += 32) {
+        const bool ok = e < distinct;
+        a.idx[tok * a.code_len + col + e] = ok ? (int32_t)w.id[e] : 0;
+        a.val[tok * a.code_len + col + e] = ok ? w.z[e] : 0.f;
+    }
+    __syncwarp();
+    if (par_out) w.par[lane] = lane < min(K, distinct) ? w.id[lane] : 0u;
+    __syncwarp();
+    return distinct;
+}
+
+__device__ __forceinline__ float standardise(float s, uint32_t c, const float *mu, const float *sigma,
+                                             int32_t *status) {
+    if (!mu) return s;
+    const float sd = sigma[c];
+    if (status && !(sd > 0.f)) set_status(status, DPB_DEV_BAD_SIGMA);
+    return (s - mu[c]) / sd;
+}
+
+// ---- the kernel ----------------------------------------------------------------------
+
+__global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
+    extern __shared__ __align__(1024) uint8_t smem[];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int d = a.d, nblk = a.nblk, L = a.levels;
+    const Layout lay = layout(d, L, a.kvh, a.dmax);
+    uint8_t *sA = smem + lay.a;
+    uint8_t *sB = smem + lay.b;
+    uint32_t *xw = reinterpret_cast<uint32_t *>(smem + lay.xw);
+    uint32_t *vh = reinterpret_cast<uint32_t *>(smem + lay.vh);
+    uint32_t *gs = reinterpret_cast<uint32_t *>(smem + lay.g);
+    uint32_t *w5 = reinterpret_cast<uint32_t *>(smem + lay.w5);
+    uint64_t *mbar = reinterpret_cast<uint64_t *>(smem + lay.mbar);  // full_b[2], mma_done[2]
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(mbar + 4);
+    WarpBufs wb;
+    {
+        uint8_t *base = smem + lay.warps + warp * kWarpBytes;
+        wb.par = reinterpret_cast<uint32_t *>(base);
+        wb.z = reinterpret_cast<float *>(base + 4 * kRows);
+        wb.id = reinterpret_cast<uint32_t *>(base + 4 * kRows + 4 * kSelCap);
+    }
+    for (int i = tid; i < a.kvh * nblk * 32; i += blockDim.x) vh[i] = a.VH2[i];
+    for (int i = tid; i < L * 256; i += blockDim.x) gs[i] = a.G[(i >> 8) * DPB_MAX_CHILDREN + (i & 255)];
+    if (tid < 32) {
+        uint32_t word = 0;
+        for (int l = 0; l < 32; ++l) word |= (uint32_t)(__popc(l & tid) & 1) << l;
+        w5[tid] = word;
+    }
+    if (tid == 0) {
+        for (int i = 0; i < 4; ++i) asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(mbar + i)));
+        asm volatile("fence.mbarrier_init.release.cluster;");
+    }
+    if (warp == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 256;" ::"r"(smem_u32(tmem_slot)));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;");
+    const uint32_t tmem = *tmem_slot;
+    const uint32_t full_b[2] = {smem_u32(mbar), smem_u32(mbar + 1)};
+    const uint32_t mma_done[2] = {smem_u32(mbar + 2), smem_u32(mbar + 3)};
+    uint32_t issued[2] = {0u, 0u}, waited[2] = {0u, 0u}, bcopies[2] = {0u, 0u};
+    bool failed = false;
+    const uint32_t lo_mask = (1u << a.t) - 1u;
+    const int64_t ngroups = (a.T + kTokens - 1) / kTokens;
+    uint16_t *xh = reinterpret_cast<uint16_t *>(xw + warp * nblk * 16);
+
+    for (int64_t grp = blockIdx.x; grp < ngroups && !failed; grp += gridDim.x) {
+        const int64_t tok = grp * kTokens + warp;
+        const bool live = tok < a.T;
+        // ---- the row in the pair layout: word m*16 + i = (x[32m+i], x[32m+i+16]); |x|; level 0 ----
+        if (live) {
+            const uint4 *row = reinterpret_cast<const uint4 *>(a.x + tok * d);
+            float ss = 0.f;
+            for (int ch = lane; ch < d / 8; ch += 32) {
+                const uint4 v = row[ch];
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    const uint32_t bits = mmaenc::elem16(v, e);
+                    const int cd = 8 * ch + e, m = cd >> 5, wl = cd & 31;
+                    xh[(m * 16 + (wl & 15)) * 2 + (wl >> 4)] = (uint16_t)bits;
+                    const float xf = __uint_as_float(bits << 16);
+                    ss = fmaf(xf, xf, ss);
+                }
+            }
+            ss = warp_sum(ss);
+            if (lane == 0 && a.xnorm) a.xnorm[tok] = sqrtf(ss);
+            __syncwarp();
+            auto scan0 = [&](auto f) {
+                for (int i = lane; i < d; i += 32) {
+                    const int m = i >> 5, wl = i & 31;
+                    const float xv = __uint_as_float((uint32_t)xh[(m * 16 + (wl & 15)) * 2 + (wl >> 4)] << 16);
+                    f(standardise(xv, (uint32_t)i, a.mu, a.sigma, nullptr), (uint32_t)i, true);
+                }
+            };
+            if (a.mu)
+                for (int i = lane; i < d; i += 32) standardise(0.f, (uint32_t)i, a.mu, a.sigma, a.status);
+            select_level(scan0, min(32, d / 32 * 32), a.kl[0], wb, a, tok, a.off[0], L > 1);
+        } else {
+            wb.par[lane] = 0u;
+            __syncwarp();
+        }
+        __syncthreads();
+
+        for (int l = 1; l < L && !failed; ++l) {
+            const int P = a.kl[l - 1], D = a.delta[l], nch = d / kChunk;
+            const bool rv = live && lane < P;
+            const uint32_t p = rv ? wb.par[lane] : 0u;
+            const uint32_t w5p = w5[p & 31u], u = (p & lo_mask) >> 5;
+            uint32_t hv[4];  // the 5-bit chunks of p's high half
+#pragma unroll
+            for (int k = 0; k < 4; ++k) hv[k] = (p >> min(a.t + 5 * k, 31)) & 31u;
+            const uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(D >> 3) << 17) | (8u << 24);
+            const uint32_t *xt = xw + warp * nblk * 16;
+            const uint32_t *gt = a.GT + a.gt_off[l];
+            for (int c = 0; c < nch; ++c) {
+                const int s = c & 1;
+                if (issued[s] > waited[s]) {  // the MMAs that last read this stage
+                    const bool ok = mbar_wait(mma_done[s], waited[s] & 1u);
+                    if (__syncthreads_or(!ok)) {  // every thread leaves together
+                        failed = true;
+                        break;
+                    }
+                    ++waited[s];
+                }
+                uint8_t *At = sA + s * kATile;
+                uint8_t *Bt = sB + s * a.dmax * 128;
+                if (tid == 0) {
+                    const uint32_t bytes = (uint32_t)D * 128u;
+                    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(full_b[s]), "r"(bytes)
+                                 : "memory");
+                    asm volatile(
+                        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                            smem_u32(Bt)),
+                        "l"(gt + (int64_t)c * D * 32), "r"(bytes), "r"(full_b[s])
+                        : "memory");
+                }
+#pragma unroll
+                for (int b = 0; b < 2; ++b) {
+                    const int m = 2 * c + b;
+                    uint32_t sw = w5p ^ (0u - (uint32_t)(__popc((uint32_t)m & u) & 1));
+#pragma unroll
+                    for (int k = 0; k < 4; ++k)
+                        if (k < a.kvh) sw ^= vh[(k * nblk + m) * 32 + hv[k]];
+                    const uint4 *xs = reinterpret_cast<const uint4 *>(xt + m * 16);
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        const uint4 xv = xs[q];
+                        const int sh = 15 - 4 * q;
+                        uint4 av;
+                        av.x = rv ? xv.x ^ ((sw << sh) & 0x80008000u) : 0u;
+                        av.y = rv ? xv.y ^ ((sw << (sh - 1)) & 0x80008000u) : 0u;
+                        av.z = rv ? xv.z ^ ((sw << (sh - 2)) & 0x80008000u) : 0u;
+                        av.w = rv ? xv.w ^ ((sw << (sh - 3)) & 0x80008000u) : 0u;
+                        *reinterpret_cast<uint4 *>(At + (tid >> 3) * 1024 + (4 * b + q) * 128 + (tid & 7) * 16) = av;
+                    }
+                }
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                __syncthreads();
+                if (tid == 0) {
+                    if (!mbar_wait(full_b[s], bcopies[s] & 1u)) {
+                        set_status(a.status, DPB_DEV_TIMEOUT);  // the commit below still arrives
+                    } else {
+                        asm volatile("tcgen05.fence::after_thread_sync;");
+                        const uint32_t ab = smem_u32(At), bb = smem_u32(Bt);
+#pragma unroll
+                        for (int k = 0; k < kChunk / 16; ++k) {
+                            const uint32_t acc = (c > 0 || k > 0) ? 1u : 0u;
+                            asm volatile(
+                                "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+                                "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem),
+                                "l"(tile_desc(ab + 256 * k)), "l"(tile_desc(bb + 256 * k)), "r"(idesc), "r"(acc));
+                        }
+                    }
+                    ++bcopies[s];
+                    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                        mma_done[s]));
+                }
+                ++issued[s];
+            }
+            if (failed) break;
+            {
+                const int s = (nch - 1) & 1;  // the last commit covers every MMA of the level
+                const bool ok = mbar_wait(mma_done[s], waited[s] & 1u);
+                if (__syncthreads_or(!ok)) {
+                    failed = true;
+                    break;
+                }
+                ++waited[s];
+            }
+            asm volatile("tcgen05.fence::after_thread_sync;");
+            // ---- the level's selection, one warp per token ----
+            if (live) {
+                const uint32_t taddr = tmem + ((uint32_t)(32 * warp) << 16);
+                const uint32_t *gl = gs + l * 256;
+                auto scanl = [&](auto f) {
+                    for (int c0 = 0; c0 < D; c0 += 32) {
+                        uint32_t v[32];
+                        tmem_ld32(taddr + c0, v);
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) {
+                            const uint32_t ci = p ^ gl[c0 + j];
+                            f(standardise(__uint_as_float(v[j]) * a.inv_sqrt_d, ci, a.mu, a.sigma, nullptr), ci,
+                              rv && c0 + j < D);
+                        }
+                    }
+                };
+                select_level(scanl, P, a.kl[l], wb, a, tok, a.off[l], l + 1 < L);
+            }
+            asm volatile("tcgen05.fence::before_thread_sync;");
+            __syncthreads();
+        }
+    }
+    if (failed) set_status(a.status, DPB_DEV_TIMEOUT);
+    // drain: every commit issued is waited for (bounded) before TMEM is freed
+    for (int s = 0; s < 2; ++s)
+        while (issued[s] > waited[s]) {
+            if (!mbar_wait(mma_done[s], waited[s] & 1u)) break;
+            ++waited[s];
+        }
+    asm volatile("tcgen05.fence::before_thread_sync;");
+    __syncthreads();
+    if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 256;" ::"r"(tmem));
+}
+
+}  // namespace
+
+// ---- host side ----------------------------------------------------------------------
+
+dpb_status check_per_level(const dpb_config &c) {
+    if (c.dtype != DPB_BF16) return fail(DPB_ERR_UNSUPPORTED, "per-level selection needs bf16 rows");
+    if (c.d % kChunk != 0 || c.d < kChunk || c.d > 2048)
+        return fail(DPB_ERR_UNSUPPORTED, "per-level selection needs d a multiple of 64 in [64, 2048] (d=%d)", c.d);
+    int prev = 0;
+    for (int l = 0; l < c.levels; ++l) {
+        const int K = c.k_per_level[l];
+        if (K < 1 || K > kMaxK) return fail(DPB_ERR_UNSUPPORTED, "k_per_level[%d]=%d outside [1, %d]", l, K, kMaxK);
+        if (l == 0 && K > c.d) return fail(DPB_ERR_INVALID_ARG, "k_per_level[0]=%d exceeds d=%d", K, c.d);
+        if (l >= 1) {
+            const int D = c.children[l];
+            if (D % 16 != 0 || D < 16 || D > 256)
+                return fail(DPB_ERR_UNSUPPORTED, "per-level selection needs children[%d] a multiple of 16 in [16, 256]",
+                            l);
+            if (prev > kRows)
+                return fail(DPB_ERR_UNSUPPORTED, "k_per_level[%d]=%d parents exceed %d", l - 1, prev, kRows);
+            if (K > prev * D) return fail(DPB_ERR_INVALID_ARG, "k_per_level[%d]=%d exceeds its %d candidates", l, K, prev * D);
+        }
+        prev = K;
+    }
+    return DPB_OK;
+}
+
+void build_per_level_tables(dpb_plan *p) {
+    const dpb_config &c = p->cfg;
+    const int nblk = c.d / 32, nch = c.d / kChunk;
+    auto sign = [&](uint32_t g, int iota) -> uint32_t {
+        return (__builtin_popcount(p->M[iota] & g) & 1) ? 0xBF80u : 0x3F80u;
+    };
+    // generator tiles: K position kk = 32 b + 2 i + h of chunk ch holds coordinate 32 (2 ch + b) + i + 16 h
+    std::vector<uint16_t> gt;
+    for (int l = 0; l < DPB_MAX_LEVELS; ++l) p->gt_off[l] = 0;
+    for (int l = 1; l < c.levels; ++l) {
+        const int D = c.children[l];
+        p->gt_off[l] = (int64_t)gt.size() / 2;
+        const size_t base = gt.size();
+        gt.resize(base + (size_t)nch * D * kChunk, 0);
+        const uint32_t *g = &p->G[(size_t)l * DPB_MAX_CHILDREN];
+        for (int ch = 0; ch < nch; ++ch)
+            for (int n = 0; n < D; ++n)
+                for (int kk = 0; kk < kChunk; ++kk) {
+                    const int b = kk / 32, i = (kk % 32) / 2, h = kk % 2;
+                    const int iota = 32 * (2 * ch + b) + i + 16 * h;
+                    const size_t byte = (size_t)(n / 8) * 1024 + (size_t)(kk / 8) * 128 + (n % 8) * 16 + (kk % 8) * 2;
+                    gt[base + (size_t)ch * D * kChunk + byte / 2] = (uint16_t)sign(g[n], iota);
+                }
+    }
+    p->GT.assign(gt.size() / 2, 0u);
+    for (size_t w = 0; w < p->GT.size(); ++w) p->GT[w] = (uint32_t)gt[2 * w] | ((uint32_t)gt[2 * w + 1] << 16);
+    // inverse-coordinate sign words per 32-coordinate block (any d <= 2048)
+    const int kvh = std::max(1, (c.field_t + 4) / 5);
+    p->VH2.assign((size_t)kvh * nblk * 32, 0u);
+    for (int k = 0; k < kvh; ++k)
+        for (int q = 0; q < nblk; ++q)
+            for (int v = 0; v < 32; ++v) {
+                uint32_t w = 0;
+                const uint32_t mask = (uint32_t)v << (5 * k);
+                for (int l = 0; l < 32; ++l) {
+                    const uint32_t kappa = p->M[32 * q + l] >> c.field_t;
+                    w |= (uint32_t)(__builtin_popcount(kappa & mask) & 1) << l;
+                }
+                p->VH2[((size_t)k * nblk + q) * 32 + v] = w;
+            }
+}
+
+size_t encode_pl_smem(const dpb_plan *p) {
+    const dpb_config &c = p->cfg;
+    int dmax = 16;
+    for (int l = 1; l < c.levels; ++l) dmax = std::max(dmax, c.children[l]);
+    const int kvh = std::max(1, (c.field_t + 4) / 5);
+    return (size_t)std::max(layout(c.d, c.levels, kvh, dmax).total, kMinSmem);
+}
+
+cudaError_t launch_encode_pl(const dpb_plan *p, const void *x, int64_t T, const float *mu, const float *sigma,
+                             int32_t *idx, float *val, float *xnorm, int32_t *status, cudaStream_t stream) {
+    const dpb_config &c = p->cfg;
+    Args a{};
+    a.x = static_cast<const __nv_bfloat16 *>(x);
+    a.T = T;
+    a.mu = mu;
+    a.sigma = sigma;
+    a.idx = idx;
+    a.val = val;
+    a.xnorm = xnorm;
+    a.status = status;
+    a.GT = p->dGT;
+    a.G = p->dG;
+    a.VH2 = p->dVH2;
+    a.d = c.d;
+    a.nblk = c.d / 32;
+    a.levels = c.levels;
+    a.t = c.field_t;
+    a.kvh = std::max(1, (c.field_t + 4) / 5);
+    a.code_len = p->code_len;
+    a.dmax = 16;
+    int off = 0;
+    for (int l = 0; l < c.levels; ++l) {
+        a.kl[l] = c.k_per_level[l];
+        a.delta[l] = l ? c.children[l] : 0;
+        a.off[l] = off;
+        off += c.k_per_level[l];
+        a.gt_off[l] = p->gt_off[l];
+        if (l) a.dmax = std::max(a.dmax, c.children[l]);
+    }
+    a.inv_sqrt_d = p->inv_sqrt_d;
+    const size_t smem = encode_pl_smem(p);
+    const cudaError_t e = cudaFuncSetAttribute(encode_pl_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    int sms = 0;
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, p->device);
+    const int64_t groups = (T + kTokens - 1) / kTokens;
+    const int grid = (int)std::min<int64_t>(groups, (int64_t)std::max(sms, 1));
+    encode_pl_kernel<<<grid, kTokens * 32, smem, stream>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace dpb

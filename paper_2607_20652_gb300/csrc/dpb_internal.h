@@ -32,11 +32,24 @@ struct dpb_plan {
     bool mma_encode = false;
     std::vector<uint32_t> FRAG;
     std::vector<uint32_t> DD;
+    // Per-level (tensor-core) encoder tables, built for DPB_SELECT_PER_LEVEL:
+    //  GT: every level's generator signs gamma_j as bf16 +-1, per 64-coordinate
+    //    chunk a [Delta_l][64] tile in the K-major core-matrix layout of
+    //    tcgen05 (8 x 16-byte core matrices; element (n, kk) at byte
+    //    (n / 8) 1024 + (kk / 8) 128 + (n % 8) 16 + (kk % 8) 2), where K
+    //    position kk = 32 b + 2 i + h of the chunk holds coordinate
+    //    32 (2 c + b) + i + 16 h; level l starts at word gt_off[l];
+    //  VH2[k][q][v]: as VH, for every 32-coordinate block of d <= 2048.
+    std::vector<uint32_t> GT;
+    std::vector<uint32_t> VH2;
+    int64_t gt_off[DPB_MAX_LEVELS] = {};
     uint32_t *dM = nullptr;     // device copy of M
     uint32_t *dG = nullptr;     // device copy of G
     uint32_t *dVH = nullptr;    // device copy of VH
     uint32_t *dFRAG = nullptr;  // device copy of FRAG
     uint32_t *dDD = nullptr;    // device copy of DD
+    uint32_t *dGT = nullptr;    // device copy of GT
+    uint32_t *dVH2 = nullptr;   // device copy of VH2
 };
 
 namespace dpb {
@@ -54,6 +67,13 @@ __host__ __device__ inline int frag_coord(int q4, int pair, int half) { return q
 
 // Builds the tensor-core encoder tables when the plan qualifies (dpb_plan.cu).
 void build_mma_tables(dpb_plan *p);
+
+// Per-level encoder (dpb_encode_pl.cu): support check, tables, launch.
+dpb_status check_per_level(const dpb_config &c);
+void build_per_level_tables(dpb_plan *p);
+size_t encode_pl_smem(const dpb_plan *p);
+cudaError_t launch_encode_pl(const dpb_plan *p, const void *x, int64_t T, const float *mu, const float *sigma,
+                             int32_t *idx, float *val, float *xnorm, int32_t *status, cudaStream_t stream);
 
 // Launch shape of the tensor-core encoder: the most warps per block (16, 12,
 // 8 or 4) whose shared memory fits, or 0 if none does; and that memory.

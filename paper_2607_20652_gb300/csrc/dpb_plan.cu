@@ -253,7 +253,10 @@ dpb_status resolve_and_build(const dpb_config *in, const uint32_t *generators, d
         if (c.k > c.d) return fail(DPB_ERR_INVALID_ARG, "k=%d exceeds d=%d", c.k, c.d);
         p->code_len = c.k;
     } else if (c.select_mode == DPB_SELECT_PER_LEVEL) {
-        return fail(DPB_ERR_UNSUPPORTED, "per-level selection is not built yet");
+        const dpb_status st = check_per_level(c);
+        if (st != DPB_OK) return st;
+        p->code_len = 0;
+        for (int l = 0; l < c.levels; ++l) p->code_len += c.k_per_level[l];
     } else {
         return fail(DPB_ERR_INVALID_ARG, "unknown select_mode %d", c.select_mode);
     }
@@ -311,6 +314,7 @@ dpb_status resolve_and_build(const dpb_config *in, const uint32_t *generators, d
     }
     p->cfg = c;
     build_mma_tables(p);
+    if (c.select_mode == DPB_SELECT_PER_LEVEL) build_per_level_tables(p);
     p->t = c.field_t;
     p->poly = c.field_poly;
     p->m_mask = (N >= 32) ? 0xffffffffu : ((1u << N) - 1u);

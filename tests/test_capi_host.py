@@ -104,3 +104,29 @@ def test_invalid_configs_are_rejected(lib, kw, status):
     with pytest.raises(dpb.DPBError) as e:
         dpb.Plan(**args)
     assert e.value.status == status
+
+
+@pytest.mark.parametrize("kw,status", [
+    (dict(dtype="f32"), 2),                                   # per-level scoring needs bf16 rows
+    (dict(d=96, bits=[7, 10, 12]), 2),                        # d a multiple of 64
+    (dict(children=[0, 24, 32]), 2),                          # Delta_l a multiple of 16
+    (dict(k_per_level=[40, 8, 8]), 2),                        # at most 32 parents per token
+    (dict(k_per_level=[4, 65, 8]), 2),                        # K_l at most 64
+    (dict(k_per_level=[65, 8, 8], d=64), 2),                  # K_0 beyond [1, 64]
+    (dict(k_per_level=[2, 40, 8], children=[0, 16, 32]), 1),  # 40 of 2 x 16 candidates
+])
+def test_per_level_configs_are_checked(lib, kw, status):
+    args = dict(d=64, levels=3, bits=[6, 9, 12], children=[0, 16, 32], dtype="bf16",
+                select_mode=dpb.SELECT_PER_LEVEL, k_per_level=[4, 8, 8])
+    args.update(kw)
+    with pytest.raises(dpb.DPBError) as e:
+        dpb.Plan(**args)
+    assert e.value.status == status
+
+
+def test_per_level_code_length(lib):
+    # the paper's 3L layout (App. G): K = 16, 32, 64 over 2^10, 2^15, 2^17 indices
+    plan = dpb.Plan(d=1024, levels=3, bits=[10, 15, 17], children=[0, 256, 256], dtype="bf16",
+                    select_mode=dpb.SELECT_PER_LEVEL, k_per_level=[16, 32, 64])
+    assert plan.code_len == 112
+    assert plan.config["select_mode"] == dpb.SELECT_PER_LEVEL

@@ -1,0 +1,131 @@
+"""Per-level selection (the paper's form, §2.2 with the per-level table of
+App. G) on the GPU, whose child scores run on the tcgen05 tensor cores,
+against the oracle's per-level encoder on the same seeded inputs.
+
+Each level's segment of the code must hold the same indices as the oracle's
+(tokens with a near-tie at some cut excepted and counted), in
+(|val| descending, index ascending) order, with coefficients within 1e-5 |x|;
+decode and backward run on the GPU's own code against the oracle.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2607_20652_gb300 import build, dpb, inputs
+from tests import parity
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _library():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    build.build()
+    dpb.load()
+
+
+def _plan_ref(d, bits, children, kls, **kw):
+    plan = dpb.Plan(d=d, levels=len(bits), bits=bits, children=children, dtype="bf16",
+                    select_mode=dpb.SELECT_PER_LEVEL, k_per_level=kls, **kw)
+    c = plan.config
+    ref = oracle.resolve(d=d, m_bits=bits[-1], levels=len(bits), children=children, beam=1, k=1,
+                         seed=c["generator_seed"], norm_match=c["norm_match"], t=c["field_t"],
+                         poly=c["field_poly"], bits=bits, k_per_level=kls)
+    return plan, ref
+
+
+def _gpu(plan, x_np, mu=None, sigma=None, gy_np=None):
+    dev = torch.device("cuda")
+    x = torch.from_numpy(np.ascontiguousarray(x_np)).to(dev).to(torch.bfloat16)
+    ws = plan.workspace(len(x), dev)
+    mu_t = None if mu is None else torch.from_numpy(mu.astype(np.float32)).to(dev)
+    sg_t = None if sigma is None else torch.from_numpy(sigma.astype(np.float32)).to(dev)
+    idx, val, xn = dpb.encode(plan, x, mu_t, sg_t, workspace=ws)
+    out = dict(idx=idx, val=val, xnorm=xn, y=dpb.decode(plan, idx, val, xn, workspace=ws))
+    if gy_np is not None:
+        gy = torch.from_numpy(np.ascontiguousarray(gy_np)).to(dev).to(torch.bfloat16)
+        out["gx"], out["gv"] = dpb.backward(plan, x, idx, val, gy, sg_t, workspace=ws)
+    torch.cuda.synchronize()
+    res = {k: (v.float().cpu().numpy() if v.dtype != torch.int32 else v.cpu().numpy()) for k, v in out.items()}
+    res["status"] = dpb.workspace_status(ws)
+    return res
+
+
+def _check(plan, ref, kls, x, g, mu=None, sigma=None, gy=None):
+    xr = x.astype(np.float64)
+    idx_o, val_o, gap = oracle.encode_per_level(ref, xr, mu=mu, sigma=sigma)
+    xn_o = np.linalg.norm(xr, axis=1)
+    assert np.all(np.abs(g["xnorm"] - xn_o) <= 1e-5 * np.maximum(xn_o, 1e-30))
+    near, worst, off = 0, 0.0, 0
+    for K in kls:
+        seg = slice(off, off + K)
+        parity.check_code_order(g["idx"][:, seg], g["val"][:, seg])
+        n, w = parity.compare_codes(g["idx"][:, seg], g["val"][:, seg], idx_o[:, seg], val_o[:, seg], gap, xn_o)
+        near, worst, off = max(near, n), max(worst, w), off + K
+    y_o = oracle.decode(ref, g["idx"], g["val"].astype(np.float64), g["xnorm"].astype(np.float64))
+    e = parity.rel_rows(g["y"], y_o)
+    assert e.max() <= parity.TOL["bf16"], f"decode error {e.max():.3e}"
+    report = dict(tokens=len(x), near_ties=near, val_err=worst, dec_err=float(e.max()))
+    if gy is not None:
+        gx_o, gv_o = oracle.backward(ref, xr, g["idx"], g["val"].astype(np.float64), gy.astype(np.float64),
+                                     sigma=sigma)
+        ex, ev = parity.rel_rows(g["gx"], gx_o), parity.rel_rows(g["gv"], gv_o)
+        assert ex.max() <= parity.TOL["bf16"], f"grad_x error {ex.max():.3e}"
+        assert ev.max() <= 1e-5, f"grad_val error {ev.max():.3e}"
+        report.update(gx_err=float(ex.max()), gv_err=float(ev.max()))
+    assert g["status"] == 0, f"device status 0x{g['status']:x}"
+    assert near <= max(2, len(x) // 10), report
+    print(report)
+    return report
+
+
+def test_paper_3l_layout():
+    # PT-Small-3L (App. G): d = 1024; K = 16, 32, 64; Delta = 256; 2^10, 2^15, 2^17
+    kls = [16, 32, 64]
+    plan, ref = _plan_ref(1024, [10, 15, 17], [0, 256, 256], kls)
+    x = inputs.to_bf16(inputs.gaussian_rows(37, 1024, 0))
+    _check(plan, ref, kls, x, _gpu(plan, x))
+
+
+def test_paper_2l_layout_with_backward():
+    # the 2L variants at d = 1024: K = 16, 32; Delta = 256; 2^10, 2^15
+    kls = [16, 32]
+    plan, ref = _plan_ref(1024, [10, 15], [0, 256], kls)
+    x = inputs.to_bf16(inputs.gaussian_rows(64, 1024, 3))
+    gy = inputs.to_bf16(inputs.normal((64, 1024), 4))
+    _check(plan, ref, kls, x, _gpu(plan, x, gy_np=gy), gy=gy)
+
+
+def test_paper_2l_layout_d2048():
+    # PT-Large-2L: d = 2048 (t = 11, three 5-bit chunks of the inverse half)
+    kls = [16, 32]
+    plan, ref = _plan_ref(2048, [11, 15], [0, 256], kls)
+    x = inputs.to_bf16(inputs.gaussian_rows(9, 2048, 5))
+    _check(plan, ref, kls, x, _gpu(plan, x))
+
+
+@pytest.mark.parametrize("T", [1, 2, 5, 130])
+def test_small_layout_ragged(T):
+    kls = [4, 8, 8]
+    plan, ref = _plan_ref(64, [6, 9, 12], [0, 16, 32], kls)
+    x = inputs.to_bf16(inputs.gaussian_rows(T, 64, 7))
+    _check(plan, ref, kls, x, _gpu(plan, x))
+
+
+def test_standardisation_tables():
+    kls = [4, 8, 8]
+    plan, ref = _plan_ref(64, [6, 9, 12], [0, 16, 32], kls)
+    rng = np.random.default_rng(11)
+    mu = (0.1 * rng.standard_normal(1 << 12)).astype(np.float32)
+    sigma = (0.5 + rng.random(1 << 12)).astype(np.float32)
+    x = inputs.to_bf16(inputs.gaussian_rows(50, 64, 8))
+    _check(plan, ref, kls, x, _gpu(plan, x, mu, sigma), mu=mu.astype(np.float64), sigma=sigma.astype(np.float64))
+
+
+def test_empty_batch():
+    plan, _ = _plan_ref(64, [6, 9, 12], [0, 16, 32], [4, 8, 8])
+    x = torch.zeros((0, 64), dtype=torch.bfloat16, device="cuda")
+    idx, val, xn = dpb.encode(plan, x)
+    assert idx.shape == (0, 20)
