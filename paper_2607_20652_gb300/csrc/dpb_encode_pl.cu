@@ -42,7 +42,7 @@ constexpr int kTokens = 4;      // tokens per block, one per warp
 constexpr int kRows = 32;       // tensor-core rows per token (parent slots)
 constexpr int kChunk = 64;      // coordinates per K chunk
 constexpr int kATile = 128 * kChunk * 2;
-constexpr int kSelCap = 256;    // gathered candidates per token and level
+constexpr int kSelCap = 256;    // gathered candidates per token and level (up to 8 per lane)
 constexpr int kMaxK = 64;       // K_l per level
 constexpr uint32_t kSpin = 1u << 20;  // bound of every mbarrier wait
 // at least this much shared memory per block, so that at most two blocks (2 x
@@ -110,6 +110,17 @@ __device__ __forceinline__ uint64_t tile_desc(uint32_t saddr) {
            ((uint64_t)1 << 46);
 }
 
+// Bulk copy of one generator tile (D rows x 128 bytes) into shared memory,
+// completing on mbarrier `full`.
+__device__ __forceinline__ void copy_b(void *dst, const uint32_t *src, int D, uint32_t full) {
+    const uint32_t bytes = (uint32_t)D * 128u;
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(full), "r"(bytes) : "memory");
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     smem_u32(dst)),
+                 "l"(src), "r"(bytes), "r"(full)
+                 : "memory");
+}
+
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
     asm volatile(
         "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,"
@@ -130,11 +141,99 @@ struct WarpBufs {
     uint32_t *id;    // [kSelCap]
 };
 
+// One compare-exchange stage (size, stride) of a warp bitonic sort,
+// descending, of 32 R 64-bit words held R per lane (element lane * R + r).
+template <int R>
+__device__ __forceinline__ void sort_stage64(uint64_t (&v)[R], int size, int stride) {
+    const int lane = threadIdx.x & 31;
+    if (stride >= R) {
+        const bool lower = (lane & (stride / R)) == 0;
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+            const bool desc = (((lane * R + r) & size) == 0);
+            const uint64_t o = __shfl_xor_sync(kFull, v[r], stride / R);
+            const bool gt = v[r] > o;
+            v[r] = (lower == desc) ? (gt ? v[r] : o) : (gt ? o : v[r]);
+        }
+    } else {
+#pragma unroll
+        for (int cs = 1; cs < R; cs <<= 1) {
+            if (stride == cs) {
+#pragma unroll
+                for (int r = 0; r < R; ++r) {
+                    const int q = r ^ cs;
+                    if (q > r) {
+                        const bool desc = (((lane * R + r) & size) == 0);
+                        const uint64_t hi = v[r] > v[q] ? v[r] : v[q], lo = v[r] > v[q] ? v[q] : v[r];
+                        v[r] = desc ? hi : lo;
+                        v[q] = desc ? lo : hi;
+                    }
+                }
+            }
+        }
+    }
+}
+
+// Sorts the n (<= 32 R) gathered candidates as 64-bit words, drops repeated
+// indices (equal candidates score equally, so copies sit side by side) and
+// writes the first K to code columns [col, col + K) of row `tok` (and the
+// parents of the next level). Returns the number of distinct candidates.
+template <int R>
+__device__ __forceinline__ int sort_keep(int n, int K, const WarpBufs &w, const Args &a, int64_t tok, int col,
+                                         bool par_out, bool write) {
+    const int lane = threadIdx.x & 31;
+    uint64_t v[R];
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+        const int e = R * lane + r;
+        v[r] = e < n ? mmaenc::cword(w.z[e], w.id[e]) : 0ull;
+    }
+#pragma unroll 1
+    for (int size = 2; size <= 32 * R; size <<= 1)
+#pragma unroll 1
+        for (int stride = size / 2; stride > 0; stride >>= 1) sort_stage64<R>(v, size, stride);
+    bool keep[R];
+    uint32_t prev = __shfl_up_sync(kFull, mmaenc::cword_idx(v[R - 1]), 1);
+    int kept = 0;
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+        const uint32_t id = mmaenc::cword_idx(v[r]);
+        keep[r] = v[r] != 0ull && ((r == 0 && lane == 0) || id != prev);
+        prev = id;
+        kept += keep[r];
+    }
+    int base = kept;  // exclusive prefix of kept entries over the lanes
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int t = __shfl_up_sync(kFull, base, o);
+        if (lane >= o) base += t;
+    }
+    const int distinct = __shfl_sync(kFull, base, 31);
+    base -= kept;
+    if (write) {
+        if (par_out) w.par[lane] = 0u;
+        __syncwarp();
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+            if (keep[r] && base < K) {
+                const uint32_t id = mmaenc::cword_idx(v[r]);
+                a.idx[tok * a.code_len + col + base] = (int32_t)id;
+                a.val[tok * a.code_len + col + base] = mmaenc::cword_z(v[r]);
+                if (par_out && base < kRows) w.par[base] = id;
+            }
+            base += keep[r];
+        }
+    }
+    __syncwarp();
+    return distinct;
+}
+
 // The top K distinct candidates of one token, as explained in the header.
 // `scan(f)` calls f(z, index, live) for every candidate of this lane, in the
-// same order each time. Writes code columns [col, col + K) of row `tok` and,
-// when `par_out`, the K indices as the next level's parents. Returns the
-// number of distinct candidates written (< K only with the status bit set).
+// same order each time and in step across the warp. Writes code columns
+// [col, col + K) of row `tok` and, when `par_out`, the kept indices as the
+// next level's parents. Returns the number of distinct candidates kept
+// (< K only with the status bit set).
 template <class Scan>
 __device__ __forceinline__ int select_level(Scan scan, int nlive, int K, const WarpBufs &w, const Args &a,
                                             int64_t tok, int col, bool par_out) {
@@ -150,24 +249,54 @@ __device__ __forceinline__ int select_level(Scan scan, int nlive, int K, const W
         }
     });
     mmaenc::warp_sort_desc<4>(top);
-    const int nunion = min(4 * nlive, 128);
-    int n = 0, distinct = 0;
-    // the threshold's rank in the union: K + K/2 first; K when too many
-    // candidates reach it; the union's last when repeats leave fewer than K
-    int rank = min(K + K / 2, nunion);
-    for (int attempt = 0; attempt < 3; ++attempt) {
+    // distinct keys of the sorted union (copies of one child share a key):
+    // drank[r] = rank among them, 0 for a repeat or an empty slot
+    int drank[4];
+    {
+        uint32_t prev = __shfl_up_sync(kFull, top[3], 1);
+        int cnt = 0;
+        bool first[4];
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+            first[r] = top[r] != 0u && ((r == 0 && lane == 0) || top[r] != prev);
+            prev = top[r];
+            cnt += first[r];
+        }
+        int base = cnt;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int t = __shfl_up_sync(kFull, base, o);
+            if (lane >= o) base += t;
+        }
+        base -= cnt;
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+            drank[r] = first[r] ? base + 1 : 0;
+            base += first[r];
+        }
+    }
+    int nd = 0;  // distinct keys in the union
+#pragma unroll
+    for (int r = 0; r < 4; ++r) nd = max(nd, drank[r]);
+    nd = __reduce_max_sync(kFull, (uint32_t)nd);
+    (void)nlive;
+    int distinct = 0;
+    // tau = the union's distinct key of rank K + K/2 (so that at least that many
+    // distinct candidates reach it), rank K when too many candidates do
+    int target = min(K + K / 2, nd);
+    for (int attempt = 0; attempt < 2; ++attempt) {
         uint32_t mine = 0u;
 #pragma unroll
         for (int r = 0; r < 4; ++r)
-            if (r == (rank - 1) % 4) mine = top[r];
-        uint32_t tau = __shfl_sync(kFull, mine, (rank - 1) / 4);
+            if (drank[r] == target) mine = top[r];
+        uint32_t tau = __reduce_max_sync(kFull, mine);
         if (tau == 0u) tau = 1u;
         int cnt = 0;
         scan([&](float z, uint32_t, bool live) { cnt += live && akey(z) + 1u >= tau; });
-        n = __reduce_add_sync(kFull, cnt);
+        int n = __reduce_add_sync(kFull, cnt);
         if (n > kSelCap) {
-            if (rank > K) {  // a tighter threshold
-                rank = min(K, nunion);
+            if (attempt == 0 && target > K) {
+                target = min(K, nd);
                 continue;
             }
             set_status(a.status, DPB_DEV_SHORT_CODE);
@@ -176,51 +305,32 @@ __device__ __forceinline__ int select_level(Scan scan, int nlive, int K, const W
         int off = cnt;  // exclusive prefix over the lanes
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
-            const int v = __shfl_up_sync(kFull, off, o);
-            if (lane >= o) off += v;
+            const int t = __shfl_up_sync(kFull, off, o);
+            if (lane >= o) off += t;
         }
         off -= cnt;
         scan([&](float z, uint32_t ci, bool live) {
-            if (live && akey(z) + 1u >= tau) {
-                if (off < kSelCap) {
+            const bool take = live && akey(z) + 1u >= tau;
+            if (__any_sync(kFull, take)) {  // rare: most candidates fall short of tau
+                if (take && off < kSelCap) {
                     w.z[off] = z;
                     w.id[off] = ci;
                 }
-                ++off;
+                off += take;
             }
         });
         __syncwarp();
-        int cap = 32;
-        while (cap < n) cap <<= 1;
-        warp_sort(w.z, w.id, n, cap);
-        // repeated indices are adjacent (equal candidates score equally)
-        distinct = 0;
-        for (int e0 = 0; e0 < n; e0 += 32) {
-            const int e = e0 + lane;
-            const bool keep = e < n && (e == 0 || w.id[e] != w.id[e - 1]);
-            const unsigned mb = __ballot_sync(kFull, keep);
-            const float zv = keep ? w.z[e] : 0.f;
-            const uint32_t iv = keep ? w.id[e] : 0u;
-            __syncwarp();
-            if (keep) {
-                const int pos = distinct + __popc(mb & mmaenc::lanes_below());
-                w.z[pos] = zv;
-                w.id[pos] = iv;
-            }
-            distinct += __popc(mb);
-            __syncwarp();
+        distinct = n <= 128 ? sort_keep<4>(n, K, w, a, tok, col, par_out, true)
+                            : sort_keep<8>(n, K, w, a, tok, col, par_out, true);
+        break;
+    }
+    if (distinct < K) {
+        set_status(a.status, DPB_DEV_SHORT_CODE);
+        for (int e = distinct + lane; e < K; e += 32) {
+            a.idx[tok * a.code_len + col + e] = 0;
+            a.val[tok * a.code_len + col + e] = 0.f;
         }
-        if (distinct >= K || rank >= nunion) break;
-        rank = nunion;  // repeats took the margin: the loosest threshold
     }
-    if (distinct < K) set_status(a.status, DPB_DEV_SHORT_CODE);
-    for (int e = lane; e < K; e += 32) {
-        const bool ok = e < distinct;
-        a.idx[tok * a.code_len + col + e] = ok ? (int32_t)w.id[e] : 0;
-        a.val[tok * a.code_len + col + e] = ok ? w.z[e] : 0.f;
-    }
-    __syncwarp();
-    if (par_out) w.par[lane] = lane < min(K, distinct) ? w.id[lane] : 0u;
     __syncwarp();
     return distinct;
 }
@@ -331,26 +441,22 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
             const uint32_t *gt = a.GT + a.gt_off[l];
             for (int c = 0; c < nch; ++c) {
                 const int s = c & 1;
-                if (issued[s] > waited[s]) {  // the MMAs that last read this stage
-                    const bool ok = mbar_wait(mma_done[s], waited[s] & 1u);
+                {
+                    // the MMAs that last read this stage (thread 0 may have seen
+                    // them already, when it prefetched this chunk's B)
+                    bool ok = true;
+                    if (issued[s] > waited[s]) {
+                        ok = mbar_wait(mma_done[s], waited[s] & 1u);
+                        if (ok) ++waited[s];
+                    }
                     if (__syncthreads_or(!ok)) {  // every thread leaves together
                         failed = true;
                         break;
                     }
-                    ++waited[s];
                 }
                 uint8_t *At = sA + s * kATile;
                 uint8_t *Bt = sB + s * a.dmax * 128;
-                if (tid == 0) {
-                    const uint32_t bytes = (uint32_t)D * 128u;
-                    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(full_b[s]), "r"(bytes)
-                                 : "memory");
-                    asm volatile(
-                        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                            smem_u32(Bt)),
-                        "l"(gt + (int64_t)c * D * 32), "r"(bytes), "r"(full_b[s])
-                        : "memory");
-                }
+                if (tid == 0 && c == 0) copy_b(Bt, gt, D, full_b[s]);  // later chunks: prefetched below
 #pragma unroll
                 for (int b = 0; b < 2; ++b) {
                     const int m = 2 * c + b;
@@ -391,6 +497,20 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
                     ++bcopies[s];
                     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
                         mma_done[s]));
+                    // prefetch the next chunk's B into the other stage once the
+                    // MMAs that read it (chunk c - 1) are done
+                    if (c + 1 < nch) {
+                        const int s1 = s ^ 1;
+                        bool ok = true;
+                        if (issued[s1] > waited[s1]) {
+                            ok = mbar_wait(mma_done[s1], waited[s1] & 1u);
+                            if (ok) ++waited[s1];
+                        }
+                        if (ok)
+                            copy_b(sB + s1 * a.dmax * 128, gt + (int64_t)(c + 1) * D * 32, D, full_b[s1]);
+                        else
+                            set_status(a.status, DPB_DEV_TIMEOUT);
+                    }
                 }
                 ++issued[s];
             }

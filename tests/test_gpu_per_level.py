@@ -129,3 +129,17 @@ def test_empty_batch():
     x = torch.zeros((0, 64), dtype=torch.bfloat16, device="cuda")
     idx, val, xn = dpb.encode(plan, x)
     assert idx.shape == (0, 20)
+
+
+def test_paper_3l_layout_at_scale_sampled():
+    # T = 8192 tokens in the launch the benchmark uses; 48 sampled tokens
+    # checked against the oracle; no device status bit may be set (level 2's
+    # 32 parents share children often, which the repeat removal must absorb)
+    kls = [16, 32, 64]
+    plan, ref = _plan_ref(1024, [10, 15, 17], [0, 256, 256], kls)
+    T = 8192
+    x = inputs.to_bf16(inputs.gaussian_rows(T, 1024, 21))
+    g = _gpu(plan, x)
+    rows = np.random.default_rng(5).choice(T, 48, replace=False)
+    sub = {k: (v[rows] if isinstance(v, np.ndarray) and v.shape[:1] == (T,) else v) for k, v in g.items()}
+    _check(plan, ref, kls, x[rows], sub)
