@@ -490,6 +490,105 @@ def run_e2e(plan, x, gy, args, device, stream, world):
             "h2d_bytes_per_step": bi, "d2h_bytes_per_step": bo, "steps": steps}
 
 
+# ---------------------------------------------------------------------------
+# the paper's per-level layouts (supplementary lines; the headline is "wide")
+# ---------------------------------------------------------------------------
+
+def per_level_work(w, T: int, k_hash: float, s: int):
+    """Algorithmic work of the per-level layouts: level l scores K_{l-1} x
+    Delta_l children (Eq. 6: 2 d flops and d sign applications each)."""
+    d, kl, ch = w["d"], w["k_per_level"], w["children"]
+    code = sum(kl)
+    mma = sum(2 * kl[l - 1] * ch[l] * d for l in range(1, w["levels"]))
+    signs = sum(kl[l - 1] * d for l in range(1, w["levels"]))
+    return {
+        "encode": {"bytes": T * (d * s + 8 * code + 4), "tensor_flops": T * mma, "int_ops": T * signs},
+        "decode": {"bytes": T * (8 * code + 4 + d * s), "fp_ops": T * (k_hash * d + 3 * d)},
+        "backward": {"bytes": T * (3 * d * s + 12 * code), "fp_ops": T * (2 * k_hash * d + 6 * d)},
+    }
+
+
+def run_per_level(args, world, rank, local):
+    import torch
+    from paper_2607_20652_gb300 import configs, dpb, inputs
+
+    device = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(device)
+    w = dict(configs.PER_LEVEL[args.workload])
+    T, d = w["T"], w["d"]
+    plan = dpb.Plan(d=d, levels=w["levels"], bits=w["bits"], children=w["children"], dtype="bf16",
+                    select_mode=dpb.SELECT_PER_LEVEL, k_per_level=w["k_per_level"])
+    seed = shard_seed(w["seed"], rank)
+    x = torch.from_numpy(inputs.to_bf16(inputs.gaussian_rows(T, d, seed))).to(device).to(torch.bfloat16)
+    gy = torch.from_numpy(inputs.to_bf16(inputs.normal((T, d), seed + w["grad_seed"]))).to(device).to(torch.bfloat16)
+    k = plan.code_len
+    idx = torch.empty((T, k), dtype=torch.int32, device=device)
+    val = torch.empty((T, k), dtype=torch.float32, device=device)
+    xn = torch.empty((T,), dtype=torch.float32, device=device)
+    y, gx = torch.empty_like(x), torch.empty_like(x)
+    gv = torch.empty((T, k), dtype=torch.float32, device=device)
+    ws = plan.workspace(T, device)
+    stream = torch.cuda.current_stream(device)
+
+    def step(ev=None):
+        if ev:
+            ev[0].record(stream)
+        dpb.encode(plan, x, idx=idx, val=val, xnorm=xn, workspace=ws, stream=stream)
+        if ev:
+            ev[1].record(stream)
+        dpb.decode(plan, idx, val, xn, y=y, workspace=ws, stream=stream)
+        if ev:
+            ev[2].record(stream)
+        dpb.backward(plan, x, idx, val, gy, grad_x=gx, grad_val=gv, workspace=ws, stream=stream)
+        if ev:
+            ev[3].record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize(device)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    clocks = ClockSampler(None)
+    clocks.start()
+    time.sleep(0.3)
+    barrier(world)
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for i in range(args.steps):
+        step(evs[i])
+    end.record(stream)
+    torch.cuda.synchronize(device)
+    barrier(world)
+    clk = clocks.stop()
+    ms_max = max_over_ranks(start.elapsed_time(end), world, device)
+    kern_ms = {n: statistics.mean(e[j].elapsed_time(e[j + 1]) for e in evs)
+               for j, n in enumerate(("encode", "decode", "backward"))}
+    k_hash = float(np.mean(np.sum(idx.cpu().numpy() >= d, axis=1)))
+    peaks, src = load_peaks()
+    work = per_level_work(w, T, k_hash, 2)
+    kernels = {n: {"ms": round(v, 4), **{kk: vv for kk, vv in roofline_for(n, work[n], v / 1e3, peaks, src).items()
+                                          if kk in ("bound", "frac", "t_roofline_us", "achieved", "unit")}}
+               for n, v in kern_ms.items()}
+    dom = max(kern_ms, key=kern_ms.get)
+    line = {
+        "metric": f"DPB tokens/sec (encode+decode+bwd), per-level selection, paper {args.workload[5:].upper()} layout "
+                  f"(d={d}, K={w['k_per_level']}, Delta=256), 1 GB300",
+        "value": round(whole_job_rate(T, world, args.steps, ms_max / 1e3), 1), "unit": "tokens/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(ms_max / args.steps, 4), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": args.workload, "T_per_gpu": T, "d": d, "levels": w["levels"], "bits": w["bits"],
+                   "children": w["children"], "k_per_level": w["k_per_level"], "select": "per_level",
+                   "inputs": "bf16 x ~ N(0,1), grad_y ~ N(0,1)",
+                   "l2": "inputs (2 x 128 MiB) larger than the 129 MB L2 (no flush needed)"},
+        "roofline": roofline_for(dom, work[dom], kern_ms[dom] / 1e3, peaks, src),
+        "kernels": kernels, "k_hash": round(k_hash, 2), "gpu_launches": 3 * args.steps, "clocks": clk,
+        "device_status": dpb.workspace_status(ws),
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    return 0
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -500,6 +599,8 @@ def main(argv=None):
     ap.add_argument("--ref-tokens", type=int, default=512)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--workload", default=WORKLOAD, choices=[WORKLOAD, "paper3l", "paper2l"],
+                    help="wide (the headline, global selection) or one of the paper's per-level layouts")
     args = ap.parse_args(argv)
     world, rank, local = dist_env()
     if args.warmup < 3 and args.impl == "ours":
@@ -507,6 +608,8 @@ def main(argv=None):
         args.warmup = 3
     if args.impl == "reference":
         return run_reference(args, world, rank)
+    if args.workload != WORKLOAD:
+        return run_per_level(args, world, rank, local)
     return run_ours(args, world, rank, local)
 
 

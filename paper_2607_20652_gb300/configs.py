@@ -23,6 +23,19 @@ WORKLOADS = {
                  passes="fwd+bwd"),
 }
 
+# The paper's own per-level layouts (App. G), per-level selection: PT-Small-3L
+# (d = 1024; K = 16, 32, 64 over 2^10, 2^15, 2^17 indices; 256 children per
+# parent) and the 2L variants at d = 1024 (K = 16, 32 over 2^10, 2^15); bf16
+# x ~ N(0, 1); encode + decode + backward with grad_y ~ N(0, 1)
+PER_LEVEL = {
+    "paper3l": dict(T=65536, d=1024, levels=3, bits=[10, 15, 17], children=[0, 256, 256],
+                    k_per_level=[16, 32, 64], dtype="bf16", inputs="gaussian", seed=0, grad_seed=1,
+                    passes="fwd+bwd"),
+    "paper2l": dict(T=65536, d=1024, levels=2, bits=[10, 15], children=[0, 256],
+                    k_per_level=[16, 32], dtype="bf16", inputs="gaussian", seed=0, grad_seed=1,
+                    passes="fwd+bwd"),
+}
+
 # d=768, T=32768: features 2^16/2^18/2^20/2^22, k in {16,32,64,128}, beam in {4,8,16}
 SWEEP = [dict(T=32768, d=768, m_bits=mb, levels=5, children=16, beam=b, k=k, dtype="bf16",
               inputs="gaussian", seed=0, grad_seed=1, passes="fwd+bwd")
