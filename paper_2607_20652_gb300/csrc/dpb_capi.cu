@@ -78,7 +78,7 @@ dpb_status dpb_plan_create(const dpb_config *cfg, const uint32_t *generators, dp
     const size_t smem = p->cfg.select_mode == DPB_SELECT_GLOBAL
                             ? dpb::encode_smem_header(p) + dpb::encode_smem_per_warp(p)
                             : dpb::encode_pl_smem(p);
-    if (smem > 200 * 1024) {
+    if (smem > (p->cfg.select_mode == DPB_SELECT_GLOBAL ? (size_t)200 * 1024 : dpb::kMaxSmemPerBlock)) {
         delete p;
         return dpb::fail(DPB_ERR_UNSUPPORTED, "encoder needs %zu bytes of shared memory per warp", smem);
     }

@@ -4,11 +4,14 @@
 // l-1 and keeps its top K_l distinct children; the code is every level's kept
 // set, level by level, each in (|z| descending, index ascending) order.
 //
-// Child scoring (Eq. 6) runs on the tcgen05 tensor cores. A block of 4 warps
-// owns 4 tokens. At level l its 128 tensor-core rows are (token, parent
-// slot), 32 slots per token, and its Delta_l columns the level's generators,
-// so one tcgen05.mma of M = 128, N = Delta_l, K = 16 scores 128 x Delta_l
-// children at once; K runs over d in chunks of 64 coordinates, double
+// Child scoring (Eq. 6) runs on the tcgen05 tensor cores. A block of 8 warps
+// owns 8 tokens. At level l its tensor-core rows are (token, parent slot):
+// 16 slots per token (one M = 128 tile) when K_{l-1} <= 16, else 32 (two
+// tiles); its Delta_l columns are the level's generators, so one tcgen05.mma
+// of M = 128, N = Delta_l, K = 16 scores 128 x Delta_l children at once. Tile
+// t's TMEM lane quarter q holds the rows of token q + 4 t (32 slots), or of
+// tokens q and q + 4 (16 slots each), so that warp w reads its token's rows
+// from its own quarter. K runs over d in chunks of 64 coordinates, double
 // buffered:
 //  - A (128 x 64 bf16) is built in shared memory by the block's threads,
 //    each writing its row x (.) phi~_parent: the token's x pairs XOR the
@@ -38,16 +41,16 @@ namespace dpb {
 
 namespace {
 
-constexpr int kTokens = 4;      // tokens per block, one per warp
+constexpr int kTokens = 8;      // tokens per block, one per warp
 constexpr int kRows = 32;       // tensor-core rows per token (parent slots)
 constexpr int kChunk = 64;      // coordinates per K chunk
-constexpr int kATile = 128 * kChunk * 2;
+constexpr int kATile = 128 * kChunk * 2;  // one M = 128 tile of a chunk
 constexpr int kSelCap = 256;    // gathered candidates per token and level (up to 8 per lane)
 constexpr int kMaxK = 64;       // K_l per level
 constexpr uint32_t kSpin = 1u << 20;  // bound of every mbarrier wait
-// at least this much shared memory per block, so that at most two blocks (2 x
-// 256 TMEM columns) share an SM
-constexpr int kMinSmem = 80 * 1024;
+// at least this much shared memory per block, so that one block (holding all
+// 512 TMEM columns) runs per SM
+constexpr int kMinSmem = 120 * 1024;
 
 struct Args {
     const __nv_bfloat16 *x;
@@ -75,7 +78,7 @@ __host__ __device__ inline Layout layout(int d, int levels, int kvh, int dmax) {
     const int nblk = d / 32;
     Layout l;
     l.a = 0;
-    l.b = l.a + 2 * kATile;
+    l.b = l.a + 2 * 2 * kATile;  // 2 stages x 2 tiles
     l.xw = l.b + 2 * dmax * 128;
     l.vh = l.xw + kTokens * nblk * 16 * 4;
     l.g = l.vh + kvh * nblk * 32 * 4;
@@ -377,7 +380,7 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
         asm volatile("fence.mbarrier_init.release.cluster;");
     }
     if (warp == 0) {
-        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 256;" ::"r"(smem_u32(tmem_slot)));
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 512;" ::"r"(smem_u32(tmem_slot)));
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
     }
     __syncthreads();
@@ -430,14 +433,29 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
 
         for (int l = 1; l < L && !failed; ++l) {
             const int P = a.kl[l - 1], D = a.delta[l], nch = d / kChunk;
-            const bool rv = live && lane < P;
-            const uint32_t p = rv ? wb.par[lane] : 0u;
-            const uint32_t w5p = w5[p & 31u], u = (p & lo_mask) >> 5;
-            uint32_t hv[4];  // the 5-bit chunks of p's high half
+            const int pp = P <= 16 ? 16 : 32, ntiles = pp / 16;  // slots per token, M = 128 tiles
+            // this thread builds block half hb of row rr of each tile
+            const int rr = tid & 127, hb = tid >> 7;
+            uint32_t ip[2], iw5[2], iu[2], ihv[2][4];
+            bool irv[2];
+            const uint32_t *ixt[2];
 #pragma unroll
-            for (int k = 0; k < 4; ++k) hv[k] = (p >> min(a.t + 5 * k, 31)) & 31u;
+            for (int tt = 0; tt < 2; ++tt) {
+                const int q = rr >> 5, jj = rr & 31;
+                const int tokw = pp == 32 ? q + 4 * tt : q + 4 * (jj >> 4);
+                const int slot = pp == 32 ? jj : jj & 15;
+                const bool ok = tt < ntiles && grp * kTokens + tokw < a.T && slot < P;
+                const uint32_t *par = reinterpret_cast<const uint32_t *>(smem + lay.warps + tokw * kWarpBytes);
+                const uint32_t pv = ok ? par[slot] : 0u;
+                irv[tt] = ok;
+                ip[tt] = pv;
+                iw5[tt] = w5[pv & 31u];
+                iu[tt] = (pv & lo_mask) >> 5;
+#pragma unroll
+                for (int k = 0; k < 4; ++k) ihv[tt][k] = (pv >> min(a.t + 5 * k, 31)) & 31u;
+                ixt[tt] = xw + tokw * nblk * 16;
+            }
             const uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(D >> 3) << 17) | (8u << 24);
-            const uint32_t *xt = xw + warp * nblk * 16;
             const uint32_t *gt = a.GT + a.gt_off[l];
             for (int c = 0; c < nch; ++c) {
                 const int s = c & 1;
@@ -454,27 +472,32 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
                         break;
                     }
                 }
-                uint8_t *At = sA + s * kATile;
+                uint8_t *As = sA + s * 2 * kATile;
                 uint8_t *Bt = sB + s * a.dmax * 128;
                 if (tid == 0 && c == 0) copy_b(Bt, gt, D, full_b[s]);  // later chunks: prefetched below
 #pragma unroll
-                for (int b = 0; b < 2; ++b) {
-                    const int m = 2 * c + b;
-                    uint32_t sw = w5p ^ (0u - (uint32_t)(__popc((uint32_t)m & u) & 1));
+                for (int tt = 0; tt < 2; ++tt) {
+                    if (tt < ntiles) {
+                        const int m = 2 * c + hb;
+                        const bool rv = irv[tt];
+                        uint32_t sw = iw5[tt] ^ (0u - (uint32_t)(__popc((uint32_t)m & iu[tt]) & 1));
 #pragma unroll
-                    for (int k = 0; k < 4; ++k)
-                        if (k < a.kvh) sw ^= vh[(k * nblk + m) * 32 + hv[k]];
-                    const uint4 *xs = reinterpret_cast<const uint4 *>(xt + m * 16);
+                        for (int k = 0; k < 4; ++k)
+                            if (k < a.kvh) sw ^= vh[(k * nblk + m) * 32 + ihv[tt][k]];
+                        const uint4 *xs = reinterpret_cast<const uint4 *>(ixt[tt] + m * 16);
+                        uint8_t *At = As + tt * kATile;
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        const uint4 xv = xs[q];
-                        const int sh = 15 - 4 * q;
-                        uint4 av;
-                        av.x = rv ? xv.x ^ ((sw << sh) & 0x80008000u) : 0u;
-                        av.y = rv ? xv.y ^ ((sw << (sh - 1)) & 0x80008000u) : 0u;
-                        av.z = rv ? xv.z ^ ((sw << (sh - 2)) & 0x80008000u) : 0u;
-                        av.w = rv ? xv.w ^ ((sw << (sh - 3)) & 0x80008000u) : 0u;
-                        *reinterpret_cast<uint4 *>(At + (tid >> 3) * 1024 + (4 * b + q) * 128 + (tid & 7) * 16) = av;
+                        for (int q = 0; q < 4; ++q) {
+                            const uint4 xv = xs[q];
+                            const int sh = 15 - 4 * q;
+                            uint4 av;
+                            av.x = rv ? xv.x ^ ((sw << sh) & 0x80008000u) : 0u;
+                            av.y = rv ? xv.y ^ ((sw << (sh - 1)) & 0x80008000u) : 0u;
+                            av.z = rv ? xv.z ^ ((sw << (sh - 2)) & 0x80008000u) : 0u;
+                            av.w = rv ? xv.w ^ ((sw << (sh - 3)) & 0x80008000u) : 0u;
+                            *reinterpret_cast<uint4 *>(At + (rr >> 3) * 1024 + (4 * hb + q) * 128 + (rr & 7) * 16) =
+                                av;
+                        }
                     }
                 }
                 asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -484,14 +507,17 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
                         set_status(a.status, DPB_DEV_TIMEOUT);  // the commit below still arrives
                     } else {
                         asm volatile("tcgen05.fence::after_thread_sync;");
-                        const uint32_t ab = smem_u32(At), bb = smem_u32(Bt);
+                        const uint32_t bb = smem_u32(Bt);
+                        for (int tt = 0; tt < ntiles; ++tt) {
+                            const uint32_t ab = smem_u32(As + tt * kATile);
 #pragma unroll
-                        for (int k = 0; k < kChunk / 16; ++k) {
-                            const uint32_t acc = (c > 0 || k > 0) ? 1u : 0u;
-                            asm volatile(
-                                "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-                                "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem),
-                                "l"(tile_desc(ab + 256 * k)), "l"(tile_desc(bb + 256 * k)), "r"(idesc), "r"(acc));
+                            for (int k = 0; k < kChunk / 16; ++k) {
+                                const uint32_t acc = (c > 0 || k > 0) ? 1u : 0u;
+                                asm volatile(
+                                    "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+                                    "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem + 256 * tt),
+                                    "l"(tile_desc(ab + 256 * k)), "l"(tile_desc(bb + 256 * k)), "r"(idesc), "r"(acc));
+                            }
                         }
                     }
                     ++bcopies[s];
@@ -527,7 +553,13 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
             asm volatile("tcgen05.fence::after_thread_sync;");
             // ---- the level's selection, one warp per token ----
             if (live) {
-                const uint32_t taddr = tmem + ((uint32_t)(32 * warp) << 16);
+                // this warp's rows: tile (warp / 4 when 32 slots), quarter warp % 4,
+                // lanes [base, base + pp) of it
+                const int tile = pp == 32 ? warp >> 2 : 0, base = pp == 16 ? 16 * (warp >> 2) : 0;
+                const uint32_t taddr = tmem + ((uint32_t)(32 * (warp & 3)) << 16) + 256u * tile;
+                const int slot = lane - base;
+                const bool rv = slot >= 0 && slot < pp && slot < P;
+                const uint32_t p = rv ? wb.par[slot] : 0u;
                 const uint32_t *gl = gs + l * 256;
                 auto scanl = [&](auto f) {
                     for (int c0 = 0; c0 < D; c0 += 32) {
@@ -556,7 +588,7 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
         }
     asm volatile("tcgen05.fence::before_thread_sync;");
     __syncthreads();
-    if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 256;" ::"r"(tmem));
+    if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" ::"r"(tmem));
 }
 
 }  // namespace
