@@ -6,7 +6,7 @@
 //   dL/dr      = c (g - (<g,r> / |r|^2) r)          (g without norm matching)
 //   grad_val_e = <phi_e, dL/dr>
 //   grad_x     = sum_e (grad_val_e / sigma_e) phi_e + (<g,r>/|r|) x / |x|.
-// The table-driven kernel (d <= 1024) evaluates the two sums over phi with the
+// The table-driven kernel (d <= 2048) evaluates the two sums over phi with the
 // sweeps of dpb_lut.cuh and the inner products <phi_e, dL/dr> with per-token
 // tables of signed sums of dL/dr over 4 coordinates (see analyse()).
 #include <algorithm>
@@ -149,7 +149,7 @@ __global__ void __launch_bounds__(128) backward_warp_kernel(BackwardArgs a) {
 }
 
 
-// ---- table-driven backward (d <= 1024) ---------------------------------------
+// ---- table-driven backward (d <= 2048) ---------------------------------------
 
 constexpr int kChunkBlocks = 4;                       // 32-coordinate blocks per analysis chunk
 constexpr int kTabStride = 17;                        // 16 entries + 1 pad (bank spread)
@@ -163,7 +163,7 @@ __host__ __device__ constexpr int bwd_warp_words(int d, int k) {
 }
 
 __host__ __device__ constexpr int bwd_block_words(int d, int nkc) {
-    return pad4(d) /* koff */ + 32 /* W5 */ + 1024 /* PQ */ + nkc * 1024 /* VH */;
+    return pad4(d) /* koff */ + 32 /* W5 */ + nkc * ((d + 31) / 32) * 32 /* VH2 */;
 }
 
 struct BwdWarp {
@@ -172,36 +172,34 @@ struct BwdWarp {
     float *ha;      // [k] hashed coefficients, later grad_val / sigma
     int *cmap;      // [k] code entry -> hashed position (>= 0) or -(c+1) (basis) or INT_MIN
     float *gv;      // [k] analysis sums per hashed position
-    uint32_t *o1;   // [k] packed table offsets (W5, PQ, VH_0, VH_1)
-    uint32_t *o2;   // [k] packed table offsets (VH_2, VH_3); later basis grad_x terms
+    uint32_t *o1;   // [k] the Walsh word W5[c & 31] of each hashed code
+    uint32_t *o2;   // [k] its block-parity index and high-half chunks; later basis grad_x terms
     uint32_t *scratch;
 };
 
-// Table offsets (bytes) of code c in the sign-word tables of a block:
-// W5[c & 31], PQ[q][(c_lo >> 5) & 31], VH_k[q][(c >> (t + 5k)) & 31].
-__device__ __forceinline__ void code_offsets(uint32_t c, int t, uint32_t &o1, uint32_t &o2) {
-    const uint32_t lo = c & ((1u << t) - 1u);
-    const uint32_t b0 = (c & 31u) * 4u, b1 = ((lo >> 5) & 31u) * 4u;
-    const uint32_t h0 = ((c >> t) & 31u) * 4u, h1 = ((c >> (t + 5)) & 31u) * 4u;
-    const uint32_t h2 = (t + 10 < 32) ? ((c >> (t + 10)) & 31u) * 4u : 0u;
-    const uint32_t h3 = (t + 15 < 32) ? ((c >> (t + 15)) & 31u) * 4u : 0u;
-    o1 = b0 | (b1 << 8) | (h0 << 16) | (h1 << 24);
-    o2 = h2 | (h3 << 8);
+// Per-code parts of the sign words (bit l of block q = parity(M[32q + l] AND
+// c), App. A.4 Eq. 26): o1 = W5[c & 31], the Walsh part; o2 = u | h0 << 11 |
+// h1 << 16 | h2 << 21 | h3 << 26 with u = c_lo >> 5 (the block-parity mask)
+// and h_k the 5-bit chunks of the high half.
+__device__ __forceinline__ void code_offsets(uint32_t c, int t, const uint32_t *w5, uint32_t &o1, uint32_t &o2) {
+    const uint32_t u = (c & ((1u << t) - 1u)) >> 5;
+    uint32_t h = 0;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) h |= ((c >> min(t + 5 * k, 31)) & 31u) << (5 * k);
+    o1 = w5[c & 31u];
+    o2 = u | (h << 11);
 }
 
-// Sign word of code (o1, o2) over block q: bit l = parity(M[32q + l] AND c).
+// Sign word of code (o1, o2) over block q (VH2 holds NKC chunk tables of
+// nblk blocks x 32 words).
 template <int NKC>
-__device__ __forceinline__ uint32_t block_signs(const uint32_t *w5, const uint32_t *pq, const uint32_t *vh,
-                                                int q, uint32_t o1, uint32_t o2) {
-    const char *W = reinterpret_cast<const char *>(w5);
-    const char *P = reinterpret_cast<const char *>(pq + q * 32);
-    const char *V = reinterpret_cast<const char *>(vh + q * 32);
-    uint32_t s = *reinterpret_cast<const uint32_t *>(W + __byte_perm(o1, 0, 0x4440)) ^
-                 *reinterpret_cast<const uint32_t *>(P + __byte_perm(o1, 0, 0x4441)) ^
-                 *reinterpret_cast<const uint32_t *>(V + __byte_perm(o1, 0, 0x4442));
-    s ^= *reinterpret_cast<const uint32_t *>(V + 4096 + __byte_perm(o1, 0, 0x4443));
-    if (NKC > 2) s ^= *reinterpret_cast<const uint32_t *>(V + 8192 + __byte_perm(o2, 0, 0x4440));
-    if (NKC > 3) s ^= *reinterpret_cast<const uint32_t *>(V + 12288 + __byte_perm(o2, 0, 0x4441));
+__device__ __forceinline__ uint32_t block_signs(const uint32_t *vh2, int nblk, int q, uint32_t o1, uint32_t o2) {
+    const uint32_t *V = vh2 + q * 32;
+    uint32_t s = o1 ^ (0u - (uint32_t)(__popc((uint32_t)q & (o2 & 0x7FFu)) & 1));
+    s ^= V[(o2 >> 11) & 31u];
+    s ^= V[nblk * 32 + ((o2 >> 16) & 31u)];
+    if (NKC > 2) s ^= V[2 * nblk * 32 + ((o2 >> 21) & 31u)];
+    if (NKC > 3) s ^= V[3 * nblk * 32 + ((o2 >> 26) & 31u)];
     return s;
 }
 
@@ -212,8 +210,7 @@ __device__ __forceinline__ uint32_t block_signs(const uint32_t *w5, const uint32
 // Items of one warp step have distinct codes, so the shared-memory
 // accumulation order is fixed.
 template <int NKC>
-__device__ __forceinline__ void analyse(const BwdWarp &w, int nh, int d, const uint32_t *w5,
-                                        const uint32_t *pq, const uint32_t *vh) {
+__device__ __forceinline__ void analyse(const BwdWarp &w, int nh, int d, const uint32_t *vh2) {
     const int lane = threadIdx.x & 31;
     const int qn = (d + 31) / 32;
     const int nhp = nh > 32 ? nh : 32;
@@ -248,7 +245,7 @@ __device__ __forceinline__ void analyse(const BwdWarp &w, int nh, int d, const u
             // block of the chunk and code of this item (cq <= 4 blocks)
             const int qq = (it >= nhp) + (it >= 2 * nhp) + (it >= 3 * nhp), e = it - qq * nhp;
             if (e < nh) {
-                const uint32_t s = block_signs<NKC>(w5, pq, vh, q0 + qq, w.o1[e], w.o2[e]);
+                const uint32_t s = block_signs<NKC>(vh2, qn, q0 + qq, w.o1[e], w.o2[e]);
                 const char *T = reinterpret_cast<const char *>(TH + qq * 8 * kTabStride);
                 constexpr int S4 = 4 * kTabStride;  // bytes per table
                 float p0 = *reinterpret_cast<const float *>(T + ((s << 2) & 0x3Cu));
@@ -274,15 +271,13 @@ __global__ void __launch_bounds__(kBwdWarps * 32, 3) backward_lut_kernel(Backwar
     const int dp = pad4(d), kp = pad4(k);
     uint32_t *koff = smem;
     uint32_t *w5 = koff + dp;
-    uint32_t *pq = w5 + 32;
-    uint32_t *vh = pq + 1024;
+    uint32_t *vh2 = w5 + 32;
     for (int v = threadIdx.x; v < 32; v += blockDim.x) {
         uint32_t word = 0;
         for (int l = 0; l < 32; ++l) word |= (uint32_t)(__popc(l & v) & 1) << l;
         w5[v] = word;
     }
-    for (int i = threadIdx.x; i < 1024; i += blockDim.x) pq[i] = (__popc((i >> 5) & (i & 31)) & 1) ? ~0u : 0u;
-    for (int i = threadIdx.x; i < NKC * 1024; i += blockDim.x) vh[i] = a.VH[i];
+    for (int i = threadIdx.x; i < NKC * ((d + 31) / 32) * 32; i += blockDim.x) vh2[i] = a.VH[i];
     load_koff(a.M, d, t, koff);  // ends with __syncthreads()
 
     uint32_t *base = smem + bwd_block_words(d, NKC) + (size_t)warp * bwd_warp_words(d, k);
@@ -334,7 +329,7 @@ __global__ void __launch_bounds__(kBwdWarps * 32, 3) backward_lut_kernel(Backwar
                 w.ha[pos] = v;
                 w.cmap[e] = pos;
                 w.gv[pos] = 0.f;
-                code_offsets((uint32_t)ci, t, w.o1[pos], w.o2[pos]);
+                code_offsets((uint32_t)ci, t, w5, w.o1[pos], w.o2[pos]);
             }
             nh += __popc(m);
         }
@@ -352,7 +347,7 @@ __global__ void __launch_bounds__(kBwdWarps * 32, 3) backward_lut_kernel(Backwar
         for (int pass = a.norm_match ? 0 : 1;; ++pass) {
             if (pass == 1) {
                 // ---- grad_val = <phi_e, dL/dr> ----
-                analyse<NKC>(w, nh, d, w5, pq, vh);
+                analyse<NKC>(w, nh, d, vh2);
                 // ---- grad_val of every entry; the grad_x coefficients ----
                 for (int e = lane; e < k; e += 32) {
                     const int cm = w.cmap[e];
@@ -458,9 +453,9 @@ cudaError_t launch_backward(const dpb_plan *p, const void *x, const int32_t *idx
                             void *grad_x, float *grad_val, int32_t *status,
                             cudaStream_t stream) {
     const dpb_config &c = p->cfg;
-    BackwardArgs a{x, grad_y, idx, val, sigma, grad_x, grad_val, T, status, p->dM, p->dVH,
+    BackwardArgs a{x, grad_y, idx, val, sigma, grad_x, grad_val, T, status, p->dM, p->dVH2,
                    c.d, p->code_len, c.norm_match, p->m_mask, p->inv_sqrt_d};
-    if (c.d <= 1024) {
+    if (c.d <= 2048) {
         return c.dtype == DPB_BF16 ? dispatch_backward_lut<__nv_bfloat16>(p, a, T, stream)
                                    : dispatch_backward_lut<float>(p, a, T, stream);
     }

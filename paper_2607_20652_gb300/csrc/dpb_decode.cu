@@ -84,7 +84,7 @@ __global__ void __launch_bounds__(128) decode_warp_kernel(DecodeArgs a) {
     }
 }
 
-// ---- table-driven decoder (d <= 1024) -----------------------------------------
+// ---- table-driven decoder (d <= 2048) -----------------------------------------
 
 // Per-warp shared memory of the decoder, in 4-byte words: r (d), the hashed
 // list (indices, coefficients) and one sweep's tables.
@@ -164,7 +164,7 @@ cudaError_t launch_decode(const dpb_plan *p, const int32_t *idx, const float *va
     const dpb_config &c = p->cfg;
     DecodeArgs a{idx, val, xnorm, y, T, status, p->dM, c.d, p->code_len, c.norm_match, p->m_mask,
                  p->inv_sqrt_d};
-    if (c.d <= 1024) {
+    if (c.d <= 2048) {
         return c.dtype == DPB_BF16 ? dispatch_decode_lut<__nv_bfloat16>(p, a, T, stream)
                                    : dispatch_decode_lut<float>(p, a, T, stream);
     }

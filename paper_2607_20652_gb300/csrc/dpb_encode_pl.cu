@@ -644,20 +644,7 @@ void build_per_level_tables(dpb_plan *p) {
     }
     p->GT.assign(gt.size() / 2, 0u);
     for (size_t w = 0; w < p->GT.size(); ++w) p->GT[w] = (uint32_t)gt[2 * w] | ((uint32_t)gt[2 * w + 1] << 16);
-    // inverse-coordinate sign words per 32-coordinate block (any d <= 2048)
-    const int kvh = std::max(1, (c.field_t + 4) / 5);
-    p->VH2.assign((size_t)kvh * nblk * 32, 0u);
-    for (int k = 0; k < kvh; ++k)
-        for (int q = 0; q < nblk; ++q)
-            for (int v = 0; v < 32; ++v) {
-                uint32_t w = 0;
-                const uint32_t mask = (uint32_t)v << (5 * k);
-                for (int l = 0; l < 32; ++l) {
-                    const uint32_t kappa = p->M[32 * q + l] >> c.field_t;
-                    w |= (uint32_t)(__builtin_popcount(kappa & mask) & 1) << l;
-                }
-                p->VH2[((size_t)k * nblk + q) * 32 + v] = w;
-            }
+    // (VH2, the inverse-coordinate sign words per block, is built with the plan)
 }
 
 size_t encode_pl_smem(const dpb_plan *p) {

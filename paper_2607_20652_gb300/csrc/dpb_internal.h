@@ -39,7 +39,8 @@ struct dpb_plan {
     //    (n / 8) 1024 + (kk / 8) 128 + (n % 8) 16 + (kk % 8) 2), where K
     //    position kk = 32 b + 2 i + h of the chunk holds coordinate
     //    32 (2 c + b) + i + 16 h; level l starts at word gt_off[l];
-    //  VH2[k][q][v]: as VH, for every 32-coordinate block of d <= 2048.
+    //  VH2[k][q][v]: as VH, for every 32-coordinate block of d <= 2048 (built
+    //    for every plan; max(2, kvh) chunks).
     std::vector<uint32_t> GT;
     std::vector<uint32_t> VH2;
     int64_t gt_off[DPB_MAX_LEVELS] = {};

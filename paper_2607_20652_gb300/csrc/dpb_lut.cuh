@@ -31,14 +31,15 @@ constexpr int kMaxRuns = 13;     // ceil(64 / 5) runs of 5 codes per sweep
 constexpr int kShflRuns = 7;     // even runs 0, 2, ..., 12
 
 // Shared-memory words of one sweep's tables.
-constexpr int kSweepWords = 2 * 32 /* ZQ (uint2 per block, up to 32 blocks) */ +
+constexpr int kMaxBlocks = 64;   // 32-coordinate blocks of d <= 2048
+constexpr int kSweepWords = 2 * kMaxBlocks /* ZQ (uint2 per block) */ +
                             2 * 32 * kMaxKChunks /* ZH (uint2 entries) */ +
                             32 * kShflRuns /* odd runs' value tables */ + 64 /* coefficients */;
 
 struct Sweep {
     uint2 zl;                 // ZL(lane) for codes 0..31 (x) and 32..63 (y)
     float vt[kShflRuns];      // lane v holds the table of run 2i at v
-    uint2 *zq;                // [32] (shared)
+    uint2 *zq;                // [kMaxBlocks] (shared)
     uint2 *zh;                // [kMaxKChunks][32] (shared)
     float *vto;               // [6][32] odd runs (shared)
     float *coef;              // [64] (shared)
@@ -48,7 +49,7 @@ struct Sweep {
 __device__ __forceinline__ Sweep sweep_at(uint32_t *base) {
     Sweep s;
     s.zq = reinterpret_cast<uint2 *>(base);
-    s.zh = s.zq + 32;
+    s.zh = s.zq + kMaxBlocks;
     s.vto = reinterpret_cast<float *>(s.zh + 32 * kMaxKChunks);
     s.coef = s.vto + 32 * (kMaxRuns - kShflRuns);
     return s;
@@ -63,7 +64,7 @@ __device__ __forceinline__ uint32_t kappa_offsets8(uint32_t kappa) {
 }
 
 // Sign tables of a sweep from its codes (lane holds codes lane and 32 + lane;
-// 0 for empty slots). qn = number of 32-coordinate blocks (<= 32).
+// 0 for empty slots). qn = number of 32-coordinate blocks (<= kMaxBlocks).
 __device__ __forceinline__ void sweep_build_signs(uint32_t ca, uint32_t cb, int t, int qn, Sweep &s) {
     const int lane = threadIdx.x & 31;
     uint2 zl = make_uint2(0u, 0u);
@@ -76,22 +77,22 @@ __device__ __forceinline__ void sweep_build_signs(uint32_t ca, uint32_t cb, int 
         }
     }
     s.zl = zl;
-    uint32_t qa[5], qb[5];  // iota bits 5..9 are the bits of the block index q
+    uint32_t qa[6], qb[6];  // iota bits 5..10 are the bits of the block index q
 #pragma unroll
-    for (int b = 0; b < 5; ++b) {
+    for (int b = 0; b < 6; ++b) {
         const bool live = 5 + b < t;
         qa[b] = live ? __ballot_sync(kFull, (ca >> (5 + b)) & 1u) : 0u;
         qb[b] = live ? __ballot_sync(kFull, (cb >> (5 + b)) & 1u) : 0u;
     }
-    if (lane < qn) {
+    for (int q = lane; q < qn; q += 32) {
         uint2 z = make_uint2(0u, 0u);
 #pragma unroll
-        for (int b = 0; b < 5; ++b)
-            if ((lane >> b) & 1) {
+        for (int b = 0; b < 6; ++b)
+            if ((q >> b) & 1) {
                 z.x ^= qa[b];
                 z.y ^= qb[b];
             }
-        s.zq[lane] = z;
+        s.zq[q] = z;
     }
 #pragma unroll
     for (int k = 0; k < kMaxKChunks; ++k) {

@@ -312,6 +312,24 @@ dpb_status resolve_and_build(const dpb_config *in, const uint32_t *generators, d
                     p->VH[((size_t)k * 32 + q) * 32 + v] = w;
                 }
     }
+    // the same words for every 32-coordinate block of d <= 2048, [chunk][block][v]
+    if (c.d <= 2048) {
+        const int nblk = (c.d + 31) / 32, nk = std::max(p->kvh, 2);
+        p->VH2.assign((size_t)nk * nblk * 32, 0u);
+        for (int k = 0; k < p->kvh; ++k)
+            for (int q = 0; q < nblk; ++q)
+                for (int v = 0; v < 32; ++v) {
+                    uint32_t w = 0;
+                    const uint32_t mask = (uint32_t)v << (5 * k);
+                    for (int l = 0; l < 32; ++l) {
+                        const int iota = 32 * q + l;
+                        if (iota >= c.d) continue;
+                        const uint32_t kappa = p->M[iota] >> c.field_t;
+                        w |= (uint32_t)(__builtin_popcount(kappa & mask) & 1) << l;
+                    }
+                    p->VH2[((size_t)k * nblk + q) * 32 + v] = w;
+                }
+    }
     p->cfg = c;
     build_mma_tables(p);
     if (c.select_mode == DPB_SELECT_PER_LEVEL) build_per_level_tables(p);
