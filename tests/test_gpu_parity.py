@@ -262,6 +262,21 @@ def test_no_norm_match_and_odd_width(norm_match):
     _check_all(plan, ref, x, g, gy=gy)
 
 
+@pytest.mark.parametrize("d,dtype", [(2048, "bf16"), (1600, "f32")])
+def test_wide_rows_global_mode(d, dtype):
+    # d up to 2048 in the table-driven decode and backward (64 blocks of 32
+    # coordinates, t = 11 with three 5-bit chunks of the inverse half); 1600
+    # leaves a partial last block
+    plan = dpb.Plan(d=d, levels=3, m_bits=22, children=16, beam=4, k=24, dtype=dtype)
+    ref = _ref(plan)
+    x = inputs.gaussian_rows(21, d, 41)
+    x = inputs.to_bf16(x) if dtype == "bf16" else x
+    gy = inputs.normal((21, d), 42)
+    gy = inputs.to_bf16(gy) if dtype == "bf16" else gy
+    g = _gpu(plan, x, gy_np=gy)
+    _check_all(plan, ref, x, g, gy=gy)
+
+
 def test_limits_config():
     # beam 32, 256 children per parent, k = 256, L = 3, bf16
     plan = dpb.Plan(d=512, levels=3, m_bits=21, children=256, beam=32, k=256, dtype="bf16")

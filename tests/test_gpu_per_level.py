@@ -99,11 +99,13 @@ def test_paper_2l_layout_with_backward():
 
 
 def test_paper_2l_layout_d2048():
-    # PT-Large-2L: d = 2048 (t = 11, three 5-bit chunks of the inverse half)
+    # PT-Large-2L: d = 2048 (t = 11, three 5-bit chunks of the inverse half,
+    # 64 blocks of 32 coordinates in the decode and backward tables)
     kls = [16, 32]
     plan, ref = _plan_ref(2048, [11, 15], [0, 256], kls)
     x = inputs.to_bf16(inputs.gaussian_rows(9, 2048, 5))
-    _check(plan, ref, kls, x, _gpu(plan, x))
+    gy = inputs.to_bf16(inputs.normal((9, 2048), 6))
+    _check(plan, ref, kls, x, _gpu(plan, x, gy_np=gy), gy=gy)
 
 
 @pytest.mark.parametrize("T", [1, 2, 5, 130])
