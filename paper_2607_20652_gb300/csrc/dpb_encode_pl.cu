@@ -47,6 +47,7 @@ constexpr int kChunk = 64;      // coordinates per K chunk
 constexpr int kATile = 128 * kChunk * 2;  // one M = 128 tile of a chunk
 constexpr int kSelCap = 256;    // gathered candidates per token and level (up to 8 per lane)
 constexpr int kMaxK = 64;       // K_l per level
+constexpr int kMaxStages = 4;   // generator-tile stages in flight
 constexpr uint32_t kSpin = 1u << 20;  // bound of every mbarrier wait
 // at least this much shared memory per block, so that one block (holding all
 // 512 TMEM columns) runs per SM
@@ -60,7 +61,7 @@ struct Args {
     float *val, *xnorm;
     int32_t *status;
     const uint32_t *GT, *G, *VH2;
-    int d, nblk, levels, t, kvh, code_len, dmax;
+    int d, nblk, levels, t, kvh, code_len, dmax, nbs;
     int kl[DPB_MAX_LEVELS], delta[DPB_MAX_LEVELS], off[DPB_MAX_LEVELS];
     int64_t gt_off[DPB_MAX_LEVELS];
     float inv_sqrt_d;
@@ -68,24 +69,28 @@ struct Args {
 
 // ---- layout --------------------------------------------------------------------
 
-constexpr int kWarpBytes = 4 * kRows /* parents */ + 4 * kSelCap /* z */ + 4 * kSelCap /* index */;
+constexpr int kSelBytes = 8 * kSelCap;  // a warp's gathered (z, index) pairs
 
 struct Layout {
-    int a, b, xw, vh, g, w5, warps, mbar, total;
+    int a, b, xw, vh, g, w5, par, mbar, total;
 };
 
-__host__ __device__ inline Layout layout(int d, int levels, int kvh, int dmax) {
+// The gathered candidates of the 8 warps share the generator-tile stages: a
+// level's selection starts once its MMAs are done and before the next
+// level's tiles are copied.
+__host__ __device__ inline Layout layout(int d, int levels, int kvh, int dmax, int nbs) {
     const int nblk = d / 32;
+    const int bbytes = nbs * dmax * 128 > kTokens * kSelBytes ? nbs * dmax * 128 : kTokens * kSelBytes;
     Layout l;
     l.a = 0;
     l.b = l.a + 2 * 2 * kATile;  // 2 stages x 2 tiles
-    l.xw = l.b + 2 * dmax * 128;
+    l.xw = l.b + bbytes;
     l.vh = l.xw + kTokens * nblk * 16 * 4;
     l.g = l.vh + kvh * nblk * 32 * 4;
     l.w5 = l.g + levels * 256 * 4;
-    l.warps = l.w5 + 32 * 4;
-    l.mbar = l.warps + kTokens * kWarpBytes;
-    l.total = l.mbar + 4 * 8 + 16;
+    l.par = l.w5 + 32 * 4;
+    l.mbar = l.par + kTokens * kRows * 4;
+    l.total = l.mbar + 2 * kMaxStages * 8 + 16;
     return l;
 }
 
@@ -352,22 +357,19 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
     extern __shared__ __align__(1024) uint8_t smem[];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int d = a.d, nblk = a.nblk, L = a.levels;
-    const Layout lay = layout(d, L, a.kvh, a.dmax);
+    const Layout lay = layout(d, L, a.kvh, a.dmax, a.nbs);
     uint8_t *sA = smem + lay.a;
     uint8_t *sB = smem + lay.b;
     uint32_t *xw = reinterpret_cast<uint32_t *>(smem + lay.xw);
     uint32_t *vh = reinterpret_cast<uint32_t *>(smem + lay.vh);
     uint32_t *gs = reinterpret_cast<uint32_t *>(smem + lay.g);
     uint32_t *w5 = reinterpret_cast<uint32_t *>(smem + lay.w5);
-    uint64_t *mbar = reinterpret_cast<uint64_t *>(smem + lay.mbar);  // full_b[2], mma_done[2]
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(mbar + 4);
+    uint64_t *mbar = reinterpret_cast<uint64_t *>(smem + lay.mbar);  // full_b[stages], mma_done[stages]
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(mbar + 2 * kMaxStages);
     WarpBufs wb;
-    {
-        uint8_t *base = smem + lay.warps + warp * kWarpBytes;
-        wb.par = reinterpret_cast<uint32_t *>(base);
-        wb.z = reinterpret_cast<float *>(base + 4 * kRows);
-        wb.id = reinterpret_cast<uint32_t *>(base + 4 * kRows + 4 * kSelCap);
-    }
+    wb.par = reinterpret_cast<uint32_t *>(smem + lay.par) + warp * kRows;
+    wb.z = reinterpret_cast<float *>(sB + warp * kSelBytes);
+    wb.id = reinterpret_cast<uint32_t *>(sB + warp * kSelBytes + 4 * kSelCap);
     for (int i = tid; i < a.kvh * nblk * 32; i += blockDim.x) vh[i] = a.VH2[i];
     for (int i = tid; i < L * 256; i += blockDim.x) gs[i] = a.G[(i >> 8) * DPB_MAX_CHILDREN + (i & 255)];
     if (tid < 32) {
@@ -376,7 +378,8 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
         w5[tid] = word;
     }
     if (tid == 0) {
-        for (int i = 0; i < 4; ++i) asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(mbar + i)));
+        for (int i = 0; i < 2 * kMaxStages; ++i)
+            asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(mbar + i)));
         asm volatile("fence.mbarrier_init.release.cluster;");
     }
     if (warp == 0) {
@@ -386,9 +389,18 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
     __syncthreads();
     asm volatile("tcgen05.fence::after_thread_sync;");
     const uint32_t tmem = *tmem_slot;
-    const uint32_t full_b[2] = {smem_u32(mbar), smem_u32(mbar + 1)};
-    const uint32_t mma_done[2] = {smem_u32(mbar + 2), smem_u32(mbar + 3)};
-    uint32_t issued[2] = {0u, 0u}, waited[2] = {0u, 0u}, bcopies[2] = {0u, 0u};
+    // Chunk g (counted over every level and group) uses A stage g & 1 and
+    // generator stage g % nbs; its copy completes full_b[g % nbs] and its MMAs'
+    // commit mma_done[g % nbs], each the (g / nbs)-th time, so the parity of
+    // that count names the phase to wait for. Waits never fall a phase behind:
+    // a stage is refilled only after the MMAs that read it are seen done.
+    const int nbs = a.nbs;
+    const uint32_t mbar0 = smem_u32(mbar);
+    auto full_b = [&](uint32_t g) { return mbar0 + 8u * (g % (uint32_t)nbs); };
+    auto mma_done = [&](uint32_t g) { return mbar0 + 8u * (kMaxStages + g % (uint32_t)nbs); };
+    auto phase = [&](uint32_t g) { return (g / (uint32_t)nbs) & 1u; };
+    auto stage_b = [&](uint32_t g) { return sB + (g % (uint32_t)nbs) * a.dmax * 128; };
+    uint32_t G = 0;  // chunks whose MMAs were committed
     bool failed = false;
     const uint32_t lo_mask = (1u << a.t) - 1u;
     const int64_t ngroups = (a.T + kTokens - 1) / kTokens;
@@ -445,7 +457,7 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
                 const int tokw = pp == 32 ? q + 4 * tt : q + 4 * (jj >> 4);
                 const int slot = pp == 32 ? jj : jj & 15;
                 const bool ok = tt < ntiles && grp * kTokens + tokw < a.T && slot < P;
-                const uint32_t *par = reinterpret_cast<const uint32_t *>(smem + lay.warps + tokw * kWarpBytes);
+                const uint32_t *par = reinterpret_cast<const uint32_t *>(smem + lay.par) + tokw * kRows;
                 const uint32_t pv = ok ? par[slot] : 0u;
                 irv[tt] = ok;
                 ip[tt] = pv;
@@ -457,24 +469,24 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
             }
             const uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(D >> 3) << 17) | (8u << 24);
             const uint32_t *gt = a.GT + a.gt_off[l];
+            const uint32_t G0 = G;
+            // the level's first nbs - 1 tiles (every earlier MMA is done, so
+            // every stage is free)
+            if (tid == 0)
+                for (int c = 0; c < min(nbs - 1, nch); ++c)
+                    copy_b(stage_b(G0 + c), gt + (int64_t)c * D * 32, D, full_b(G0 + c));
             for (int c = 0; c < nch; ++c) {
-                const int s = c & 1;
+                const uint32_t g = G0 + c;
                 {
-                    // the MMAs that last read this stage (thread 0 may have seen
-                    // them already, when it prefetched this chunk's B)
+                    // A stage g & 1 is free once the MMAs of chunk g - 2 are done
                     bool ok = true;
-                    if (issued[s] > waited[s]) {
-                        ok = mbar_wait(mma_done[s], waited[s] & 1u);
-                        if (ok) ++waited[s];
-                    }
+                    if (c >= 2) ok = mbar_wait(mma_done(g - 2), phase(g - 2));
                     if (__syncthreads_or(!ok)) {  // every thread leaves together
                         failed = true;
                         break;
                     }
                 }
-                uint8_t *As = sA + s * 2 * kATile;
-                uint8_t *Bt = sB + s * a.dmax * 128;
-                if (tid == 0 && c == 0) copy_b(Bt, gt, D, full_b[s]);  // later chunks: prefetched below
+                uint8_t *As = sA + (g & 1u) * 2 * kATile;
 #pragma unroll
                 for (int tt = 0; tt < 2; ++tt) {
                     if (tt < ntiles) {
@@ -503,11 +515,11 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
                 asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                 __syncthreads();
                 if (tid == 0) {
-                    if (!mbar_wait(full_b[s], bcopies[s] & 1u)) {
+                    if (!mbar_wait(full_b(g), phase(g))) {
                         set_status(a.status, DPB_DEV_TIMEOUT);  // the commit below still arrives
                     } else {
                         asm volatile("tcgen05.fence::after_thread_sync;");
-                        const uint32_t bb = smem_u32(Bt);
+                        const uint32_t bb = smem_u32(stage_b(g));
                         for (int tt = 0; tt < ntiles; ++tt) {
                             const uint32_t ab = smem_u32(As + tt * kATile);
 #pragma unroll
@@ -520,35 +532,28 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
                             }
                         }
                     }
-                    ++bcopies[s];
                     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-                        mma_done[s]));
-                    // prefetch the next chunk's B into the other stage once the
-                    // MMAs that read it (chunk c - 1) are done
-                    if (c + 1 < nch) {
-                        const int s1 = s ^ 1;
-                        bool ok = true;
-                        if (issued[s1] > waited[s1]) {
-                            ok = mbar_wait(mma_done[s1], waited[s1] & 1u);
-                            if (ok) ++waited[s1];
-                        }
+                        mma_done(g)));
+                    // the tile nbs - 1 chunks ahead goes to the stage chunk g - 1
+                    // read, once its MMAs are done
+                    if (c + nbs - 1 < nch) {
+                        const bool ok = c == 0 || mbar_wait(mma_done(g - 1), phase(g - 1));
                         if (ok)
-                            copy_b(sB + s1 * a.dmax * 128, gt + (int64_t)(c + 1) * D * 32, D, full_b[s1]);
+                            copy_b(stage_b(g + nbs - 1), gt + (int64_t)(c + nbs - 1) * D * 32, D, full_b(g + nbs - 1));
                         else
                             set_status(a.status, DPB_DEV_TIMEOUT);
                     }
                 }
-                ++issued[s];
+                G = g + 1;
             }
             if (failed) break;
             {
-                const int s = (nch - 1) & 1;  // the last commit covers every MMA of the level
-                const bool ok = mbar_wait(mma_done[s], waited[s] & 1u);
+                // the last commit covers every MMA of the level
+                const bool ok = mbar_wait(mma_done(G - 1), phase(G - 1));
                 if (__syncthreads_or(!ok)) {
                     failed = true;
                     break;
                 }
-                ++waited[s];
             }
             asm volatile("tcgen05.fence::after_thread_sync;");
             // ---- the level's selection, one warp per token ----
@@ -580,12 +585,8 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
         }
     }
     if (failed) set_status(a.status, DPB_DEV_TIMEOUT);
-    // drain: every commit issued is waited for (bounded) before TMEM is freed
-    for (int s = 0; s < 2; ++s)
-        while (issued[s] > waited[s]) {
-            if (!mbar_wait(mma_done[s], waited[s] & 1u)) break;
-            ++waited[s];
-        }
+    // drain: the last commit is waited for (bounded) before TMEM is freed
+    if (failed && G > 0) mbar_wait(mma_done(G - 1), phase(G - 1));
     asm volatile("tcgen05.fence::before_thread_sync;");
     __syncthreads();
     if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" ::"r"(tmem));
@@ -647,12 +648,27 @@ void build_per_level_tables(dpb_plan *p) {
     // (VH2, the inverse-coordinate sign words per block, is built with the plan)
 }
 
-size_t encode_pl_smem(const dpb_plan *p) {
-    const dpb_config &c = p->cfg;
+namespace {
+
+// Generator-tile stages: as many as fit (at least 2).
+int pl_stages(const dpb_config &c, int kvh, int dmax) {
+    for (int nbs = kMaxStages; nbs > 2; --nbs)
+        if ((size_t)layout(c.d, c.levels, kvh, dmax, nbs).total <= kMaxSmemPerBlock) return nbs;
+    return 2;
+}
+
+int pl_dmax(const dpb_config &c) {
     int dmax = 16;
     for (int l = 1; l < c.levels; ++l) dmax = std::max(dmax, c.children[l]);
-    const int kvh = std::max(1, (c.field_t + 4) / 5);
-    return (size_t)std::max(layout(c.d, c.levels, kvh, dmax).total, kMinSmem);
+    return dmax;
+}
+
+}  // namespace
+
+size_t encode_pl_smem(const dpb_plan *p) {
+    const dpb_config &c = p->cfg;
+    const int dmax = pl_dmax(c), kvh = std::max(1, (c.field_t + 4) / 5);
+    return (size_t)std::max(layout(c.d, c.levels, kvh, dmax, pl_stages(c, kvh, dmax)).total, kMinSmem);
 }
 
 cudaError_t launch_encode_pl(const dpb_plan *p, const void *x, int64_t T, const float *mu, const float *sigma,
@@ -687,6 +703,7 @@ cudaError_t launch_encode_pl(const dpb_plan *p, const void *x, int64_t T, const 
         if (l) a.dmax = std::max(a.dmax, c.children[l]);
     }
     a.inv_sqrt_d = p->inv_sqrt_d;
+    a.nbs = pl_stages(c, a.kvh, a.dmax);
     const size_t smem = encode_pl_smem(p);
     const cudaError_t e = cudaFuncSetAttribute(encode_pl_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
