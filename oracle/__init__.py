@@ -81,6 +81,8 @@ def _load():
             "orc_decode": (i32, [i32, i32, i32, p, p, p, i64, p, p]),
             "orc_backward": (i32, [i32, i32, i32, p, p, p, p, i64, p, p, p, p]),
             "orc_gf_tables": (None, [i32, u32, p, p, p]),
+            "orc_stats_accumulate": (i32, [i32, i32, p, p, p, p, i32, p, i64, p, p, p, i32, p, i64]),
+            "orc_stats_update": (None, [i64, p, dbl, p, p]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(lib, name)
@@ -310,3 +312,47 @@ def backward(cfg: Config, x, idx, val, gy, sigma=None, norm_match: Optional[int]
     _load().orc_backward(cfg.d, k, nm, _ptr(cfg.M), _ptr(x), _ptr(idx), _ptr(val), T, _ptr(sg),
                          _ptr(gy), _ptr(gx), _ptr(gv))
     return gx, gv
+
+
+# ----------------------------------------------------------------------------
+# standardisation moments (§2.2 "Score Standardization")
+# ----------------------------------------------------------------------------
+
+def keep_per_level(cfg: Config) -> list:
+    """Kept-set size of every level: the beam (global mode) or K_l (per-level)."""
+    if cfg.k_per_level:
+        return list(cfg.k_per_level[: cfg.levels])
+    return [cfg.beam] * cfg.levels
+
+
+def stats_accumulate(cfg: Config, x, sample, mu=None, sigma=None, acc=None):
+    """Moment sums [3, 2^N] (count, sum s, sum s^2): level 0 over every row of
+    x, levels >= 1 over the rows listed in ``sample`` (readings R16, R18).
+    Adds to ``acc`` when given (float64 [3, 2^N], C order)."""
+    x = _f64(x)
+    T = x.shape[0]
+    m = 1 << cfg.m_bits
+    if acc is None:
+        acc = np.zeros((3, m), dtype=np.float64)
+    assert acc.shape == (3, m) and acc.dtype == np.float64 and acc.flags.c_contiguous
+    smp = np.ascontiguousarray(np.asarray(sample, dtype=np.int32).reshape(-1))
+    mu = None if mu is None else _f64(mu)
+    sigma = None if sigma is None else _f64(sigma)
+    rc = _load().orc_stats_accumulate(cfg.d, cfg.levels, _ptr(_i32(cfg.children)),
+                                      _ptr(_i32(keep_per_level(cfg))), _ptr(cfg.M), _ptr(cfg.G),
+                                      GSTRIDE, _ptr(x), T, _ptr(mu), _ptr(sigma),
+                                      _ptr(smp) if smp.size else None, int(smp.size), _ptr(acc), m)
+    if rc != 0:
+        raise ValueError(f"oracle stats accumulate failed ({rc})")
+    return acc
+
+
+def stats_update(acc, alpha: float, mu, sigma):
+    """One EMA step (reading R17). Returns new (mu, sigma) as float64 copies;
+    ``acc`` is zeroed in place."""
+    assert acc.dtype == np.float64 and acc.flags.c_contiguous and acc.shape[0] == 3
+    m = acc.shape[1]
+    mu2 = np.array(mu, dtype=np.float64, copy=True).reshape(m)
+    sg2 = np.array(sigma, dtype=np.float64, copy=True).reshape(m)
+    _load().orc_stats_update(m, _ptr(acc), float(alpha), _ptr(mu2), _ptr(sg2))
+    return mu2, sg2

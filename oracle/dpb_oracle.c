@@ -38,6 +38,15 @@
  *   R10 global selection: beam B at every level, final code = top k over
  *       every candidate visited (all d basis entries and every level's set).
  *   R12 normalised output: y = r * |x| / |r|, and y = 0 when |r| = 0.
+ *   R16 a feature is "considered" on a token when the search scores it
+ *       there: every basis coordinate on every token (level 0), every
+ *       distinct child of the previous level's kept set (level >= 1).
+ *   R17 the EMA step: with n considered occurrences in the sample, mean
+ *       m = (sum s) / n and population deviation v = sqrt(sum s^2 / n - m^2);
+ *       mu += alpha (m - mu) when n >= 1, sigma += alpha (v - sigma) when
+ *       n >= 2; untouched features keep their moments.
+ *   R18 level 0 takes every token of the batch, levels >= 1 a caller-given
+ *       list of token rows (the paper's 64-token sub-sample).
  */
 #include <math.h>
 #include <stdint.h>
@@ -484,6 +493,130 @@ int orc_encode_per_level(int d, int levels, const int *children, const int *k_pe
     free(lvl);
     free(parents);
     return rc;
+}
+
+/* ------------------------------------------------------------------ */
+/* Standardisation moments  (§2.2 "Score Standardization"; R16-R18)     */
+/* ------------------------------------------------------------------ */
+
+/*
+ * Adds the moment sums of the raw scores s to acc, three arrays of m doubles
+ * (count, sum of s, sum of s^2), over the occurrences where a feature is a
+ * candidate (R16, R18):
+ *   level 0    every basis coordinate i < d on every token t < T: s = x_t[i];
+ *   level l>0  on each sampled token only: every distinct child p ^ g_j of the
+ *              previous level's kept set, s = <phi_c, x_t>.
+ * The kept set of a level is its top keep[l] candidates by standardised score
+ * (R9 order; mu/sigma as in the encoder, both NULL = identity), so the search
+ * is the encoder's: keep[l] = beam (global mode) or K_l (per-level mode).
+ * Returns 0, or -1 on bad arguments (a sampled row outside [0, T)).
+ */
+int orc_stats_accumulate(int d, int levels, const int *children, const int *keep,
+                         const uint32_t *M, const uint32_t *G, int gstride,
+                         const double *x, long T, const double *mu, const double *sigma,
+                         const int32_t *sample, int n_sample, double *acc, long m)
+{
+    if (d < 1 || levels < 1 || levels > ORC_MAX_LEVELS || m < d || n_sample < 0)
+        return -1;
+    for (int s = 0; s < n_sample; s++)
+        if (sample[s] < 0 || sample[s] >= T)
+            return -1;
+    double *cnt = acc, *sum = acc + m, *sq = acc + 2 * m;
+
+    /* level 0: every token considers every basis coordinate */
+    for (long t = 0; t < T; t++)
+        for (int i = 0; i < d; i++) {
+            double v = x[t * d + i];
+            cnt[i] += 1.0;
+            sum[i] += v;
+            sq[i] += v * v;
+        }
+
+    long cap = d;
+    for (int l = 1; l < levels; l++)
+        if ((long)keep[l - 1] * children[l] > cap)
+            cap = (long)keep[l - 1] * children[l];
+    cand_t *lvl = (cand_t *)malloc(sizeof(cand_t) * (size_t)cap);
+    double *raw = (double *)malloc(sizeof(double) * (size_t)cap);
+    uint32_t *parents = (uint32_t *)malloc(sizeof(uint32_t) * (size_t)cap);
+    if (!lvl || !raw || !parents) {
+        free(lvl);
+        free(raw);
+        free(parents);
+        return -1;
+    }
+    for (int s = 0; s < n_sample; s++) {
+        const double *xt = x + (long)sample[s] * d;
+        int nl = 0;
+        for (int i = 0; i < d; i++) {
+            lvl[nl].idx = (uint32_t)i;
+            lvl[nl].z = standardise(xt[i], (uint32_t)i, mu, sigma);
+            lvl[nl].exact = 0;
+            nl++;
+        }
+        for (int l = 1; l < levels; l++) {
+            /* kept set of level l-1 */
+            qsort(lvl, (size_t)nl, sizeof(cand_t), cand_cmp);
+            int np = nl < keep[l - 1] ? nl : keep[l - 1];
+            for (int b = 0; b < np; b++)
+                parents[b] = lvl[b].idx;
+            /* the distinct children of the kept set (R8) */
+            nl = 0;
+            for (int b = 0; b < np; b++) {
+                for (int j = 0; j < children[l]; j++) {
+                    uint32_t c = parents[b] ^ G[l * gstride + j];
+                    int seen = 0;
+                    for (int q = 0; q < nl; q++)
+                        if (lvl[q].idx == c)
+                            seen = 1;
+                    if (!seen) {
+                        lvl[nl].idx = c;
+                        lvl[nl].exact = 0;
+                        nl++;
+                    }
+                }
+            }
+            /* each is considered once on this token: its raw score joins the sums */
+            for (int q = 0; q < nl; q++) {
+                uint32_t c = lvl[q].idx;
+                raw[q] = direct_score(d, M, c, xt);
+                if ((long)c < m) {
+                    cnt[c] += 1.0;
+                    sum[c] += raw[q];
+                    sq[c] += raw[q] * raw[q];
+                }
+                lvl[q].z = standardise(raw[q], c, mu, sigma);
+            }
+        }
+    }
+    free(lvl);
+    free(raw);
+    free(parents);
+    return 0;
+}
+
+/*
+ * One EMA step of the standardisation tables from the sums of
+ * orc_stats_accumulate (R17), then acc = 0. For feature i with n = acc
+ * count >= 1: m = sum / n, mu_i += alpha (m - mu_i); with n >= 2 also
+ * v = sqrt(max(sum s^2 / n - m^2, 0)), sigma_i += alpha (v - sigma_i).
+ */
+void orc_stats_update(long m, double *acc, double alpha, double *mu, double *sigma)
+{
+    double *cnt = acc, *sum = acc + m, *sq = acc + 2 * m;
+    for (long i = 0; i < m; i++) {
+        double n = cnt[i];
+        if (n >= 1.0) {
+            double mean = sum[i] / n;
+            mu[i] += alpha * (mean - mu[i]);
+            if (n >= 2.0) {
+                double var = sq[i] / n - mean * mean;
+                double v = sqrt(var > 0.0 ? var : 0.0);
+                sigma[i] += alpha * (v - sigma[i]);
+            }
+        }
+        cnt[i] = sum[i] = sq[i] = 0.0;
+    }
 }
 
 /* ------------------------------------------------------------------ */

@@ -1,7 +1,8 @@
 """Each pin must fail on a plausible mistake. These tests plant the mistake in
 a copy of the oracle's outputs (on the CPU) and check that the pin notices:
 swapped halves of the seed matrix, a flipped sign map, a wrong inverse,
-a dropped normalisation, a dropped 1/sigma or norm term in the backward."""
+a dropped normalisation, a dropped 1/sigma or norm term in the backward,
+sampled rows counted at level 0 and a sample deviation in the EMA step."""
 import math
 
 import numpy as np
@@ -79,3 +80,24 @@ def test_order_invariant_catches_reversed_tie_break():
     assert keys == sorted(keys) and idx[0, :3].tolist() == [3, 9, 20]
     rev = [(-abs(v), -i) for i, v in zip(idx[0], val[0])]                   # index descending
     assert rev != sorted(rev)
+
+
+def test_moment_pins_catch_level0_and_deviation_mistakes():
+    cfg = oracle.resolve(d=64, m_bits=12, levels=3, children=16, beam=4, k=8)
+    x = np.random.default_rng(7).standard_normal((20, cfg.d))
+    acc = oracle.stats_accumulate(cfg, x, sample=[1, 2])
+    assert pins.column_moment_mismatch(acc, x, cfg.d) < 1e-10
+    twice = acc.copy()
+    twice[:, : cfg.d] += oracle.stats_accumulate(cfg, x[[1, 2]], sample=[])[:, : cfg.d]
+    assert pins.column_moment_mismatch(twice, x, cfg.d) > 1.0      # sampled rows counted again
+    m = 1 << cfg.m_bits
+    samples = {i: x[:, i] for i in range(cfg.d)}
+    acc0 = oracle.stats_accumulate(cfg, x, sample=[])
+    mu, sg = oracle.stats_update(acc0, 0.5, np.zeros(m), np.ones(m))
+    assert pins.ema_mismatch(mu, sg, np.zeros(m), np.ones(m), 0.5, samples) < 1e-12
+    ddof1 = sg.copy()
+    ddof1[: cfg.d] = 0.5 + 0.5 * x.std(axis=0, ddof=1)            # sample (n - 1) deviation
+    assert pins.ema_mismatch(mu, ddof1, np.zeros(m), np.ones(m), 0.5, samples) > 1e-3
+    raw2 = sg.copy()
+    raw2[: cfg.d] = 0.5 + 0.5 * np.sqrt((x * x).mean(axis=0))      # second moment, not deviation
+    assert pins.ema_mismatch(mu, raw2, np.zeros(m), np.ones(m), 0.5, samples) > 1e-3
