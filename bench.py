@@ -32,6 +32,8 @@ if ROOT not in sys.path:
 
 METRIC = "DPB tokens/sec (encode+decode+bwd) at d=768, 2^20 feats, 1 GB300; % of roofline"
 WORKLOAD = "wide"
+EMA_SAMPLE = 64        # rows per batch for the level >= 1 moments (§2.2 "Score Standardization")
+EMA_ALPHA = 0.01       # EMA weight of one batch
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
                   "sm_max_mhz": 2070.0}
 GB300_SMS = 152
@@ -324,12 +326,17 @@ def run_reference(args, world, rank):
     return 0
 
 
-def config_block(w, world, n_tokens=None):
-    return {"workload": WORKLOAD, "T_per_gpu": n_tokens or w["T"], "d": w["d"], "features": 2 ** w["m_bits"],
-            "levels": w["levels"], "children": w["children"], "beam": w["beam"], "k": w["k"],
-            "accumulate": "fp32", "inputs": "planted tree of 64 parity directions + N(0,0.1^2), bf16",
-            "l2": "working set ~450 MB > 129 MB L2 (no flush needed)",
-            "parallelism": f"dp{world} (independent token shards)"}
+def config_block(w, world, n_tokens=None, standardise=False):
+    c = {"workload": WORKLOAD, "T_per_gpu": n_tokens or w["T"], "d": w["d"], "features": 2 ** w["m_bits"],
+         "levels": w["levels"], "children": w["children"], "beam": w["beam"], "k": w["k"],
+         "accumulate": "fp32", "inputs": "planted tree of 64 parity directions + N(0,0.1^2), bf16",
+         "l2": "working set ~450 MB > 129 MB L2 (no flush needed)",
+         "parallelism": f"dp{world} (independent token shards)"}
+    if standardise:
+        c["standardise"] = {"tables": "live fp32 mu/sigma (2^N each)", "ema_sample_rows": EMA_SAMPLE,
+                            "ema_alpha": EMA_ALPHA,
+                            "exchange": "all-reduce of the fp64 moment sums" if world > 1 else "none (1 rank)"}
+    return c
 
 
 def run_ours(args, world, rank, local):
@@ -356,26 +363,43 @@ def run_ours(args, world, rank, local):
     gv = torch.empty((T, k), dtype=torch.float32, device=device)
     ws = plan.workspace(T, device)
     stream = torch.cuda.current_stream(device)
+    # live standardisation (§2.2): encode and backward read the tables, and
+    # each step ends with the EMA update from the level-0 column sums and a
+    # 64-row sub-sample (tables start at mu = 0, sigma = 1)
+    std = args.standardise
+    mu_t = sg_t = acc = None
+    samples = []
+    if std:
+        mu_t = torch.zeros(plan.n_features, dtype=torch.float32, device=device)
+        sg_t = torch.ones(plan.n_features, dtype=torch.float32, device=device)
+        acc = dpb.stats_buffer(plan, device)
+        gen = torch.Generator().manual_seed(seed)
+        samples = [dpb.sample_rows(T, EMA_SAMPLE, gen, device) for _ in range(max(args.steps, args.warmup))]
+    stages = ["encode", "decode", "backward"] + (["stats"] if std else [])
 
-    def step(ev=None):
+    def step(ev=None, i=0):
         if ev:
             ev[0].record(stream)
-        dpb.encode(plan, x, idx=idx, val=val, xnorm=xn, workspace=ws, stream=stream)
+        dpb.encode(plan, x, mu_t, sg_t, idx=idx, val=val, xnorm=xn, workspace=ws, stream=stream)
         if ev:
             ev[1].record(stream)
         dpb.decode(plan, idx, val, xn, y=y, workspace=ws, stream=stream)
         if ev:
             ev[2].record(stream)
-        dpb.backward(plan, x, idx, val, gy, grad_x=gx, grad_val=gv, workspace=ws, stream=stream)
+        dpb.backward(plan, x, idx, val, gy, sigma=sg_t, grad_x=gx, grad_val=gv, workspace=ws, stream=stream)
         if ev:
             ev[3].record(stream)
+        if std:
+            dpb.stats_step(plan, x, mu_t, sg_t, EMA_ALPHA, samples[i], acc=acc, workspace=ws, stream=stream)
+            if ev:
+                ev[4].record(stream)
 
-    for _ in range(args.warmup):
-        step()
+    for i in range(args.warmup):
+        step(None, i)
     torch.cuda.synchronize(device)
     status = dpb.workspace_status(ws)
 
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(len(stages) + 1)] for _ in range(args.steps)]
     gpu_id = None
     try:
         gpu_id = "GPU-" + str(torch.cuda.get_device_properties(device).uuid)
@@ -390,19 +414,16 @@ def run_ours(args, world, rank, local):
     end = torch.cuda.Event(enable_timing=True)
     start.record(stream)
     for i in range(args.steps):
-        step(evs[i])
+        step(evs[i], i)
     end.record(stream)
     torch.cuda.synchronize(device)
     barrier(world)
     clk = clocks.stop()
     ms = start.elapsed_time(end)
     ms_max = max_over_ranks(ms, world, device)
-    per = {"encode": [], "decode": [], "backward": []}
-    for e in evs:
-        per["encode"].append(e[0].elapsed_time(e[1]))
-        per["decode"].append(e[1].elapsed_time(e[2]))
-        per["backward"].append(e[2].elapsed_time(e[3]))
-    kern_ms = {n: statistics.mean(v) for n, v in per.items()}
+    kern_ms = {n: statistics.mean(e[j].elapsed_time(e[j + 1]) for e in evs) for j, n in enumerate(stages)}
+    if std:
+        status |= dpb.workspace_status(ws)
 
     # algorithmic work and roofline of the dominant kernel
     idx_np = idx.cpu().numpy()
@@ -410,6 +431,9 @@ def run_ours(args, world, rank, local):
     recovered = float(np.mean([len(set(idx_np[t]) & set(idx_true[t])) / k for t in range(0, T, 64)]))
     peaks, src = load_peaks()
     work = algorithmic_work(plan.config, T, k_hash, 2)
+    if std:
+        # the column pass reads x once; the update scans the 2^N counts
+        work["stats"] = {"bytes": T * d * 2 + 8 * plan.n_features}
     dom = max(kern_ms, key=kern_ms.get)
     roof = roofline_for(dom, work[dom], kern_ms[dom] / 1e3, peaks, src, measured_traffic(dom, T))
     kernels = {n: {"ms": round(v, 4), **{kk: vv for kk, vv in roofline_for(n, work[n], v / 1e3, peaks, src).items()
@@ -419,7 +443,7 @@ def run_ours(args, world, rank, local):
 
     # end to end through the public API with host buffers
     e2e = None
-    if not args.no_e2e:
+    if not args.no_e2e and not std:
         e2e = run_e2e(plan, x, gy, args, device, stream, world)
 
     value = whole_job_rate(T, world, args.steps, ms_max / 1e3)
@@ -427,13 +451,13 @@ def run_ours(args, world, rank, local):
         "metric": METRIC, "value": round(value, 1), "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_max / args.steps, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-        "data": "synthetic", "config": config_block(w, world),
+        "data": "synthetic", "config": config_block(w, world, standardise=std),
         "roofline": roof,
         "step_roofline": {"t_roofline_us": round(step_roof_us, 2),
                           "t_measured_us": round(1e3 * ms_max / args.steps, 2),
                           "frac": round(step_roof_us / (1e3 * ms_max / args.steps), 4)},
         "kernels": kernels, "k_hash": round(k_hash, 2), "planted_recovery": round(recovered, 4),
-        "gpu_launches": 3 * args.steps, "clocks": clk, "device_status": status,
+        "gpu_launches": (3 + (3 if std else 0)) * args.steps, "clocks": clk, "device_status": status,
     }
     if e2e:
         line["e2e"] = e2e
@@ -529,24 +553,38 @@ def run_per_level(args, world, rank, local):
     gv = torch.empty((T, k), dtype=torch.float32, device=device)
     ws = plan.workspace(T, device)
     stream = torch.cuda.current_stream(device)
+    std = args.standardise
+    mu_t = sg_t = acc = None
+    samples = []
+    if std:
+        mu_t = torch.zeros(plan.n_features, dtype=torch.float32, device=device)
+        sg_t = torch.ones(plan.n_features, dtype=torch.float32, device=device)
+        acc = dpb.stats_buffer(plan, device)
+        gen = torch.Generator().manual_seed(seed)
+        samples = [dpb.sample_rows(T, EMA_SAMPLE, gen, device) for _ in range(max(args.steps, args.warmup))]
+    stages = ["encode", "decode", "backward"] + (["stats"] if std else [])
 
-    def step(ev=None):
+    def step(ev=None, i=0):
         if ev:
             ev[0].record(stream)
-        dpb.encode(plan, x, idx=idx, val=val, xnorm=xn, workspace=ws, stream=stream)
+        dpb.encode(plan, x, mu_t, sg_t, idx=idx, val=val, xnorm=xn, workspace=ws, stream=stream)
         if ev:
             ev[1].record(stream)
         dpb.decode(plan, idx, val, xn, y=y, workspace=ws, stream=stream)
         if ev:
             ev[2].record(stream)
-        dpb.backward(plan, x, idx, val, gy, grad_x=gx, grad_val=gv, workspace=ws, stream=stream)
+        dpb.backward(plan, x, idx, val, gy, sigma=sg_t, grad_x=gx, grad_val=gv, workspace=ws, stream=stream)
         if ev:
             ev[3].record(stream)
+        if std:
+            dpb.stats_step(plan, x, mu_t, sg_t, EMA_ALPHA, samples[i], acc=acc, workspace=ws, stream=stream)
+            if ev:
+                ev[4].record(stream)
 
-    for _ in range(args.warmup):
-        step()
+    for i in range(args.warmup):
+        step(None, i)
     torch.cuda.synchronize(device)
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(len(stages) + 1)] for _ in range(args.steps)]
     clocks = ClockSampler(None)
     clocks.start()
     time.sleep(0.3)
@@ -554,17 +592,18 @@ def run_per_level(args, world, rank, local):
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     start.record(stream)
     for i in range(args.steps):
-        step(evs[i])
+        step(evs[i], i)
     end.record(stream)
     torch.cuda.synchronize(device)
     barrier(world)
     clk = clocks.stop()
     ms_max = max_over_ranks(start.elapsed_time(end), world, device)
-    kern_ms = {n: statistics.mean(e[j].elapsed_time(e[j + 1]) for e in evs)
-               for j, n in enumerate(("encode", "decode", "backward"))}
+    kern_ms = {n: statistics.mean(e[j].elapsed_time(e[j + 1]) for e in evs) for j, n in enumerate(stages)}
     k_hash = float(np.mean(np.sum(idx.cpu().numpy() >= d, axis=1)))
     peaks, src = load_peaks()
     work = per_level_work(w, T, k_hash, 2)
+    if std:
+        work["stats"] = {"bytes": T * d * 2 + 8 * plan.n_features}
     kernels = {n: {"ms": round(v, 4), **{kk: vv for kk, vv in roofline_for(n, work[n], v / 1e3, peaks, src).items()
                                           if kk in ("bound", "frac", "t_roofline_us", "achieved", "unit")}}
                for n, v in kern_ms.items()}
@@ -579,9 +618,12 @@ def run_per_level(args, world, rank, local):
         "config": {"workload": args.workload, "T_per_gpu": T, "d": d, "levels": w["levels"], "bits": w["bits"],
                    "children": w["children"], "k_per_level": w["k_per_level"], "select": "per_level",
                    "inputs": "bf16 x ~ N(0,1), grad_y ~ N(0,1)",
-                   "l2": "inputs (2 x 128 MiB) larger than the 129 MB L2 (no flush needed)"},
+                   "l2": "inputs (2 x 128 MiB) larger than the 129 MB L2 (no flush needed)",
+                   **({"standardise": {"tables": "live fp32 mu/sigma (2^N each)", "ema_sample_rows": EMA_SAMPLE,
+                                       "ema_alpha": EMA_ALPHA}} if std else {})},
         "roofline": roofline_for(dom, work[dom], kern_ms[dom] / 1e3, peaks, src),
-        "kernels": kernels, "k_hash": round(k_hash, 2), "gpu_launches": 3 * args.steps, "clocks": clk,
+        "kernels": kernels, "k_hash": round(k_hash, 2), "gpu_launches": (3 + (3 if std else 0)) * args.steps,
+        "clocks": clk,
         "device_status": dpb.workspace_status(ws),
     }
     if rank == 0:
@@ -599,6 +641,8 @@ def main(argv=None):
     ap.add_argument("--ref-tokens", type=int, default=512)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--standardise", action="store_true",
+                    help="live standardisation tables and the per-step EMA update in the timed step")
     ap.add_argument("--workload", default=WORKLOAD, choices=[WORKLOAD, "paper3l", "paper2l"],
                     help="wide (the headline, global selection) or one of the paper's per-level layouts")
     args = ap.parse_args(argv)

@@ -196,6 +196,50 @@ dpb_status dpb_backward(const dpb_plan *plan, const void *x, const int32_t *idx,
                         void *grad_x, float *grad_val, void *workspace,
                         size_t workspace_bytes, void *stream);
 
+/*
+ * dpb_stats_accumulate -- moment sums of the score standardisation (§2.2
+ * "Score Standardization": each feature's score is standardised by EMAs of
+ * its mean and deviation, taken over the tokens on which it is a candidate;
+ * levels >= 1 take them on a 64-token sub-sample of the batch). Adds to acc,
+ * fp64 [3][2^N] = count, sum of s, sum of s^2 per feature, where s is the raw
+ * (unstandardised) score:
+ *   level 0    every row of x: each basis coordinate i < d adds s = x_t[i];
+ *   level >= 1 the rows sample[0..n_sample) only: the encoder's search is run
+ *              again on each (kept set of a level = its top beam, or top
+ *              k_per_level[l] in per-level mode, by |z| under mu/sigma), and
+ *              every distinct child p ^ g_j it scores at a level l >= 1 adds
+ *              s = <phi_c, x_t> (accumulated in fp32).
+ *   x          [T][d] plan dtype, 16-byte aligned
+ *   mu, sigma  the tables the encoder selects with (both NULL = identity)
+ *   sample     device int32 [n_sample] row numbers in [0, T); a row may
+ *              repeat; a row outside [0, T) is skipped and flagged
+ *              DPB_DEV_BAD_INDEX (NULL allowed when n_sample = 0)
+ *   acc        device fp64 [3][2^N] (24 * 2^N bytes, 8-byte aligned, owned by
+ *              the caller), zero before a batch's first call; sums are fp64
+ *              atomics, so their last bits depend on the order of arrival
+ * The search rounds like the encoder but not in the same order: where two
+ * scores sit within fp32 rounding of each other at a kept-set cut, the
+ * candidates counted here can differ from those the encoder visited.
+ * Errors: INVALID_ARG, UNSUPPORTED (a kept set above 64), CUDA.
+ */
+dpb_status dpb_stats_accumulate(const dpb_plan *plan, const void *x, int64_t T, const float *mu,
+                                const float *sigma, const int32_t *sample, int32_t n_sample,
+                                double *acc, void *workspace, size_t workspace_bytes, void *stream);
+
+/*
+ * dpb_stats_update -- one EMA step of the standardisation tables from acc,
+ * then acc = 0. For each feature with n = count >= 1: m = sum / n and
+ * mu += alpha (m - mu); with n >= 2 also v = sqrt(max(sum s^2 / n - m^2, 0))
+ * (the population deviation) and sigma += alpha (v - sigma); features with
+ * n = 0 keep their moments. With 0 < alpha < 1 a positive sigma stays
+ * positive. mu, sigma: device fp32 [2^N], updated in place (fp64 arithmetic,
+ * rounded to fp32). Data-parallel callers sum acc across ranks (one
+ * all-reduce) before this call; every rank then makes the same update.
+ * Errors: INVALID_ARG (alpha outside (0, 1), NULL or misaligned buffers), CUDA.
+ */
+dpb_status dpb_stats_update(const dpb_plan *plan, double *acc, float alpha, float *mu, float *sigma,
+                            void *stream);
+
 /* Read (and with clear != 0, zero) the workspace status word: synchronises
  * `stream`, writes the sticky DPB_DEV_* bits to host *status_out, and returns
  * DPB_ERR_DEVICE if any bit is set, else DPB_OK. */

@@ -227,6 +227,44 @@ dpb_status dpb_backward(const dpb_plan *plan, const void *x, const int32_t *idx,
                     "backward");
 }
 
+dpb_status dpb_stats_accumulate(const dpb_plan *plan, const void *x, int64_t T, const float *mu,
+                                const float *sigma, const int32_t *sample, int32_t n_sample, double *acc,
+                                void *workspace, size_t workspace_bytes, void *stream) {
+    DPB_TRY(check_plan(plan));
+    if (T < 0 || n_sample < 0) return dpb::fail(DPB_ERR_INVALID_ARG, "T < 0 or n_sample < 0");
+    if (T == 0 && n_sample > 0) return dpb::fail(DPB_ERR_INVALID_ARG, "sampled rows of an empty batch");
+    if (T == 0) return DPB_OK;
+    if ((mu == nullptr) != (sigma == nullptr))
+        return dpb::fail(DPB_ERR_INVALID_ARG, "mu and sigma must both be given or both be NULL");
+    if (!dpb::stats_supported(plan, nullptr))
+        return dpb::fail(DPB_ERR_UNSUPPORTED, "kept sets above 64 or the sampled search exceeds shared memory");
+    DPB_TRY(check_rows(x, "x", true));
+    DPB_TRY(check_vec(mu, "mu", false));
+    DPB_TRY(check_vec(sigma, "sigma", false));
+    DPB_TRY(check_vec(sample, "sample", n_sample > 0));
+    if (!acc) return dpb::fail(DPB_ERR_INVALID_ARG, "acc is NULL");
+    if (!aligned(acc, 8)) return dpb::fail(DPB_ERR_INVALID_ARG, "acc must be 8-byte aligned");
+    DPB_TRY(check_workspace(workspace, workspace_bytes));
+    DPB_TRY(check_device(plan));
+    return launched(dpb::launch_stats_accumulate(plan, x, T, mu, sigma, sample, n_sample, acc,
+                                                 static_cast<int32_t *>(workspace),
+                                                 static_cast<cudaStream_t>(stream)),
+                    "stats accumulate");
+}
+
+dpb_status dpb_stats_update(const dpb_plan *plan, double *acc, float alpha, float *mu, float *sigma,
+                            void *stream) {
+    DPB_TRY(check_plan(plan));
+    if (!(alpha > 0.f && alpha < 1.f)) return dpb::fail(DPB_ERR_INVALID_ARG, "alpha must lie in (0, 1)");
+    if (!acc) return dpb::fail(DPB_ERR_INVALID_ARG, "acc is NULL");
+    if (!aligned(acc, 8)) return dpb::fail(DPB_ERR_INVALID_ARG, "acc must be 8-byte aligned");
+    DPB_TRY(check_vec(mu, "mu", true));
+    DPB_TRY(check_vec(sigma, "sigma", true));
+    DPB_TRY(check_device(plan));
+    return launched(dpb::launch_stats_update(plan, acc, alpha, mu, sigma, static_cast<cudaStream_t>(stream)),
+                    "stats update");
+}
+
 dpb_status dpb_workspace_status(const void *workspace, int clear, int32_t *status_out, void *stream) {
     if (!workspace || !status_out) return dpb::fail(DPB_ERR_INVALID_ARG, "workspace and status_out must be non-NULL");
     cudaStream_t s = static_cast<cudaStream_t>(stream);

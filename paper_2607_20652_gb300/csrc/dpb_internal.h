@@ -102,6 +102,15 @@ cudaError_t launch_backward(const dpb_plan *p, const void *x, const int32_t *idx
                             void *grad_x, float *grad_val, int32_t *status,
                             cudaStream_t stream);
 
+// Standardisation moments (dpb_stats.cu): whether the sampled search fits
+// (kept sets of at most 64, shared memory), and the two launches.
+bool stats_supported(const dpb_plan *p, size_t *smem_out);
+cudaError_t launch_stats_accumulate(const dpb_plan *p, const void *x, int64_t T, const float *mu,
+                                    const float *sigma, const int32_t *sample, int32_t n_sample, double *acc,
+                                    int32_t *status, cudaStream_t stream);
+cudaError_t launch_stats_update(const dpb_plan *p, double *acc, float alpha, float *mu, float *sigma,
+                                cudaStream_t stream);
+
 // Dynamic shared memory (bytes) the encode kernel needs per warp / per block
 // header, used both to pick the launch shape and to reject plans that do not fit.
 size_t encode_smem_per_warp(const dpb_plan *p);

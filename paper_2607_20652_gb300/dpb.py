@@ -62,7 +62,8 @@ class Config(ctypes.Structure):
 _lib = None
 EXPORTS = ("dpb_plan_create", "dpb_plan_destroy", "dpb_plan_config", "dpb_plan_tables",
            "dpb_code_length", "dpb_workspace_size", "dpb_encode", "dpb_decode", "dpb_backward",
-           "dpb_workspace_status", "dpb_status_string", "dpb_last_error", "dpb_encode_noalloc")
+           "dpb_workspace_status", "dpb_status_string", "dpb_last_error", "dpb_encode_noalloc",
+           "dpb_stats_accumulate", "dpb_stats_update")
 
 
 def library_path() -> str:
@@ -92,6 +93,8 @@ def load(path: Optional[str] = None):
     lib.dpb_backward.argtypes = [vp, vp, vp, vp, i64, vp, vp, vp, vp, vp, sz, vp]
     lib.dpb_workspace_status.argtypes = [vp, ctypes.c_int, ctypes.POINTER(ctypes.c_int32), vp]
     lib.dpb_encode_noalloc.argtypes = [vp, vp, i64, vp, vp, vp, vp, vp, vp, vp]
+    lib.dpb_stats_accumulate.argtypes = [vp, vp, i64, vp, vp, vp, ctypes.c_int32, vp, vp, sz, vp]
+    lib.dpb_stats_update.argtypes = [vp, vp, ctypes.c_float, vp, vp, vp]
     lib.dpb_status_string.argtypes = [st]
     lib.dpb_status_string.restype = ctypes.c_char_p
     lib.dpb_last_error.argtypes = []
@@ -171,6 +174,7 @@ class Plan:
         kk = ctypes.c_int32()
         _check(lib.dpb_code_length(self._h, ctypes.byref(kk)))
         self.code_len = kk.value
+        self.n_features = 1 << self.config["bits"][self.config["levels"] - 1]  # 2^N
         self.d = d
         self.torch_dtype = _DTYPES[dtype][1]
 
@@ -258,6 +262,76 @@ def backward(plan: Plan, x: torch.Tensor, idx: torch.Tensor, val: torch.Tensor, 
                                   _ptr(grad_y), _ptr(grad_x), _ptr(grad_val), _ptr(ws),
                                   ws.numel() * ws.element_size(), _stream(stream)))
     return grad_x, grad_val
+
+
+def stats_buffer(plan: Plan, device=None) -> torch.Tensor:
+    """A zeroed moment-sum buffer fp64 [3, 2^N] (count, sum s, sum s^2)."""
+    return torch.zeros((3, plan.n_features), dtype=torch.float64, device=device or "cuda")
+
+
+def stats_accumulate(plan: Plan, x: torch.Tensor, sample: torch.Tensor, acc: torch.Tensor, mu=None,
+                     sigma=None, workspace=None, stream=None):
+    """dpb_stats_accumulate: adds the batch's moment sums to ``acc`` (level 0
+    over every row of x, levels >= 1 over the rows in ``sample``)."""
+    _rows(x, plan, "x")
+    if sample.dtype != torch.int32 or not sample.is_contiguous() or sample.dim() != 1:
+        raise ValueError("sample must be a contiguous 1-D int32 tensor of row numbers")
+    if acc.dtype != torch.float64 or not acc.is_contiguous() or acc.numel() != 3 * plan.n_features:
+        raise ValueError("acc must be a contiguous float64 tensor of 3 * 2^N entries (stats_buffer)")
+    T = x.shape[0]
+    ws = plan.workspace(T, x.device) if workspace is None else workspace
+    _check(plan._lib.dpb_stats_accumulate(plan.handle, _ptr(x), T, _ptr(mu), _ptr(sigma),
+                                          _ptr(sample) if sample.numel() else None, sample.numel(),
+                                          _ptr(acc), _ptr(ws), ws.numel() * ws.element_size(),
+                                          _stream(stream)))
+    return acc
+
+
+def stats_update(plan: Plan, acc: torch.Tensor, alpha: float, mu: torch.Tensor, sigma: torch.Tensor,
+                 stream=None):
+    """dpb_stats_update: one EMA step of (mu, sigma) in place; zeroes ``acc``."""
+    if acc.dtype != torch.float64 or not acc.is_contiguous():
+        raise ValueError("acc must be a contiguous float64 tensor")
+    for name, t in (("mu", mu), ("sigma", sigma)):
+        if t.dtype != torch.float32 or not t.is_contiguous() or t.numel() * 3 != acc.numel():
+            raise ValueError(f"{name} must be a contiguous float32 tensor of 2^N entries")
+    _check(plan._lib.dpb_stats_update(plan.handle, _ptr(acc), float(alpha), _ptr(mu), _ptr(sigma),
+                                      _stream(stream)))
+    return mu, sigma
+
+
+def ema_step(accumulate, update, acc, group=None):
+    """One standardisation step under data parallelism: each rank adds its
+    own moment sums (``accumulate(acc)``), the sums are added up across the
+    ranks of ``group`` (one all-reduce; skipped when torch.distributed is not
+    initialised or the group has one rank), and every rank makes the same EMA
+    step (``update(acc)``), so the tables stay identical everywhere."""
+    accumulate(acc)
+    import torch.distributed as dist
+    if dist.is_available() and dist.is_initialized() and dist.get_world_size(group) > 1:
+        dist.all_reduce(acc, op=dist.ReduceOp.SUM, group=group)
+    update(acc)
+
+
+def sample_rows(T: int, n: int, generator: Optional[torch.Generator] = None, device=None) -> torch.Tensor:
+    """n distinct row numbers of [0, T) (all of them when T <= n), drawn
+    uniformly by ``generator``: the sub-sample of levels >= 1."""
+    n = min(n, T)
+    rows = torch.randperm(T, generator=generator)[:n].to(torch.int32)
+    return rows.to(device) if device is not None else rows
+
+
+def stats_step(plan: Plan, x: torch.Tensor, mu: torch.Tensor, sigma: torch.Tensor, alpha: float,
+               sample: torch.Tensor, acc: Optional[torch.Tensor] = None, workspace=None, stream=None,
+               group=None):
+    """The whole EMA update of one batch (§2.2 "Score Standardization"):
+    moment sums on this rank, summed across ``group``, then the EMA step of
+    mu and sigma in place."""
+    acc = stats_buffer(plan, x.device) if acc is None else acc
+    ema_step(lambda a: stats_accumulate(plan, x, sample, a, mu=mu, sigma=sigma, workspace=workspace,
+                                        stream=stream),
+             lambda a: stats_update(plan, a, alpha, mu, sigma, stream=stream), acc, group)
+    return mu, sigma
 
 
 def workspace_status(workspace: torch.Tensor, clear: bool = False, stream=None) -> int:

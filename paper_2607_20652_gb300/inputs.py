@@ -56,6 +56,20 @@ def normal(shape, seed: int, scale: float = 1.0) -> np.ndarray:
     return (rng(seed).standard_normal(shape, dtype=np.float32) * np.float32(scale))
 
 
+def sample_rows(T: int, n: int, seed: int) -> np.ndarray:
+    """min(n, T) distinct row numbers of [0, T), drawn uniformly (int32)."""
+    return rng(seed).permutation(T)[: min(n, T)].astype(np.int32)
+
+
+def moment_tables(m: int, seed: int, mean_scale: float = 0.2, sigma_range=(0.5, 2.0)):
+    """Standardisation tables (mu, sigma) fp32 [m]: mu ~ N(0, mean_scale^2),
+    sigma uniform in sigma_range."""
+    g = rng(seed)
+    mu = (g.standard_normal(m) * mean_scale).astype(np.float32)
+    sigma = g.uniform(sigma_range[0], sigma_range[1], m).astype(np.float32)
+    return mu, sigma
+
+
 @dataclasses.dataclass
 class PlantedTree:
     """Random choices of a planted hierarchical code, per token.

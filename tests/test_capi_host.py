@@ -130,3 +130,31 @@ def test_per_level_code_length(lib):
                     select_mode=dpb.SELECT_PER_LEVEL, k_per_level=[16, 32, 64])
     assert plan.code_len == 112
     assert plan.config["select_mode"] == dpb.SELECT_PER_LEVEL
+
+
+def test_stats_arguments_are_checked(lib):
+    # Host-side validation of the moment calls runs before any device work, so
+    # a plan without a device still reports each bad argument (the pointers
+    # below are never dereferenced).
+    INVALID, CUDA = 1, 3
+    plan = dpb.Plan(d=64, levels=3, m_bits=12, children=16, beam=4, k=8, dtype="f32")
+    P = ctypes.c_void_p
+    buf, odd = P(0x10000), P(0x10004)
+    acc = lib.dpb_stats_accumulate
+    # mu without sigma
+    assert acc(plan.handle, buf, 4, buf, None, buf, 1, buf, buf, 256, None) == INVALID
+    # negative sample count, sampled rows of an empty batch, misaligned acc
+    assert acc(plan.handle, buf, 4, None, None, buf, -1, buf, buf, 256, None) == INVALID
+    assert acc(plan.handle, buf, 0, None, None, buf, 1, buf, buf, 256, None) == INVALID
+    assert acc(plan.handle, buf, 4, None, None, buf, 1, odd, buf, 256, None) == INVALID
+    assert acc(plan.handle, buf, 0, None, None, None, 0, buf, buf, 256, None) == 0   # empty batch
+    up = lib.dpb_stats_update
+    for alpha in (0.0, 1.0, -0.5, float("nan")):
+        assert up(plan.handle, buf, alpha, buf, buf, None) == INVALID
+    assert up(plan.handle, odd, 0.5, buf, buf, None) == INVALID
+    assert up(plan.handle, buf, 0.5, None, buf, None) == INVALID
+    # the largest kept sets (32 parents of 256 children each) still fit the sampled
+    # search: valid arguments reach the device check
+    big = dpb.Plan(d=1024, levels=2, bits=[10, 17], children=[0, 256], dtype="bf16",
+                   select_mode=dpb.SELECT_PER_LEVEL, k_per_level=[32, 64])
+    assert acc(big.handle, buf, 4, None, None, buf, 1, buf, buf, 256, None) == CUDA
