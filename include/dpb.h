@@ -145,9 +145,13 @@ dpb_status dpb_plan_tables(const dpb_plan *plan, uint32_t *M_out, uint32_t *G_ou
 /* Code length per token: k (global mode) or sum_l k_per_level[l]. */
 dpb_status dpb_code_length(const dpb_plan *plan, int32_t *k_out);
 
-/* Bytes of workspace the calls need for T tokens (at least 256; 256-byte
- * aligned pointer required). The workspace holds the device status word; it
- * must be zero-filled once before its first use, and may be reused by every
+/* Bytes of workspace for T tokens (256-byte aligned pointer required): 256
+ * bytes for the device status word, then 8 * 2^N bytes (for 2^N <= 2^26)
+ * where dpb_encode packs the standardisation tables as (mu, 1 / sigma) pairs,
+ * so that each candidate costs one table load instead of two. Any workspace of
+ * at least 256 bytes is accepted; a smaller one than this size only leaves the
+ * tables unpacked (same results, slower with tables). The status word must be
+ * zero-filled once before its first use; the workspace may be reused by every
  * call on the same stream. Calls that run concurrently need separate
  * workspaces. */
 dpb_status dpb_workspace_size(const dpb_plan *plan, int64_t T, size_t *bytes);

@@ -162,7 +162,7 @@ dpb_status dpb_code_length(const dpb_plan *plan, int32_t *k_out) {
 dpb_status dpb_workspace_size(const dpb_plan *plan, int64_t T, size_t *bytes) {
     DPB_TRY(check_plan(plan));
     if (!bytes || T < 0) return dpb::fail(DPB_ERR_INVALID_ARG, "bytes is NULL or T < 0");
-    *bytes = 256;
+    *bytes = dpb::kStatusBytes + dpb::tab_bytes(plan);
     return DPB_OK;
 }
 
@@ -182,8 +182,12 @@ dpb_status dpb_encode(const dpb_plan *plan, const void *x, int64_t T, const floa
     DPB_TRY(check_vec(xnorm, "xnorm", false));
     DPB_TRY(check_workspace(workspace, workspace_bytes));
     DPB_TRY(check_device(plan));
+    const size_t tb = dpb::tab_bytes(plan);
+    float2 *tab = tb > 0 && workspace_bytes >= dpb::kStatusBytes + tb
+                      ? reinterpret_cast<float2 *>(static_cast<char *>(workspace) + dpb::kStatusBytes)
+                      : nullptr;
     return launched(dpb::launch_encode(plan, x, T, mu, sigma, idx, val, xnorm,
-                                       static_cast<int32_t *>(workspace),
+                                       static_cast<int32_t *>(workspace), tab,
                                        static_cast<cudaStream_t>(stream)),
                     "encode");
 }

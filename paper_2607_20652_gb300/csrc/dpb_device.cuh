@@ -7,6 +7,8 @@
 
 #include <cstdint>
 
+#include "../../include/dpb.h"
+
 namespace dpb {
 
 constexpr unsigned kFull = 0xffffffffu;
@@ -257,6 +259,28 @@ __device__ __forceinline__ void warp_sort(float *z, uint32_t *id, int n, int cap
 
 __device__ __forceinline__ void set_status(int32_t *status, int32_t bit) {
     if (status) atomicOr(status, bit);
+}
+
+// ---- score standardisation (§2.2 "Score Standardization") -------------------------
+
+// z = (s - mu_c) / sigma_c, computed as (s - mu_c) * r_c with r_c = 1 / sigma_c
+// rounded to fp32, so that every path gives the same z for the same s. `tab`
+// (nullable) holds the pairs (mu_c, r_c): one 8-byte load instead of one from
+// each table. A sigma that is not a positive finite number (r_c outside
+// (0, inf)) sets DPB_DEV_BAD_SIGMA when `status` is given.
+__device__ __forceinline__ float zscore(float s, uint32_t c, const float *mu, const float *sigma,
+                                        const float2 *tab, int32_t *status) {
+    float m, r;
+    if (tab) {
+        const float2 p = tab[c];
+        m = p.x;
+        r = p.y;
+    } else {
+        m = mu[c];
+        r = __frcp_rn(sigma[c]);
+    }
+    if (status && !(r > 0.f && r <= 3.402823466e38f)) set_status(status, DPB_DEV_BAD_SIGMA);
+    return (s - m) * r;
 }
 
 }  // namespace dpb

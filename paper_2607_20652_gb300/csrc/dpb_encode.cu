@@ -28,12 +28,19 @@ struct EncodeArgs {
     float inv_sqrt_d;
 };
 
-__device__ __forceinline__ float standardise(float s, uint32_t i, const float *mu,
-                                             const float *sigma, int32_t *status) {
-    if (!mu) return s;
-    const float sd = sigma[i];
+// (mu_c, 1 / sigma_c) for every feature, read by the encoders in one 8-byte load.
+__global__ void pack_tables_kernel(const float *mu, const float *sigma, float2 *tab, int64_t m) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < m; i += (int64_t)gridDim.x * blockDim.x)
+        tab[i] = make_float2(mu[i], __frcp_rn(sigma[i]));
+}
+
+// z = (s - mu_c) / sigma_c (this general encoder scores in its own order, so
+// its last bits need not match the tensor-core encoders' in any case)
+__device__ __forceinline__ float standardise(float s, uint32_t c, const EncodeArgs &a, int32_t *status) {
+    if (!a.mu) return s;
+    const float sd = a.sigma[c];
     if (!(sd > 0.f)) set_status(status, DPB_DEV_BAD_SIGMA);
-    return (s - mu[i]) / sd;
+    return (s - a.mu[c]) / sd;
 }
 
 // Per-warp shared-memory carve-up (floats and words are both 4 bytes).
@@ -87,7 +94,7 @@ __global__ void __launch_bounds__(128) encode_warp_kernel(EncodeArgs a) {
 
         // ---- level 0: every coordinate is a candidate ----
         for (int i = lane; i < d; i += 32) {
-            w.lz[i] = standardise(w.xs[i], (uint32_t)i, a.mu, a.sigma, a.status);
+            w.lz[i] = standardise(w.xs[i], (uint32_t)i, a, a.status);
             w.lid[i] = (uint32_t)i;
         }
         __syncwarp();
@@ -137,7 +144,7 @@ __global__ void __launch_bounds__(128) encode_warp_kernel(EncodeArgs a) {
                     keep = true;
                     for (int r = 0; r < s; ++r)
                         if (w.lid[r] == c) keep = false;
-                    z = standardise(w.lz[s], c, a.mu, a.sigma, a.status);
+                    z = standardise(w.lz[s], c, a, a.status);
                 }
                 const unsigned m = __ballot_sync(kFull, keep);
                 if (keep) {
@@ -212,13 +219,25 @@ size_t encode_smem_per_warp(const dpb_plan *p) {
 
 cudaError_t launch_encode(const dpb_plan *p, const void *x, int64_t T, const float *mu,
                           const float *sigma, int32_t *idx, float *val, float *xnorm,
-                          int32_t *status, cudaStream_t stream) {
+                          int32_t *status, float2 *tab_scratch, cudaStream_t stream) {
+    // standardisation tables as (mu, 1 / sigma) pairs: one load per candidate
+    const float2 *tab = nullptr;
+    if (mu && tab_scratch) {
+        const int64_t m = (int64_t)p->m_mask + 1;
+        int sms = 0;
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, p->device);
+        const int64_t want = (m + 255) / 256, cap = (int64_t)sms * 8;
+        pack_tables_kernel<<<(unsigned)(want < cap ? want : cap), 256, 0, stream>>>(mu, sigma, tab_scratch, m);
+        const cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+        tab = tab_scratch;
+    }
     // the paper's per-level selection: tcgen05 scoring
     if (p->cfg.select_mode == DPB_SELECT_PER_LEVEL)
-        return launch_encode_pl(p, x, T, mu, sigma, idx, val, xnorm, status, stream);
+        return launch_encode_pl(p, x, T, mu, sigma, tab, idx, val, xnorm, status, stream);
     // bf16 rows on 16-byte boundaries, beam 8, 16 children: tensor-core scoring
     if (p->mma_encode && (reinterpret_cast<uintptr_t>(x) & 15u) == 0)
-        return launch_encode_mma(p, x, T, mu, sigma, idx, val, xnorm, status, stream);
+        return launch_encode_mma(p, x, T, mu, sigma, tab, idx, val, xnorm, status, stream);
     const dpb_config &c = p->cfg;
     EncodeArgs a{};
     a.x = x;

@@ -19,7 +19,7 @@ int encode_mma_warps(const dpb_plan *p) {
 }
 
 cudaError_t launch_encode_mma(const dpb_plan *p, const void *x, int64_t T, const float *mu,
-                              const float *sigma, int32_t *idx, float *val, float *xnorm,
+                              const float *sigma, const float2 *tab, int32_t *idx, float *val, float *xnorm,
                               int32_t *status, cudaStream_t stream) {
     const dpb_config &c = p->cfg;
     mmaenc::Args a{};
@@ -27,6 +27,7 @@ cudaError_t launch_encode_mma(const dpb_plan *p, const void *x, int64_t T, const
     a.T = T;
     a.mu = mu;
     a.sigma = sigma;
+    a.tab = tab;
     a.idx = idx;
     a.val = val;
     a.xnorm = xnorm;

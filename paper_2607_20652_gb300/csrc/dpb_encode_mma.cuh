@@ -50,6 +50,7 @@ struct Args {
     const __nv_bfloat16 *x;
     int64_t T;
     const float *mu, *sigma;
+    const float2 *tab;  // packed (mu, 1 / sigma), nullable
     int32_t *idx;
     float *val, *xnorm;
     int32_t *status;
@@ -152,12 +153,8 @@ __device__ __forceinline__ float x_at(const uint16_t *xh, int i) {
 }
 
 // z = (s - mu_c) / sigma_c (§2.2 score standardisation); identity without tables.
-__device__ __forceinline__ float standardise(float s, uint32_t c, const float *mu, const float *sigma,
-                                             int32_t *status) {
-    if (!mu) return s;
-    const float sd = sigma[c];
-    if (status && !(sd > 0.f)) set_status(status, DPB_DEV_BAD_SIGMA);
-    return (s - mu[c]) / sd;
+__device__ __forceinline__ float standardise(float s, uint32_t c, const Args &a, int32_t *status) {
+    return a.mu ? zscore(s, c, a.mu, a.sigma, a.tab, status) : s;
 }
 
 // bf16 element e (0..7) of a 16-byte chunk.
@@ -182,16 +179,21 @@ __device__ __forceinline__ int warp_append(float *z, uint32_t *id, int n, bool t
 
 // One compare-exchange stage (size, stride) of a warp bitonic sort,
 // descending, of 32 R words held R per lane (element lane * R + r).
-template <int R>
-__device__ __forceinline__ void sort_stage(uint32_t (&v)[R], int size, int stride) {
+__device__ __forceinline__ uint32_t whi(uint32_t a, uint32_t b) { return max(a, b); }
+__device__ __forceinline__ uint32_t wlo(uint32_t a, uint32_t b) { return min(a, b); }
+__device__ __forceinline__ uint64_t whi(uint64_t a, uint64_t b) { return a > b ? a : b; }
+__device__ __forceinline__ uint64_t wlo(uint64_t a, uint64_t b) { return a > b ? b : a; }
+
+template <int R, typename W>
+__device__ __forceinline__ void sort_stage(W (&v)[R], int size, int stride) {
     const int lane = threadIdx.x & 31;
     if (stride >= R) {
         const bool lower = (lane & (stride / R)) == 0;
 #pragma unroll
         for (int r = 0; r < R; ++r) {
             const bool desc = (((lane * R + r) & size) == 0);
-            const uint32_t o = __shfl_xor_sync(kFull, v[r], stride / R);
-            v[r] = (lower == desc) ? max(v[r], o) : min(v[r], o);
+            const W o = __shfl_xor_sync(kFull, v[r], stride / R);
+            v[r] = (lower == desc) ? whi(v[r], o) : wlo(v[r], o);
         }
     } else {
 #pragma unroll
@@ -202,7 +204,7 @@ __device__ __forceinline__ void sort_stage(uint32_t (&v)[R], int size, int strid
                     const int q = r ^ cs;
                     if (q > r) {
                         const bool desc = (((lane * R + r) & size) == 0);
-                        const uint32_t hi = max(v[r], v[q]), lo = min(v[r], v[q]);
+                        const W hi = whi(v[r], v[q]), lo = wlo(v[r], v[q]);
                         v[r] = desc ? hi : lo;
                         v[q] = desc ? lo : hi;
                     }
@@ -214,12 +216,12 @@ __device__ __forceinline__ void sort_stage(uint32_t (&v)[R], int size, int strid
 
 // Warp bitonic sort, descending. The stages are looped, not unrolled: the
 // encoder's other phases already fill the instruction caches.
-template <int R>
-__device__ __forceinline__ void warp_sort_desc(uint32_t (&v)[R]) {
+template <int R, typename W>
+__device__ __forceinline__ void warp_sort_desc(W (&v)[R]) {
 #pragma unroll 1
     for (int size = 2; size <= 32 * R; size <<= 1)
 #pragma unroll 1
-        for (int stride = size / 2; stride > 0; stride >>= 1) sort_stage<R>(v, size, stride);
+        for (int stride = size / 2; stride > 0; stride >>= 1) sort_stage<R, W>(v, size, stride);
 }
 
 __device__ __forceinline__ void cas_desc(uint64_t &a, uint64_t &b) {
@@ -402,22 +404,91 @@ __device__ __forceinline__ bool level0_union(const uint4 *row, int nch, int k, u
     return true;
 }
 
+// Level 0 with standardisation tables: the union path above on 64-bit words
+// of z = (x_i - mu_i) / sigma_i (a standardised score does not fit the 16-bit
+// key of a bf16 coordinate). Each lane keeps its R best words; the k-th of the
+// union is the threshold, and the few words at or above it that a lane did not
+// keep are merged in. Returns false (nothing written) when they overflow E.
+template <int R, int KPL>
+__device__ __forceinline__ bool level0_union_std(const Args &a, const uint16_t *xh, int k, uint64_t *E, int ecap,
+                                                 uint64_t *L, uint32_t *beam) {
+    const int lane = threadIdx.x & 31, d = a.d;
+    uint64_t top[R];
+#pragma unroll
+    for (int r = 0; r < R; ++r) top[r] = 0ull;
+#pragma unroll 1
+    for (int i = lane; i < d; i += 32) {
+        uint64_t c = cword(standardise(x_at(xh, i), (uint32_t)i, a, a.status), (uint32_t)i);
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+            const uint64_t hi = whi(top[r], c);
+            c = wlo(top[r], c);
+            top[r] = hi;
+        }
+    }
+    const uint64_t kept_min = top[R - 1];  // every word of this lane below it was not kept
+    warp_sort_desc<R>(top);
+    uint64_t mine = 0ull;
+#pragma unroll
+    for (int r = 0; r < R; ++r)
+        if (r == (k - 1) % R) mine = top[r];
+    const uint64_t tau = __shfl_sync(kFull, mine, (k - 1) / R);
+    int nx = 0;
+#pragma unroll 1
+    for (int i = lane; i < d; i += 32) {
+        const uint64_t w = cword(standardise(x_at(xh, i), (uint32_t)i, a, nullptr), (uint32_t)i);
+        nx += (w >= tau) & (w < kept_min);
+    }
+    const int total = __reduce_add_sync(kFull, nx);
+    if (total > ecap) return false;
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+        const int e = lane * R + r;
+        if (e < k) L[e] = top[r];
+    }
+    if (total > 0) {
+        int off = nx;  // exclusive prefix of the extras over the lanes
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int v = __shfl_up_sync(kFull, off, o);
+            if (lane >= o) off += v;
+        }
+        off -= nx;
+#pragma unroll 1
+        for (int i = lane; i < d; i += 32) {
+            const uint64_t w = cword(standardise(x_at(xh, i), (uint32_t)i, a, nullptr), (uint32_t)i);
+            if (w >= tau && w < kept_min) E[off++] = w;
+        }
+        __syncwarp();
+        merge_sorted<KPL>(L, k, E, total, nullptr);
+        if (lane < kBeam) beam[lane] = cword_idx(L[lane]);
+    } else {
+#pragma unroll
+        for (int r = 0; r < R; ++r)
+            if (lane * R + r < kBeam) beam[lane * R + r] = cword_idx(top[r]);
+    }
+    __syncwarp();
+    return true;
+}
+
 // General path: every coordinate (standardised if tables are given) is a
-// candidate; a per-lane threshold keeps at least k of them in the scratch
-// (z, id) lists of capacity `cap`, the k-th is found by bisection, and the
-// first k, sorted, become the code list; its first 8 are the beam.
+// candidate; a threshold that at least k of them reach keeps them in the
+// scratch (z, id) lists of capacity `cap`, the k-th is found by bisection, and
+// the first k, sorted, become the code list; its first 8 are the beam.
 __device__ __forceinline__ void level0_bisect(const Args &a, const uint16_t *xh, float *pz, uint32_t *pid, int cap,
                                               uint64_t *L, uint32_t *beam) {
     const int lane = threadIdx.x & 31, d = a.d, k = a.k;
     const int lowbit = a.mu ? 0 : 16;  // keys of unstandardised bf16 values have 16 zero bits
-    // Each lane's R-th best key: at least 32 R >= k candidates are at or above
-    // the smallest of them.
-    const int R = (k + 31) >> 5;
+    // Each lane's R best keys, R = 2 ceil(k / 32) (at most 8): their union
+    // holds at least k keys, and its k-th largest is a threshold that at least
+    // k candidates reach and, unlike the smallest of the lanes' R-th keys,
+    // only a few more.
+    const int R = min(8, 2 * ((k + 31) >> 5));
     uint32_t best[8];
 #pragma unroll
     for (int r = 0; r < 8; ++r) best[r] = 0u;
     for (int i = lane; i < d; i += 32) {
-        uint32_t kv = akey(standardise(x_at(xh, i), (uint32_t)i, a.mu, a.sigma, a.status)) + 1u;
+        uint32_t kv = akey(standardise(x_at(xh, i), (uint32_t)i, a, a.status)) + 1u;
 #pragma unroll
         for (int r = 0; r < 8; ++r) {
             if (r < R && kv > best[r]) {
@@ -427,11 +498,14 @@ __device__ __forceinline__ void level0_bisect(const Args &a, const uint16_t *xh,
             }
         }
     }
-    uint32_t mine = 0;
+    uint32_t tau_low = 0;  // the union's k-th largest key, bit by bit
+    for (int b = 31; b >= 0; --b) {
+        const uint32_t c = tau_low | (1u << b);
+        int cnt = 0;
 #pragma unroll
-    for (int r = 0; r < 8; ++r)
-        if (r == R - 1) mine = best[r];
-    const uint32_t tau_low = __reduce_min_sync(kFull, mine);
+        for (int r = 0; r < 8; ++r) cnt += r < R && best[r] >= c;
+        if ((int)__reduce_add_sync(kFull, (uint32_t)cnt) >= k) tau_low = c;
+    }
     int n = 0;
     bool overflow = false;
     for (int i0 = 0; i0 < d && !overflow; i0 += 32) {
@@ -439,7 +513,7 @@ __device__ __forceinline__ void level0_bisect(const Args &a, const uint16_t *xh,
         float z = 0.f;
         bool take = false;
         if (i < d) {
-            z = standardise(x_at(xh, i), (uint32_t)i, a.mu, a.sigma, nullptr);
+            z = standardise(x_at(xh, i), (uint32_t)i, a, nullptr);
             take = akey(z) + 1u >= tau_low;
         }
         if (n + __popc(__ballot_sync(kFull, take)) > cap) {
@@ -457,14 +531,14 @@ __device__ __forceinline__ void level0_bisect(const Args &a, const uint16_t *xh,
             const uint32_t c = tau | (1u << b);
             int cnt = 0;
             for (int i = lane; i < d; i += 32)
-                cnt += akey(standardise(x_at(xh, i), (uint32_t)i, a.mu, a.sigma, nullptr)) >= c;
+                cnt += akey(standardise(x_at(xh, i), (uint32_t)i, a, nullptr)) >= c;
             if (__reduce_add_sync(kFull, cnt) >= k) tau = c;
         }
         n = 0;
         for (int i0 = 0; i0 < d; i0 += 32) {
             const int i = i0 + lane;
             float z = 0.f;
-            if (i < d) z = standardise(x_at(xh, i), (uint32_t)i, a.mu, a.sigma, nullptr);
+            if (i < d) z = standardise(x_at(xh, i), (uint32_t)i, a, nullptr);
             n = warp_append(pz, pid, n, i < d && akey(z) > tau, z, (uint32_t)i);
         }
         for (int i0 = 0; i0 < d && n < k; i0 += 32) {
@@ -472,7 +546,7 @@ __device__ __forceinline__ void level0_bisect(const Args &a, const uint16_t *xh,
             float z = 0.f;
             bool tie = false;
             if (i < d) {
-                z = standardise(x_at(xh, i), (uint32_t)i, a.mu, a.sigma, nullptr);
+                z = standardise(x_at(xh, i), (uint32_t)i, a, nullptr);
                 tie = akey(z) == tau;
             }
             const unsigned mb = __ballot_sync(kFull, tie);
@@ -566,7 +640,9 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
             uint32_t *bt = beams + tk * kBeam;
             bool done = false;
             // each lane keeps R words, so the union of 32 R holds at least 2 k
-            if (!a.mu && KPL <= 4) done = level0_union<(KPL <= 2 ? 4 : 8), KPL>(row, nch, k, E, a.ecap, Lt, bt);
+            if (KPL <= 4)
+                done = a.mu ? level0_union_std<(KPL <= 2 ? 4 : 8), KPL>(a, xh + tk * nblk * 32, k, E, a.ecap, Lt, bt)
+                            : level0_union<(KPL <= 2 ? 4 : 8), KPL>(row, nch, k, E, a.ecap, Lt, bt);
             if (!done)
                 level0_bisect(a, xh + tk * nblk * 32, reinterpret_cast<float *>(E),
                               reinterpret_cast<uint32_t *>(E) + a.ecap, a.ecap, Lt, bt);
@@ -686,7 +762,7 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
                     const uint32_t ci = pcur ^ gl[8 * (e >> 1) + 2 * q4 + (e & 1)];
-                    const float z = standardise(sc[0][e], ci, a.mu, a.sigma, a.status);
+                    const float z = standardise(sc[0][e], ci, a, a.status);
                     c[e] = ((dmask >> e) & 1u) ? 0ull : cword(z, ci);
                     sc[0][e] = sc[1][e];
                 }

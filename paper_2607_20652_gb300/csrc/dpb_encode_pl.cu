@@ -57,6 +57,7 @@ struct Args {
     const __nv_bfloat16 *x;
     int64_t T;
     const float *mu, *sigma;
+    const float2 *tab;  // packed (mu, 1 / sigma), nullable
     int32_t *idx;
     float *val, *xnorm;
     int32_t *status;
@@ -139,6 +140,20 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
           "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
         : "r"(taddr));
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Stores 32 consecutive 32-bit columns of this warp's 32 TMEM lanes (one
+// lane per thread) and waits for the stores.
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&v)[32]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,"
+        "%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+        "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]),
+        "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]), "r"(v[16]),
+        "r"(v[17]), "r"(v[18]), "r"(v[19]), "r"(v[20]), "r"(v[21]), "r"(v[22]), "r"(v[23]), "r"(v[24]),
+        "r"(v[25]), "r"(v[26]), "r"(v[27]), "r"(v[28]), "r"(v[29]), "r"(v[30]), "r"(v[31])
+        : "memory");
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 
 // ---- selection ---------------------------------------------------------------------
@@ -343,12 +358,8 @@ __device__ __forceinline__ int select_level(Scan scan, int nlive, int K, const W
     return distinct;
 }
 
-__device__ __forceinline__ float standardise(float s, uint32_t c, const float *mu, const float *sigma,
-                                             int32_t *status) {
-    if (!mu) return s;
-    const float sd = sigma[c];
-    if (status && !(sd > 0.f)) set_status(status, DPB_DEV_BAD_SIGMA);
-    return (s - mu[c]) / sd;
+__device__ __forceinline__ float standardise(float s, uint32_t c, const Args &a, int32_t *status) {
+    return a.mu ? zscore(s, c, a.mu, a.sigma, a.tab, status) : s;
 }
 
 // ---- the kernel ----------------------------------------------------------------------
@@ -431,11 +442,11 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
                 for (int i = lane; i < d; i += 32) {
                     const int m = i >> 5, wl = i & 31;
                     const float xv = __uint_as_float((uint32_t)xh[(m * 16 + (wl & 15)) * 2 + (wl >> 4)] << 16);
-                    f(standardise(xv, (uint32_t)i, a.mu, a.sigma, nullptr), (uint32_t)i, true);
+                    f(standardise(xv, (uint32_t)i, a, nullptr), (uint32_t)i, true);
                 }
             };
             if (a.mu)
-                for (int i = lane; i < d; i += 32) standardise(0.f, (uint32_t)i, a.mu, a.sigma, a.status);
+                for (int i = lane; i < d; i += 32) standardise(0.f, (uint32_t)i, a, a.status);
             select_level(scan0, min(32, d / 32 * 32), a.kl[0], wb, a, tok, a.off[0], L > 1);
         } else {
             wb.par[lane] = 0u;
@@ -556,6 +567,37 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
                 }
             }
             asm volatile("tcgen05.fence::after_thread_sync;");
+            const uint32_t *gl = gs + l * 256;
+            // ---- standardised scores, once per candidate (§2.2): z replaces s in
+            // TMEM, so the selection's three passes gather no tables. Warp w
+            // takes quarter w % 4 (all 32 rows; with 16 slots a quarter holds
+            // tokens q and q + 4) of tile w / 4, or with one tile half w / 4 of
+            // the columns: all eight warps keep table loads in flight.
+            if (a.mu) {
+                {
+                    const int q = warp & 3, tile = ntiles == 2 ? warp >> 2 : 0;
+                    const int half = ((D + 31) / 32 + 1) / 2 * 32;  // whole 32-column loads
+                    const int cb = ntiles == 2 ? 0 : (warp >> 2) * half, ce = ntiles == 2 ? D : min(D, cb + half);
+                    const int tokw = pp == 32 ? q + 4 * tile : q + 4 * (lane >> 4);
+                    const int slot = pp == 32 ? lane : lane & 15;
+                    const bool ok = grp * kTokens + tokw < a.T && slot < P;
+                    const uint32_t p = ok ? reinterpret_cast<const uint32_t *>(smem + lay.par)[tokw * kRows + slot] : 0u;
+                    const uint32_t taddr = tmem + ((uint32_t)(32 * q) << 16) + 256u * tile;
+                    for (int c0 = cb; c0 < ce; c0 += 32) {
+                        uint32_t v[32];
+                        tmem_ld32(taddr + c0, v);
+#pragma unroll
+                        for (int j = 0; j < 32; ++j)
+                            if (ok && c0 + j < D)
+                                v[j] = __float_as_uint(standardise(__uint_as_float(v[j]) * a.inv_sqrt_d, p ^ gl[c0 + j], a,
+                                                                   a.status));
+                        tmem_st32(taddr + c0, v);
+                    }
+                }
+                asm volatile("tcgen05.fence::before_thread_sync;");
+                __syncthreads();
+                asm volatile("tcgen05.fence::after_thread_sync;");
+            }
             // ---- the level's selection, one warp per token ----
             if (live) {
                 // this warp's rows: tile (warp / 4 when 32 slots), quarter warp % 4,
@@ -565,7 +607,7 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
                 const int slot = lane - base;
                 const bool rv = slot >= 0 && slot < pp && slot < P;
                 const uint32_t p = rv ? wb.par[slot] : 0u;
-                const uint32_t *gl = gs + l * 256;
+                const float scale = a.mu ? 1.f : a.inv_sqrt_d;  // TMEM holds z, or s sqrt(d)
                 auto scanl = [&](auto f) {
                     for (int c0 = 0; c0 < D; c0 += 32) {
                         uint32_t v[32];
@@ -573,8 +615,7 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
 #pragma unroll
                         for (int j = 0; j < 32; ++j) {
                             const uint32_t ci = p ^ gl[c0 + j];
-                            f(standardise(__uint_as_float(v[j]) * a.inv_sqrt_d, ci, a.mu, a.sigma, nullptr), ci,
-                              rv && c0 + j < D);
+                            f(__uint_as_float(v[j]) * scale, ci, rv && c0 + j < D);
                         }
                     }
                 };
@@ -672,13 +713,15 @@ size_t encode_pl_smem(const dpb_plan *p) {
 }
 
 cudaError_t launch_encode_pl(const dpb_plan *p, const void *x, int64_t T, const float *mu, const float *sigma,
-                             int32_t *idx, float *val, float *xnorm, int32_t *status, cudaStream_t stream) {
+                             const float2 *tab, int32_t *idx, float *val, float *xnorm, int32_t *status,
+                             cudaStream_t stream) {
     const dpb_config &c = p->cfg;
     Args a{};
     a.x = static_cast<const __nv_bfloat16 *>(x);
     a.T = T;
     a.mu = mu;
     a.sigma = sigma;
+    a.tab = tab;
     a.idx = idx;
     a.val = val;
     a.xnorm = xnorm;

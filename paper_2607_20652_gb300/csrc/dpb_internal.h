@@ -74,7 +74,8 @@ dpb_status check_per_level(const dpb_config &c);
 void build_per_level_tables(dpb_plan *p);
 size_t encode_pl_smem(const dpb_plan *p);
 cudaError_t launch_encode_pl(const dpb_plan *p, const void *x, int64_t T, const float *mu, const float *sigma,
-                             int32_t *idx, float *val, float *xnorm, int32_t *status, cudaStream_t stream);
+                             const float2 *tab, int32_t *idx, float *val, float *xnorm, int32_t *status,
+                             cudaStream_t stream);
 
 // Launch shape of the tensor-core encoder: the most warps per block (16, 12,
 // 8 or 4) whose shared memory fits, or 0 if none does; and that memory.
@@ -90,11 +91,22 @@ dpb_status resolve_and_build(const dpb_config *in, const uint32_t *generators, d
 
 // Kernel launchers (return cudaGetLastError() of the launch).
 cudaError_t launch_encode_mma(const dpb_plan *p, const void *x, int64_t T, const float *mu,
-                              const float *sigma, int32_t *idx, float *val, float *xnorm,
+                              const float *sigma, const float2 *tab, int32_t *idx, float *val, float *xnorm,
                               int32_t *status, cudaStream_t stream);
+// tab_scratch (nullable, tab_bytes(p) bytes): where the standardisation tables
+// are packed as (mu, 1 / sigma) pairs before the encoder runs.
 cudaError_t launch_encode(const dpb_plan *p, const void *x, int64_t T, const float *mu,
                           const float *sigma, int32_t *idx, float *val, float *xnorm,
-                          int32_t *status, cudaStream_t stream);
+                          int32_t *status, float2 *tab_scratch, cudaStream_t stream);
+
+// Workspace: the status word (kStatusBytes, required) and, after it, the
+// optional packed standardisation tables (8 bytes per feature, for 2^N up to
+// 2^26; 0 bytes beyond).
+constexpr size_t kStatusBytes = 256;
+inline size_t tab_bytes(const dpb_plan *p) {
+    const uint64_t m = (uint64_t)p->m_mask + 1;
+    return m <= (1ull << 26) ? (size_t)((8 * m + 255) / 256 * 256) : 0;
+}
 cudaError_t launch_decode(const dpb_plan *p, const int32_t *idx, const float *val, int64_t T,
                           const float *xnorm, void *y, int32_t *status, cudaStream_t stream);
 cudaError_t launch_backward(const dpb_plan *p, const void *x, const int32_t *idx,

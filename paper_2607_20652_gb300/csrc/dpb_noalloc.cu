@@ -70,9 +70,9 @@ extern "C" dpb_status dpb_encode_noalloc(const dpb_plan *plan, const void *x, in
         return dpb::fail(DPB_ERR_INVALID_ARG, "idx, val, xnorm, mu and sigma must be 4-byte aligned");
     if ((mu == nullptr) != (sigma == nullptr))
         return dpb::fail(DPB_ERR_INVALID_ARG, "mu and sigma must both be given or both be NULL");
-    size_t need = 0;
-    const dpb_status ws = dpb_workspace_size(plan, T, &need);
-    if (ws != DPB_OK) return ws;
+    // the built-in scratch holds the status word; the optional packed tables
+    // of a workspace are left out (the encoder then reads mu and sigma apart)
+    const size_t need = dpb::kStatusBytes;
     if (need > kNoAllocScratchBytes)
         return dpb::fail(DPB_ERR_UNSUPPORTED,
                          "this plan needs %zu bytes of scratch for T=%lld; the built-in scratch holds %zu",
@@ -90,7 +90,7 @@ extern "C" dpb_status dpb_encode_noalloc(const dpb_plan *plan, const void *x, in
     // the array keeps the previous call's contents: the status word starts at zero
     if (cudaMemsetAsync(status, 0, sizeof(int32_t), s) != cudaSuccess)
         return dpb::fail(DPB_ERR_CUDA, "clearing the built-in scratch failed");
-    const cudaError_t e = dpb::launch_encode(plan, x, T, mu, sigma, idx, val, xnorm, status, s);
+    const cudaError_t e = dpb::launch_encode(plan, x, T, mu, sigma, idx, val, xnorm, status, nullptr, s);
     if (e != cudaSuccess) return dpb::fail(DPB_ERR_CUDA, "encode launch failed: %s", cudaGetErrorString(e));
     if (status_out &&
         cudaMemcpyAsync(status_out, status, sizeof(int32_t), cudaMemcpyDeviceToDevice, s) != cudaSuccess)

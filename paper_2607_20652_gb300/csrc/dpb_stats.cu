@@ -81,11 +81,9 @@ __global__ void __launch_bounds__(kColThreads) stats_columns_kernel(const Tio *x
 
 // ---- levels >= 1: the search on the sampled rows ---------------------------------
 
+// The encoder's standardisation, with the same fp32 arithmetic.
 __device__ __forceinline__ float z_of(float s, uint32_t c, const StatsArgs &a) {
-    if (!a.mu) return s;
-    const float sd = a.sigma[c];
-    if (!(sd > 0.f)) set_status(a.status, DPB_DEV_BAD_SIGMA);
-    return (s - a.mu[c]) / sd;
+    return a.mu ? zscore(s, c, a.mu, a.sigma, nullptr, a.status) : s;
 }
 
 // Ordering priority of a candidate (R9 order: larger first): |z| bits, then

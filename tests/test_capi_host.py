@@ -158,3 +158,11 @@ def test_stats_arguments_are_checked(lib):
     big = dpb.Plan(d=1024, levels=2, bits=[10, 17], children=[0, 256], dtype="bf16",
                    select_mode=dpb.SELECT_PER_LEVEL, k_per_level=[32, 64])
     assert acc(big.handle, buf, 4, None, None, buf, 1, buf, buf, 256, None) == CUDA
+
+
+def test_workspace_holds_the_packed_tables(lib):
+    # 256 bytes for the status word, then 8 bytes per feature for the
+    # standardisation tables packed as (mu, 1 / sigma)
+    for m_bits in (12, 20):
+        plan = dpb.Plan(d=64, levels=3, m_bits=m_bits, children=16, beam=4, k=8, dtype="f32")
+        assert plan.workspace_size(1) == 256 + 8 * (1 << m_bits)

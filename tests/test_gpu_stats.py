@@ -211,3 +211,27 @@ def test_stats_step_moves_the_tables_like_the_oracle():
     moved = (mu_o != mu0.astype(np.float64))
     assert moved.sum() > 256 and np.array_equal(mu_g != mu0, moved)
     assert np.max(np.abs(mu_g - mu_o)) <= 1e-5 and np.max(np.abs(sg_g - sg_o)) <= 1e-5
+
+
+@pytest.mark.parametrize("layout", ["global", "per_level"])
+def test_packed_tables_give_the_same_codes(layout):
+    # A workspace of dpb_workspace_size bytes lets the encoder pack (mu, 1/sigma)
+    # pairs; the 256-byte minimum makes it read the two tables apart. Both use
+    # the same fp32 arithmetic, so the codes must be identical bit for bit.
+    if layout == "global":
+        plan = dpb.Plan(d=768, levels=5, m_bits=20, children=16, beam=8, k=64, dtype="bf16")
+    else:
+        plan = dpb.Plan(d=1024, levels=3, bits=[10, 15, 17], children=[0, 256, 256], dtype="bf16",
+                        select_mode=dpb.SELECT_PER_LEVEL, k_per_level=[16, 32, 64])
+    dev = torch.device("cuda")
+    mu, sigma = inputs.moment_tables(plan.n_features, 50)
+    mu_t, sg_t = torch.from_numpy(mu).to(dev), torch.from_numpy(sigma).to(dev)
+    x = torch.from_numpy(inputs.to_bf16(inputs.gaussian_rows(3000, plan.d, 51))).to(dev).to(torch.bfloat16)
+    full = plan.workspace(len(x), dev)
+    assert full.numel() >= 256 + 8 * plan.n_features
+    small = torch.zeros(256, dtype=torch.uint8, device=dev)
+    a = dpb.encode(plan, x, mu_t, sg_t, workspace=full)
+    b = dpb.encode(plan, x, mu_t, sg_t, workspace=small)
+    torch.cuda.synchronize()
+    assert torch.equal(a[0], b[0]) and torch.equal(a[1], b[1])
+    assert dpb.workspace_status(full) == 0 and dpb.workspace_status(small) == 0
