@@ -662,6 +662,100 @@ def run_per_level(args, world, rank, local):
     return 0
 
 
+# ---------------------------------------------------------------------------
+# the ParityTransformer step (GPT-2 small shape): the DPB's share of a step
+# ---------------------------------------------------------------------------
+
+GPT2_SMALL = dict(layers=12, d=768, heads=12, d_mlp=3072, vocab=50257, context=1024, batch=8)
+GPT2_DPB = dict(levels=5, m_bits=20, children=16, beam=8, k=64)
+
+
+def run_transformer(args, world, rank, local):
+    import torch
+    from paper_2607_20652_gb300 import transformer
+
+    device = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(device)
+    c = GPT2_SMALL
+    B, S = c["batch"], c["context"]
+    g = torch.Generator().manual_seed(shard_seed(7, rank))
+    ids = torch.randint(0, c["vocab"], (B, S), generator=g).to(device)
+    tgt = torch.randint(0, c["vocab"], (B, S), generator=g).to(device)
+    dpb_kw = dict(GPT2_DPB, ema=EMA_ALPHA if args.standardise else None)
+
+    def build(with_dpb):
+        torch.manual_seed(0)
+        m = transformer.ParityTransformer(layers=c["layers"], d=c["d"], heads=c["heads"], d_mlp=c["d_mlp"],
+                                          vocab=c["vocab"], context=c["context"],
+                                          dpb=dpb_kw if with_dpb else None, device=device)
+        return m, torch.optim.AdamW(m.parameters(), lr=1e-4, fused=True)
+
+    def measure(model, opt, dpbs):
+        stream = torch.cuda.current_stream(device)
+
+        def step():
+            opt.zero_grad(set_to_none=True)
+            loss = model(ids, tgt)
+            loss.backward()
+            opt.step()
+            return loss
+
+        for _ in range(args.warmup):
+            step()
+        torch.cuda.synchronize(device)
+        for layer in dpbs:
+            layer.timing = []
+        barrier(world)
+        start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        start.record(stream)
+        for _ in range(args.steps):
+            loss = step()
+        end.record(stream)
+        torch.cuda.synchronize(device)
+        ms = max_over_ranks(start.elapsed_time(end), world, device) / args.steps
+        parts = {"forward": 0.0, "backward": 0.0}
+        for layer in dpbs:
+            for which, ev in layer.timing:
+                parts[which] += ev[0].elapsed_time(ev[1]) / args.steps
+            layer.timing = None
+        return ms, parts, float(loss.detach())
+
+    model, opt = build(True)
+    ms, parts, loss = measure(model, opt, model.dpb_layers())
+    status = 0
+    from paper_2607_20652_gb300 import dpb as _dpb
+    for layer in model.dpb_layers():
+        status |= _dpb.workspace_status(layer._ws)
+    del model, opt
+    torch.cuda.empty_cache()
+    dense_ms = None
+    if not args.no_dense:
+        dense, dopt = build(False)
+        dense_ms, _, _ = measure(dense, dopt, [])
+        del dense, dopt
+    tokens = B * S
+    dpb_ms = parts["forward"] + parts["backward"]
+    per_layer = (3 + (4 if args.standardise else 0))
+    line = {
+        "metric": "ParityTransformer GPT-2-small training step (fwd + bwd + AdamW), tokens/s; DPB share of the step",
+        "value": round(whole_job_rate(tokens, world, 1, ms / 1e3), 1), "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic (uniform random token ids)",
+        "config": {"workload": "gpt2small", **c, "tokens_per_step": tokens,
+                   "dpb": {**GPT2_DPB, "placement": "before every MLP input (§3)",
+                           "standardise": bool(args.standardise)},
+                   "weights": "random init (std 0.02), bf16; AdamW fused", "parallelism": f"dp{world}"},
+        "dpb_ms_per_step": {"forward": round(parts["forward"], 4), "backward": round(parts["backward"], 4),
+                            "total": round(dpb_ms, 4)},
+        "dpb_share": round(dpb_ms / ms, 4),
+        "dense_ms_per_step": round(dense_ms, 4) if dense_ms else None,
+        "loss": round(loss, 4), "gpu_launches": per_layer * c["layers"] * args.steps, "device_status": status,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    return 0
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -676,7 +770,8 @@ def main(argv=None):
                     help="chunks of the batch in the host-buffer run (copies overlap kernels across streams)")
     ap.add_argument("--standardise", action="store_true",
                     help="live standardisation tables and the per-step EMA update in the timed step")
-    ap.add_argument("--workload", default=WORKLOAD, choices=[WORKLOAD, "paper3l", "paper2l"],
+    ap.add_argument("--no-dense", action="store_true", help="gpt2small: skip the dense model of the same shape")
+    ap.add_argument("--workload", default=WORKLOAD, choices=[WORKLOAD, "paper3l", "paper2l", "gpt2small"],
                     help="wide (the headline, global selection) or one of the paper's per-level layouts")
     args = ap.parse_args(argv)
     world, rank, local = dist_env()
@@ -685,6 +780,8 @@ def main(argv=None):
         args.warmup = 3
     if args.impl == "reference":
         return run_reference(args, world, rank)
+    if args.workload == "gpt2small":
+        return run_transformer(args, world, rank, local)
     if args.workload != WORKLOAD:
         return run_per_level(args, world, rank, local)
     return run_ours(args, world, rank, local)
