@@ -320,4 +320,32 @@ __device__ __forceinline__ void load_koff(const uint32_t *M, int d, int t, uint3
     __syncthreads();
 }
 
+// ---- per-code sign words of a 32-coordinate block (backward, moments) --------------
+
+// Per-code parts of the sign words (bit l of block q = parity(M[32q + l] AND
+// c), App. A.4 Eq. 26): o1 = W5[c & 31], the Walsh part; o2 = u | h0 << 11 |
+// h1 << 16 | h2 << 21 | h3 << 26 with u = c_lo >> 5 (the block-parity mask)
+// and h_k the 5-bit chunks of the high half.
+__device__ __forceinline__ void code_offsets(uint32_t c, int t, const uint32_t *w5, uint32_t &o1, uint32_t &o2) {
+    const uint32_t u = (c & ((1u << t) - 1u)) >> 5;
+    uint32_t h = 0;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) h |= ((c >> min(t + 5 * k, 31)) & 31u) << (5 * k);
+    o1 = w5[c & 31u];
+    o2 = u | (h << 11);
+}
+
+// Sign word of code (o1, o2) over block q (VH2 holds NKC chunk tables of
+// nblk blocks x 32 words).
+template <int NKC>
+__device__ __forceinline__ uint32_t block_signs(const uint32_t *vh2, int nblk, int q, uint32_t o1, uint32_t o2) {
+    const uint32_t *V = vh2 + q * 32;
+    uint32_t s = o1 ^ (0u - (uint32_t)(__popc((uint32_t)q & (o2 & 0x7FFu)) & 1));
+    s ^= V[(o2 >> 11) & 31u];
+    s ^= V[nblk * 32 + ((o2 >> 16) & 31u)];
+    if (NKC > 2) s ^= V[2 * nblk * 32 + ((o2 >> 21) & 31u)];
+    if (NKC > 3) s ^= V[3 * nblk * 32 + ((o2 >> 26) & 31u)];
+    return s;
+}
+
 }  // namespace dpb

@@ -8,15 +8,21 @@
 //              block per row re-runs the encoder's search (kept set of each
 //              level = its top keep[l] by standardised score, children
 //              p ^ g_j, each distinct child scored once) and adds every
-//              child's raw score to the sums.
+//              child's raw score to the sums. A thread scores one child:
+//              per 32-coordinate block, the child's sign word (from the
+//              plan's per-block tables) indexes eight 16-entry tables of the
+//              row's signed nibble sums (d <= 2048; a warp of popcounts per
+//              child beyond).
 //   update     a pass over the 2^N count words; only touched features read
 //              their sums, move their moments and clear the sums.
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cstdint>
 
 #include "dpb_device.cuh"
 #include "dpb_internal.h"
+#include "dpb_lut.cuh"
 
 namespace dpb {
 namespace {
@@ -27,6 +33,8 @@ constexpr int kColChunk = 32;     // rows per fp32 partial before it joins the f
 constexpr int kSearchThreads = 512;
 constexpr int kSearchWarps = kSearchThreads / 32;
 constexpr int kMaxKeep = 64;
+constexpr int kGenSlots = 512;    // open-addressing slots of one level's generator set
+constexpr int kNibStride = 17;    // a nibble table: 16 sums + 1 pad word (bank spread)
 
 struct StatsArgs {
     const void *x;
@@ -44,7 +52,36 @@ struct StatsArgs {
     float inv_sqrt_d;
     int cap;            // per-level candidate slots (smem)
     int32_t *status;
+    const uint32_t *VH2;  // [nkc][nblk][32] inverse-coordinate sign words (d <= 2048)
+    int t;                // field degree
 };
+
+// Shared-memory carve-up of the search block (32-bit words).
+struct SearchLayout {
+    int xs, ms, th, vh, w5, par, gen, gslot, red, hist, zb, cid, words;
+};
+
+__host__ __device__ inline SearchLayout search_layout(int d, int nkc, int cap) {
+    const int nblk = (d + 31) / 32;
+    SearchLayout L{};
+    int o = 0;
+    L.xs = o, o += pad4(d);
+    L.ms = o, o += nkc ? 0 : pad4(d);                        // M rows (popcount scoring)
+    L.th = o, o += nkc ? pad4(nblk * 8 * kNibStride) : 0;    // nibble sums of the row
+    L.vh = o, o += nkc * nblk * 32;
+    L.w5 = o, o += 32;
+    L.par = o, o += kMaxKeep;
+    L.gen = o, o += DPB_MAX_CHILDREN;
+    L.gslot = o, o += kGenSlots;
+    L.red = o, o += 32;
+    L.hist = o, o += 256;
+    L.zb = o, o += cap;
+    L.cid = o, o += cap;
+    L.words = o;
+    return L;
+}
+
+__device__ __forceinline__ uint32_t gen_hash(uint32_t v) { return (v * 2654435761u) >> 23; }  // 9 bits
 
 __device__ __forceinline__ void add_moments(double *acc, int64_t m, uint32_t c, double s, double n = 1.0) {
     atomicAdd(acc + c, n);
@@ -108,115 +145,211 @@ __device__ __forceinline__ int block_sum(int v, int *red) {
 
 // The keep largest priorities among n slots (slots with zb < 0 are not
 // candidates): writes their indices to par and returns how many. PR(i) gives
-// slot i's priority. The threshold is the keep-th largest priority, built bit
-// by bit from the top (priorities are distinct).
+// slot i's priority. The threshold is the keep-th largest priority, found one
+// byte at a time from the top by 256-bin histograms (priorities are
+// distinct, so exactly keep slots reach it).
 template <typename PR>
-__device__ int select_top(int n, int keep, const float *zb, PR pr, uint32_t *par, int *red, int *cnt,
+__device__ int select_top(int n, int keep, const float *zb, PR pr, uint32_t *par, int *red, int *hist,
                           const uint32_t *cid) {
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     int valid = 0;
-    for (int i = threadIdx.x; i < n; i += blockDim.x) valid += zb[i] >= 0.f;
+    for (int i = tid; i < n; i += blockDim.x) valid += zb[i] >= 0.f;
     valid = block_sum(valid, red);
     const int K = keep < valid ? keep : valid;
     uint64_t tau = 0;
     if (K < valid) {
-        for (int bit = 63; bit >= 0; --bit) {
-            const uint64_t cand = tau | (1ull << bit);
-            int c = 0;
-            for (int i = threadIdx.x; i < n; i += blockDim.x)
-                if (zb[i] >= 0.f && pr(i) >= cand) ++c;
-            if (block_sum(c, red) >= K) tau = cand;
+        int need = K;
+        for (int shift = 56; shift >= 0; shift -= 8) {
+            const uint64_t hi = shift == 56 ? 0ull : ~0ull << (shift + 8);
+            for (int i = tid; i < 256; i += blockDim.x) hist[i] = 0;
+            __syncthreads();
+            for (int i = tid; i < n; i += blockDim.x) {
+                if (zb[i] < 0.f) continue;
+                const uint64_t P = pr(i);
+                if ((P & hi) == (tau & hi)) atomicAdd(&hist[(P >> shift) & 255u], 1);
+            }
+            __syncthreads();
+            if (warp == 0) {
+                // lane owns bins 255 - 8 lane - r, r < 8 (descending); counts above it
+                int cnt[8], tot = 0;
+#pragma unroll
+                for (int r = 0; r < 8; ++r) tot += (cnt[r] = hist[255 - 8 * lane - r]);
+                int incl = tot;
+#pragma unroll
+                for (int o = 1; o < 32; o <<= 1) {
+                    const int v = __shfl_up_sync(kFull, incl, o);
+                    if (lane >= o) incl += v;
+                }
+                int run = incl - tot;
+                if (run < need && need <= incl) {
+#pragma unroll
+                    for (int r = 0; r < 8; ++r) {
+                        if (run + cnt[r] >= need) {
+                            red[kSearchWarps] = 255 - 8 * lane - r;
+                            red[kSearchWarps + 1] = run;
+                            break;
+                        }
+                        run += cnt[r];
+                    }
+                }
+            }
+            __syncthreads();
+            tau |= (uint64_t)red[kSearchWarps] << shift;
+            need -= red[kSearchWarps + 1];
+            __syncthreads();
         }
     }
-    if (threadIdx.x == 0) *cnt = 0;
+    int *cnt = red + kSearchWarps + 2;
+    if (tid == 0) *cnt = 0;
     __syncthreads();
-    for (int i = threadIdx.x; i < n; i += blockDim.x)
+    for (int i = tid; i < n; i += blockDim.x)
         if (zb[i] >= 0.f && pr(i) >= tau) par[atomicAdd(cnt, 1)] = cid[i];
     __syncthreads();
     return K;
 }
 
-template <typename Tio>
+// NKC > 0: table-driven scoring (d <= 2048, NKC chunk tables); NKC == 0: a
+// warp of popcounts per child.
+template <typename Tio, int NKC>
 __global__ void __launch_bounds__(kSearchThreads, 1) stats_search_kernel(StatsArgs a) {
     extern __shared__ __align__(16) uint32_t smem[];
-    const int d = a.d;
-    float *xs = reinterpret_cast<float *>(smem);          // [d]
-    uint32_t *Ms = smem + d;                             // [d]
-    uint32_t *par = Ms + d;                              // [kMaxKeep]
-    uint32_t *gen = par + kMaxKeep;                      // [DPB_MAX_CHILDREN]
-    uint32_t *gsort = gen + DPB_MAX_CHILDREN;            // [DPB_MAX_CHILDREN] ascending
-    int *red = reinterpret_cast<int *>(gsort + DPB_MAX_CHILDREN);  // [kSearchWarps + 1]
-    float *zb = reinterpret_cast<float *>(red + kSearchWarps + 4);  // [cap] |z| (-1: not a candidate)
-    uint32_t *cid = reinterpret_cast<uint32_t *>(zb + a.cap);       // [cap] candidate index
+    const int d = a.d, nblk = (d + 31) / 32;
+    const SearchLayout L = search_layout(d, NKC, a.cap);
+    float *xs = reinterpret_cast<float *>(smem + L.xs);
+    uint32_t *Ms = smem + L.ms;
+    float *TH = reinterpret_cast<float *>(smem + L.th);
+    uint32_t *vh = smem + L.vh;
+    uint32_t *w5 = smem + L.w5;
+    uint32_t *par = smem + L.par;
+    uint32_t *gen = smem + L.gen;
+    uint32_t *gslot = smem + L.gslot;
+    int *red = reinterpret_cast<int *>(smem + L.red);
+    int *hist = reinterpret_cast<int *>(smem + L.hist);
+    float *zb = reinterpret_cast<float *>(smem + L.zb);  // |z| (-1: not a candidate)
+    uint32_t *cid = smem + L.cid;                         // candidate index
 
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int32_t row = a.sample[blockIdx.x];
     if (row < 0 || row >= a.T) {
-        if (threadIdx.x == 0) set_status(a.status, DPB_DEV_BAD_INDEX);
+        if (tid == 0) set_status(a.status, DPB_DEV_BAD_INDEX);
         return;
     }
     const Tio *xr = static_cast<const Tio *>(a.x) + (int64_t)row * d;
-    for (int i = threadIdx.x; i < d; i += blockDim.x) {
+    for (int i = tid; i < d; i += blockDim.x) {
         xs[i] = ld_elem(xr, i);
-        Ms[i] = a.M[i];
+        if (NKC == 0) Ms[i] = a.M[i];
+    }
+    if (NKC > 0) {
+        for (int i = tid; i < NKC * nblk * 32; i += blockDim.x) vh[i] = a.VH2[i];
+        if (tid < 32) {
+            uint32_t word = 0;
+            for (int l = 0; l < 32; ++l) word |= (uint32_t)(__popc(l & tid) & 1) << l;
+            w5[tid] = word;
+        }
     }
     __syncthreads();
+    if (NKC > 0) {
+        // nibble table tau (coordinates 4 tau .. 4 tau + 3): entry v = sum_j (-1)^{v_j} x[4 tau + j]
+        for (int tau = tid; tau < nblk * 8; tau += blockDim.x) {
+            const int i0 = 4 * tau;
+            const float h0 = i0 < d ? xs[i0] : 0.f, h1 = i0 + 1 < d ? xs[i0 + 1] : 0.f;
+            const float h2 = i0 + 2 < d ? xs[i0 + 2] : 0.f, h3 = i0 + 3 < d ? xs[i0 + 3] : 0.f;
+            const float A[4] = {h0 + h1, h1 - h0, h0 - h1, -h0 - h1};
+            const float B[4] = {h2 + h3, h3 - h2, h2 - h3, -h2 - h3};
+            float *T = TH + tau * kNibStride;
+#pragma unroll
+            for (int v = 0; v < 16; ++v) T[v] = A[v & 3] + B[v >> 2];
+        }
+    }
     // level 0: the basis coordinates
-    for (int i = threadIdx.x; i < d; i += blockDim.x) {
+    for (int i = tid; i < d; i += blockDim.x) {
         zb[i] = fabsf(z_of(xs[i], (uint32_t)i, a));
         cid[i] = (uint32_t)i;
     }
     __syncthreads();
-    int np = select_top(
-        d, a.keep[0], zb, [&](int i) { return prio(zb[i], cid[i]); }, par, red, red + kSearchWarps, cid);
+    auto pri = [&](int i) { return prio(zb[i], cid[i]); };
+    int np = select_top(d, a.keep[0], zb, pri, par, red, hist, cid);
 
     for (int l = 1; l < a.levels; ++l) {
         const int nch = a.children[l];
-        for (int j = threadIdx.x; j < nch; j += blockDim.x) gen[j] = a.G[l * DPB_MAX_CHILDREN + j];
+        for (int j = tid; j < nch; j += blockDim.x) gen[j] = a.G[l * DPB_MAX_CHILDREN + j];
+        for (int j = tid; j < kGenSlots; j += blockDim.x) gslot[j] = 0u;
         __syncthreads();
-        for (int j = threadIdx.x; j < nch; j += blockDim.x) {  // generators are distinct
-            int rank = 0;
-            for (int i = 0; i < nch; ++i) rank += gen[i] < gen[j];
-            gsort[rank] = gen[j];
+        // the level's generator set (distinct values; key g + 1, 0 = empty)
+        for (int j = tid; j < nch; j += blockDim.x) {
+            uint32_t h = gen_hash(gen[j]);
+            for (int probe = 0; probe < kGenSlots; ++probe) {
+                if (atomicCAS(&gslot[h], 0u, gen[j] + 1u) == 0u) break;
+                h = (h + 1u) & (kGenSlots - 1);
+            }
         }
         __syncthreads();
-        // pair (b, j) -> child par[b] ^ gen[j]; it is a repeat when an earlier
-        // parent b' < b reaches the same child, i.e. child ^ par[b'] is a generator
-        const int n = np * nch;
-        for (int i = warp; i < n; i += kSearchWarps) {
-            const int b = i / nch;
-            const uint32_t c = par[b] ^ gen[i - b * nch];
-            bool rep = false;
-            for (int bb = lane; bb < b; bb += 32) {
+        // pair (b, j) -> child par[b] ^ gen[j]; a repeat when an earlier parent
+        // b' < b reaches the same child, i.e. child ^ par[b'] is a generator
+        auto repeat = [&](uint32_t c, int b) {
+            for (int bb = 0; bb < b; ++bb) {
                 const uint32_t v = c ^ par[bb];
-                int lo = 0, hi = nch - 1;
-                while (lo < hi) {
-                    const int mid = (lo + hi) >> 1;
-                    if (gsort[mid] < v) lo = mid + 1; else hi = mid;
+                uint32_t h = gen_hash(v);
+                for (int probe = 0; probe < kGenSlots; ++probe) {
+                    const uint32_t e = gslot[h];
+                    if (e == 0u) break;
+                    if (e == v + 1u) return true;
+                    h = (h + 1u) & (kGenSlots - 1);
                 }
-                rep |= gsort[lo] == v;
             }
-            rep = __any_sync(kFull, rep);
-            float s = 0.f;
-            if (!rep) {
+            return false;
+        };
+        const int n = np * nch;
+        if (NKC > 0) {
+            for (int i = tid; i < n; i += blockDim.x) {
+                const int b = i / nch;
+                const uint32_t c = par[b] ^ gen[i - b * nch];
+                cid[i] = c;
+                if (repeat(c, b)) {
+                    zb[i] = -1.f;
+                    continue;
+                }
+                uint32_t o1, o2;
+                code_offsets(c, a.t, w5, o1, o2);
+                float acc = 0.f;
+                for (int q = 0; q < nblk; ++q) {
+                    const uint32_t sw = block_signs<(NKC > 1 ? NKC : 2)>(vh, nblk, q, o1, o2);
+                    const float *T = TH + q * 8 * kNibStride;
+                    float part = 0.f;
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) part += T[k * kNibStride + ((sw >> (4 * k)) & 15u)];
+                    acc += part;
+                }
+                float s = acc * a.inv_sqrt_d;
+                if (c < (uint32_t)d) s = xs[c];  // basis override (Eq. 2); not reached by the level rule
+                if ((int64_t)c < a.m) add_moments(a.acc, a.m, c, (double)s);
+                zb[i] = fabsf(z_of(s, c, a));
+            }
+        } else {
+            for (int i = warp; i < n; i += kSearchWarps) {
+                const int b = i / nch;
+                const uint32_t c = par[b] ^ gen[i - b * nch];
+                const bool rep = lane == 0 && repeat(c, b);
+                if (__shfl_sync(kFull, rep, 0)) {
+                    if (lane == 0) {
+                        cid[i] = c;
+                        zb[i] = -1.f;
+                    }
+                    continue;
+                }
+                float s = 0.f;
                 for (int io = lane; io < d; io += 32) s += flip(xs[io], sign31(Ms[io], c));
                 s = warp_sum(s) * a.inv_sqrt_d;
-                if (c < (uint32_t)d) s = xs[c];  // basis override (Eq. 2); not reached by the level rule
-            }
-            if (lane == 0) {
-                cid[i] = c;
-                if (rep) {
-                    zb[i] = -1.f;
-                } else {
+                if (c < (uint32_t)d) s = xs[c];
+                if (lane == 0) {
+                    cid[i] = c;
                     if ((int64_t)c < a.m) add_moments(a.acc, a.m, c, (double)s);
                     zb[i] = fabsf(z_of(s, c, a));
                 }
             }
         }
         __syncthreads();
-        if (l + 1 < a.levels)
-            np = select_top(
-                n, a.keep[l], zb, [&](int i) { return prio(zb[i], cid[i]); }, par, red, red + kSearchWarps,
-                cid);
+        if (l + 1 < a.levels) np = select_top(n, a.keep[l], zb, pri, par, red, hist, cid);
     }
 }
 
@@ -242,6 +375,15 @@ __global__ void stats_update_kernel(double *acc, int64_t m, double alpha, float 
     }
 }
 
+template <typename Tio, int NKC>
+cudaError_t run_search(const StatsArgs &a, int32_t n_sample, size_t smem, cudaStream_t stream) {
+    const cudaError_t e =
+        cudaFuncSetAttribute(stats_search_kernel<Tio, NKC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    stats_search_kernel<Tio, NKC><<<n_sample, kSearchThreads, smem, stream>>>(a);
+    return cudaGetLastError();
+}
+
 int search_cap(const dpb_plan *p, const int *keep) {
     int cap = p->cfg.d;
     for (int l = 1; l < p->cfg.levels; ++l) {
@@ -251,8 +393,10 @@ int search_cap(const dpb_plan *p, const int *keep) {
     return cap;
 }
 
-size_t search_smem(int d, int cap) {
-    return sizeof(uint32_t) * (2 * (size_t)d + kMaxKeep + 2 * DPB_MAX_CHILDREN + kSearchWarps + 4 + 2 * (size_t)cap);
+int search_nkc(const dpb_plan *p) { return p->cfg.d <= 2048 ? std::max(2, p->kvh) : 0; }
+
+size_t search_smem(const dpb_plan *p, int cap) {
+    return sizeof(uint32_t) * (size_t)search_layout(p->cfg.d, search_nkc(p), cap).words;
 }
 
 void keep_of(const dpb_plan *p, int *keep) {
@@ -267,7 +411,7 @@ bool stats_supported(const dpb_plan *p, size_t *smem_out) {
     keep_of(p, keep);
     for (int l = 0; l < p->cfg.levels; ++l)
         if (keep[l] < 1 || keep[l] > kMaxKeep) return false;
-    const size_t smem = search_smem(p->cfg.d, search_cap(p, keep));
+    const size_t smem = search_smem(p, search_cap(p, keep));
     if (smem_out) *smem_out = smem;
     return smem <= (size_t)kMaxSmemPerBlock;
 }
@@ -306,19 +450,20 @@ cudaError_t launch_stats_accumulate(const dpb_plan *p, const void *x, int64_t T,
     a.inv_sqrt_d = p->inv_sqrt_d;
     a.cap = search_cap(p, a.keep);
     a.status = status;
-    const size_t smem = search_smem(d, a.cap);
+    a.VH2 = p->dVH2;
+    a.t = p->t;
+    const size_t smem = search_smem(p, a.cap);
+    const int nkc = search_nkc(p);
     if (p->cfg.dtype == DPB_BF16) {
-        cudaError_t e = cudaFuncSetAttribute(stats_search_kernel<__nv_bfloat16>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        stats_search_kernel<__nv_bfloat16><<<n_sample, kSearchThreads, smem, stream>>>(a);
-    } else {
-        cudaError_t e = cudaFuncSetAttribute(stats_search_kernel<float>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        stats_search_kernel<float><<<n_sample, kSearchThreads, smem, stream>>>(a);
+        if (nkc == 0) return run_search<__nv_bfloat16, 0>(a, n_sample, smem, stream);
+        if (nkc == 2) return run_search<__nv_bfloat16, 2>(a, n_sample, smem, stream);
+        if (nkc == 3) return run_search<__nv_bfloat16, 3>(a, n_sample, smem, stream);
+        return run_search<__nv_bfloat16, 4>(a, n_sample, smem, stream);
     }
-    return cudaGetLastError();
+    if (nkc == 0) return run_search<float, 0>(a, n_sample, smem, stream);
+    if (nkc == 2) return run_search<float, 2>(a, n_sample, smem, stream);
+    if (nkc == 3) return run_search<float, 3>(a, n_sample, smem, stream);
+    return run_search<float, 4>(a, n_sample, smem, stream);
 }
 
 cudaError_t launch_stats_update(const dpb_plan *p, double *acc, float alpha, float *mu, float *sigma,

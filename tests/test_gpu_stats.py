@@ -148,6 +148,17 @@ def test_ragged_level0_and_empty_sample(T, d):
     assert not acc_g[:, d:].any()
 
 
+def test_moments_beyond_the_sign_tables():
+    # d > 2048: the sampled search scores each child with a warp of popcounts
+    plan, ref = _pair(dtype="f32", d=2304, levels=3, m_bits=16, children=16, beam=4, k=8)
+    x = inputs.gaussian_rows(40, 2304, 24)
+    rows = _safe_rows(ref, x, 6, 25)
+    acc_g, st = _gpu_acc(plan, x, rows)
+    acc_o = oracle.stats_accumulate(ref, x.astype(np.float64), rows)
+    assert st == 0
+    print(_compare(acc_g, acc_o, x, rows, 2304))
+
+
 def test_bad_rows_are_flagged_and_skipped():
     plan, ref = _pair(dtype="f32", d=64, levels=3, m_bits=12, children=16, beam=4, k=8)
     x = inputs.gaussian_rows(20, 64, 19)
