@@ -468,11 +468,12 @@ cudaError_t launch_stats_accumulate(const dpb_plan *p, const void *x, int64_t T,
 
 cudaError_t launch_stats_update(const dpb_plan *p, double *acc, float alpha, float *mu, float *sigma,
                                 cudaStream_t stream) {
+    // one feature per thread: the touched features' dependent loads and fp64
+    // arithmetic then all run at once instead of in a grid-stride chain
     const int64_t m = (int64_t)p->m_mask + 1;
-    int sms = 0;
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, p->device);
-    const int64_t want = (m + 255) / 256, cap = (int64_t)sms * 8;
-    stats_update_kernel<<<(unsigned)(want < cap ? want : cap), 256, 0, stream>>>(acc, m, (double)alpha, mu, sigma);
+    const int64_t blocks = (m + 255) / 256;
+    stats_update_kernel<<<(unsigned)(blocks < 0x7fffffff ? blocks : 0x7fffffff), 256, 0, stream>>>(
+        acc, m, (double)alpha, mu, sigma);
     return cudaGetLastError();
 }
 
