@@ -476,7 +476,9 @@ def run_e2e(plan, x, gy, args, device, stream, world):
     its inputs from pinned host memory and its outputs back, inside the timed
     region. The batch runs as chunks on a few streams, so one chunk's copies
     overlap another's kernels (each stream keeps its own device buffers and
-    workspace; calls on one stream run in order)."""
+    workspace; calls on one stream run in order). A chunk's x and grad_y sit
+    side by side in host memory and move in one copy; its outputs come back in
+    two (the [C, k] arrays, then y and grad_x)."""
     import torch
     from paper_2607_20652_gb300 import dpb
     T, d = x.shape
@@ -485,42 +487,35 @@ def run_e2e(plan, x, gy, args, device, stream, world):
     while T % nch:
         nch -= 1
     C = T // nch
-    hx = torch.empty_like(x, device="cpu").pin_memory()
-    hgy = torch.empty_like(gy, device="cpu").pin_memory()
-    hx.copy_(x)
-    hgy.copy_(gy)
-    outs = {"idx": torch.empty((T, k), dtype=torch.int32).pin_memory(),
-            "val": torch.empty((T, k), dtype=torch.float32).pin_memory(),
-            "y": torch.empty((T, d), dtype=torch.bfloat16).pin_memory(),
-            "gx": torch.empty((T, d), dtype=torch.bfloat16).pin_memory(),
-            "gv": torch.empty((T, k), dtype=torch.float32).pin_memory()}
-    nstreams = min(3, nch)
+    hin = torch.empty((nch, 2, C, d), dtype=x.dtype).pin_memory()       # [chunk][x | grad_y]
+    hin[:, 0].copy_(x.view(nch, C, d))
+    hin[:, 1].copy_(gy.view(nch, C, d))
+    hsmall = torch.empty((nch, 3, C, k), dtype=torch.int32).pin_memory()  # [chunk][idx | val | grad_val]
+    hbig = torch.empty((nch, 2, C, d), dtype=x.dtype).pin_memory()       # [chunk][y | grad_x]
+    nstreams = max(1, min(args.e2e_streams, nch))
     streams = [torch.cuda.Stream(device) for _ in range(nstreams)]
     bufs = []
     for _ in range(nstreams):
-        bufs.append({"x": torch.empty((C, d), dtype=x.dtype, device=device),
-                     "gy": torch.empty((C, d), dtype=gy.dtype, device=device),
-                     "idx": torch.empty((C, k), dtype=torch.int32, device=device),
-                     "val": torch.empty((C, k), dtype=torch.float32, device=device),
+        inp = torch.empty((2, C, d), dtype=x.dtype, device=device)
+        small = torch.empty((3, C, k), dtype=torch.int32, device=device)
+        big = torch.empty((2, C, d), dtype=x.dtype, device=device)
+        bufs.append({"inp": inp, "x": inp[0], "gy": inp[1], "small": small, "idx": small[0],
+                     "val": small[1].view(torch.float32), "gv": small[2].view(torch.float32),
+                     "big": big, "y": big[0], "gx": big[1],
                      "xn": torch.empty((C,), dtype=torch.float32, device=device),
-                     "y": torch.empty((C, d), dtype=x.dtype, device=device),
-                     "gx": torch.empty((C, d), dtype=x.dtype, device=device),
-                     "gv": torch.empty((C, k), dtype=torch.float32, device=device),
                      "ws": plan.workspace(C, device)})
 
     def step():
         for i in range(nch):
             st, b = streams[i % nstreams], bufs[i % nstreams]
-            rows = slice(i * C, (i + 1) * C)
             with torch.cuda.stream(st):
-                b["x"].copy_(hx[rows], non_blocking=True)
-                b["gy"].copy_(hgy[rows], non_blocking=True)
+                b["inp"].copy_(hin[i], non_blocking=True)
                 dpb.encode(plan, b["x"], idx=b["idx"], val=b["val"], xnorm=b["xn"], workspace=b["ws"], stream=st)
                 dpb.decode(plan, b["idx"], b["val"], b["xn"], y=b["y"], workspace=b["ws"], stream=st)
                 dpb.backward(plan, b["x"], b["idx"], b["val"], b["gy"], grad_x=b["gx"], grad_val=b["gv"],
                              workspace=b["ws"], stream=st)
-                for name in ("idx", "val", "y", "gx", "gv"):
-                    outs[name][rows].copy_(b[name], non_blocking=True)
+                hsmall[i].copy_(b["small"], non_blocking=True)
+                hbig[i].copy_(b["big"], non_blocking=True)
 
     def timed(fn):
         for _ in range(max(1, args.warmup)):
@@ -538,8 +533,8 @@ def run_e2e(plan, x, gy, args, device, stream, world):
     status = 0
     for b in bufs:
         status |= dpb.workspace_status(b["ws"])
-    bi = hx.numel() * hx.element_size() + hgy.numel() * hgy.element_size()
-    bo = sum(t.numel() * t.element_size() for t in outs.values())
+    bi = hin.numel() * hin.element_size()
+    bo = hsmall.numel() * hsmall.element_size() + hbig.numel() * hbig.element_size()
     return {"value": round(whole_job_rate(T, world, steps, secs), 1), "unit": "tokens/s",
             "h2d_bytes_per_step": bi, "d2h_bytes_per_step": bo, "steps": steps,
             "chunks": nch, "streams": nstreams, "device_status": status}
@@ -766,6 +761,7 @@ def main(argv=None):
     ap.add_argument("--ref-tokens", type=int, default=512)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--e2e-streams", type=int, default=4, help="streams of the host-buffer run")
     ap.add_argument("--e2e-chunks", type=int, default=8,
                     help="chunks of the batch in the host-buffer run (copies overlap kernels across streams)")
     ap.add_argument("--standardise", action="store_true",
