@@ -326,12 +326,14 @@ def run_reference(args, world, rank):
     return 0
 
 
-def config_block(w, world, n_tokens=None, standardise=False):
+def config_block(w, world, n_tokens=None, standardise=False, keep_r=False):
     c = {"workload": WORKLOAD, "T_per_gpu": n_tokens or w["T"], "d": w["d"], "features": 2 ** w["m_bits"],
          "levels": w["levels"], "children": w["children"], "beam": w["beam"], "k": w["k"],
          "accumulate": "fp32", "inputs": "planted tree of 64 parity directions + N(0,0.1^2), bf16",
          "l2": "working set ~450 MB > 129 MB L2 (no flush needed)",
          "parallelism": f"dp{world} (independent token shards)"}
+    if keep_r:
+        c["r_kept"] = "decode keeps r (fp32 [T, d]) for the backward"
     if standardise:
         c["standardise"] = {"tables": "live fp32 mu/sigma (2^N each)", "ema_sample_rows": EMA_SAMPLE,
                             "ema_alpha": EMA_ALPHA,
@@ -361,6 +363,8 @@ def run_ours(args, world, rank, local):
     y = torch.empty_like(x)
     gx = torch.empty_like(x)
     gv = torch.empty((T, k), dtype=torch.float32, device=device)
+    # decode keeps r (fp32) for the backward, which then does not rebuild it
+    rk = None if args.no_keep_r else torch.empty((T, d), dtype=torch.float32, device=device)
     ws = plan.workspace(T, device)
     stream = torch.cuda.current_stream(device)
     # live standardisation (§2.2): encode and backward read the tables, and
@@ -383,10 +387,10 @@ def run_ours(args, world, rank, local):
         dpb.encode(plan, x, mu_t, sg_t, idx=idx, val=val, xnorm=xn, workspace=ws, stream=stream)
         if ev:
             ev[1].record(stream)
-        dpb.decode(plan, idx, val, xn, y=y, workspace=ws, stream=stream)
+        dpb.decode(plan, idx, val, xn, y=y, workspace=ws, stream=stream, r_out=rk)
         if ev:
             ev[2].record(stream)
-        dpb.backward(plan, x, idx, val, gy, sigma=sg_t, grad_x=gx, grad_val=gv, workspace=ws, stream=stream)
+        dpb.backward(plan, x, idx, val, gy, sigma=sg_t, grad_x=gx, grad_val=gv, workspace=ws, stream=stream, r=rk)
         if ev:
             ev[3].record(stream)
         if std:
@@ -451,7 +455,7 @@ def run_ours(args, world, rank, local):
         "metric": METRIC, "value": round(value, 1), "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_max / args.steps, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-        "data": "synthetic", "config": config_block(w, world, standardise=std),
+        "data": "synthetic", "config": config_block(w, world, standardise=std, keep_r=rk is not None),
         "roofline": roof,
         "step_roofline": {"t_roofline_us": round(step_roof_us, 2),
                           "t_measured_us": round(1e3 * ms_max / args.steps, 2),
@@ -503,6 +507,7 @@ def run_e2e(plan, x, gy, args, device, stream, world):
                      "val": small[1].view(torch.float32), "gv": small[2].view(torch.float32),
                      "big": big, "y": big[0], "gx": big[1],
                      "xn": torch.empty((C,), dtype=torch.float32, device=device),
+                     "r": None if args.no_keep_r else torch.empty((C, d), dtype=torch.float32, device=device),
                      "ws": plan.workspace(C, device)})
 
     def step():
@@ -511,9 +516,9 @@ def run_e2e(plan, x, gy, args, device, stream, world):
             with torch.cuda.stream(st):
                 b["inp"].copy_(hin[i], non_blocking=True)
                 dpb.encode(plan, b["x"], idx=b["idx"], val=b["val"], xnorm=b["xn"], workspace=b["ws"], stream=st)
-                dpb.decode(plan, b["idx"], b["val"], b["xn"], y=b["y"], workspace=b["ws"], stream=st)
+                dpb.decode(plan, b["idx"], b["val"], b["xn"], y=b["y"], workspace=b["ws"], stream=st, r_out=b["r"])
                 dpb.backward(plan, b["x"], b["idx"], b["val"], b["gy"], grad_x=b["gx"], grad_val=b["gv"],
-                             workspace=b["ws"], stream=st)
+                             workspace=b["ws"], stream=st, r=b["r"])
                 hsmall[i].copy_(b["small"], non_blocking=True)
                 hbig[i].copy_(b["big"], non_blocking=True)
 
@@ -762,6 +767,7 @@ def main(argv=None):
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-streams", type=int, default=4, help="streams of the host-buffer run")
+    ap.add_argument("--no-keep-r", action="store_true", help="backward rebuilds r instead of reading the decode's")
     ap.add_argument("--e2e-chunks", type=int, default=8,
                     help="chunks of the batch in the host-buffer run (copies overlap kernels across streams)")
     ap.add_argument("--standardise", action="store_true",

@@ -180,10 +180,12 @@ dpb_status dpb_encode(const dpb_plan *plan, const void *x, int64_t T, const floa
  *             [0, 2^N) are skipped and flagged DPB_DEV_BAD_INDEX
  *   xnorm     [T] fp32, required iff norm_match
  *   y         out [T][d] plan dtype, 16-byte aligned
+ *   r_out     out fp32 [T][d], 16-byte aligned, nullable: r_t itself, kept
+ *             for dpb_backward (which then does not rebuild it)
  */
 dpb_status dpb_decode(const dpb_plan *plan, const int32_t *idx, const float *val, int64_t T,
-                      const float *xnorm, void *y, void *workspace, size_t workspace_bytes,
-                      void *stream);
+                      const float *xnorm, void *y, float *r_out, void *workspace,
+                      size_t workspace_bytes, void *stream);
 
 /*
  * dpb_backward -- gradients of L(decode(encode(x))) with the selected set
@@ -193,11 +195,14 @@ dpb_status dpb_decode(const dpb_plan *plan, const int32_t *idx, const float *val
  *   grad_x     = sum_e (grad_val_e / sigma_e) phi_e + (<g,r>/|r|) x / |x|
  * (the last term only with norm_match; zero gradients when |r| = 0).
  *   x, grad_y  [T][d] plan dtype; idx, val [T][k]; sigma [2^N] fp32 nullable
+ *   r          fp32 [T][d], 16-byte aligned, nullable: the r_out of the
+ *              dpb_decode of this code; given, it replaces the rebuilding of
+ *              r (same value up to fp32 summation order)
  *   grad_x     out [T][d] plan dtype; grad_val out fp32 [T][k]
  */
 dpb_status dpb_backward(const dpb_plan *plan, const void *x, const int32_t *idx,
-                        const float *val, int64_t T, const float *sigma, const void *grad_y,
-                        void *grad_x, float *grad_val, void *workspace,
+                        const float *val, int64_t T, const float *sigma, const float *r,
+                        const void *grad_y, void *grad_x, float *grad_val, void *workspace,
                         size_t workspace_bytes, void *stream);
 
 /*

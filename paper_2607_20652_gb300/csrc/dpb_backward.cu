@@ -26,6 +26,7 @@ struct BackwardArgs {
     const void *x, *gy;
     const int32_t *idx;
     const float *val, *sigma;
+    const float *R;  // nullable: r of the decode, fp32 [T][d], instead of rebuilding it
     void *gx;
     float *gval;
     int64_t T;
@@ -88,11 +89,11 @@ __global__ void __launch_bounds__(128) backward_warp_kernel(BackwardArgs a) {
         const float nx = sqrtf(warp_sum(sxx));
         float direct = 0.f;  // coefficient of x/|x| in grad_x
         if (a.norm_match) {
-            reconstruct(it, vt, a.k, d, a.m_mask, sM, rb, rh, a.status);
+            if (!a.R) reconstruct(it, vt, a.k, d, a.m_mask, sM, rb, rh, a.status);
             __syncwarp();
             float srr = 0.f, sgr = 0.f;
             for (int i = lane; i < d; i += 32) {
-                const float r = rb[i] + rh[i] * a.inv_sqrt_d;
+                const float r = a.R ? a.R[t * d + i] : rb[i] + rh[i] * a.inv_sqrt_d;
                 rb[i] = r;
                 srr += r * r;
                 sgr += ld_elem(GY, t * d + i) * r;
@@ -358,7 +359,10 @@ __global__ void __launch_bounds__(kBwdWarps * 32, 3) backward_lut_kernel(Backwar
                 }
                 __syncwarp();
             }
-            synthesise<NKC, kSweepCompact>(sw, w.hc, w.ha, nh, t, d, koff, a.inv_sqrt_d, w.buf);
+            if (pass == 0 && a.R)
+                RowOps<VEC>::scale_in(w.buf, a.R + tk * d, d, 1.f);  // r as the decode left it
+            else
+                synthesise<NKC, kSweepCompact>(sw, w.hc, w.ha, nh, t, d, koff, a.inv_sqrt_d, w.buf);
             if (pass == 1) break;
             // ---- dL/dr = c (g - (<g,r>/|r|^2) r) in place of r ----
             float srr = 0.f, sgr = 0.f;
@@ -409,7 +413,8 @@ bool rows_vec(int d, std::initializer_list<const void *> ptrs) {
 
 template <typename Tio, int NKC>
 cudaError_t run_backward_lut(const dpb_plan *p, const BackwardArgs &a, int64_t T, cudaStream_t stream) {
-    if (rows_vec<Tio>(p->cfg.d, {a.x, a.gy, a.gx})) return run_backward_lut<Tio, NKC, true>(p, a, T, stream);
+    if (rows_vec<Tio>(p->cfg.d, {a.x, a.gy, a.gx}) && reinterpret_cast<uintptr_t>(a.R) % 16 == 0)
+        return run_backward_lut<Tio, NKC, true>(p, a, T, stream);
     return run_backward_lut<Tio, NKC, false>(p, a, T, stream);
 }
 
@@ -423,11 +428,11 @@ cudaError_t dispatch_backward_lut(const dpb_plan *p, const BackwardArgs &a, int6
 }  // namespace
 
 cudaError_t launch_backward(const dpb_plan *p, const void *x, const int32_t *idx,
-                            const float *val, int64_t T, const float *sigma, const void *grad_y,
-                            void *grad_x, float *grad_val, int32_t *status,
+                            const float *val, int64_t T, const float *sigma, const float *r_in,
+                            const void *grad_y, void *grad_x, float *grad_val, int32_t *status,
                             cudaStream_t stream) {
     const dpb_config &c = p->cfg;
-    BackwardArgs a{x, grad_y, idx, val, sigma, grad_x, grad_val, T, status, p->dM, p->dVH2,
+    BackwardArgs a{x, grad_y, idx, val, sigma, r_in, grad_x, grad_val, T, status, p->dM, p->dVH2,
                    c.d, p->code_len, c.norm_match, p->m_mask, p->inv_sqrt_d};
     if (c.d <= 2048) {
         return c.dtype == DPB_BF16 ? dispatch_backward_lut<__nv_bfloat16>(p, a, T, stream)

@@ -193,7 +193,7 @@ dpb_status dpb_encode(const dpb_plan *plan, const void *x, int64_t T, const floa
 }
 
 dpb_status dpb_decode(const dpb_plan *plan, const int32_t *idx, const float *val, int64_t T,
-                      const float *xnorm, void *y, void *workspace, size_t workspace_bytes,
+                      const float *xnorm, void *y, float *r_out, void *workspace, size_t workspace_bytes,
                       void *stream) {
     DPB_TRY(check_plan(plan));
     if (T < 0) return dpb::fail(DPB_ERR_INVALID_ARG, "T < 0");
@@ -202,16 +202,17 @@ dpb_status dpb_decode(const dpb_plan *plan, const int32_t *idx, const float *val
     DPB_TRY(check_vec(val, "val", true));
     DPB_TRY(check_vec(xnorm, "xnorm", plan->cfg.norm_match != 0));
     DPB_TRY(check_rows(y, "y", true));
+    DPB_TRY(check_rows(r_out, "r_out", false));
     DPB_TRY(check_workspace(workspace, workspace_bytes));
     DPB_TRY(check_device(plan));
-    return launched(dpb::launch_decode(plan, idx, val, T, xnorm, y, static_cast<int32_t *>(workspace),
+    return launched(dpb::launch_decode(plan, idx, val, T, xnorm, y, r_out, static_cast<int32_t *>(workspace),
                                        static_cast<cudaStream_t>(stream)),
                     "decode");
 }
 
 dpb_status dpb_backward(const dpb_plan *plan, const void *x, const int32_t *idx,
-                        const float *val, int64_t T, const float *sigma, const void *grad_y,
-                        void *grad_x, float *grad_val, void *workspace,
+                        const float *val, int64_t T, const float *sigma, const float *r,
+                        const void *grad_y, void *grad_x, float *grad_val, void *workspace,
                         size_t workspace_bytes, void *stream) {
     DPB_TRY(check_plan(plan));
     if (T < 0) return dpb::fail(DPB_ERR_INVALID_ARG, "T < 0");
@@ -220,12 +221,13 @@ dpb_status dpb_backward(const dpb_plan *plan, const void *x, const int32_t *idx,
     DPB_TRY(check_vec(idx, "idx", true));
     DPB_TRY(check_vec(val, "val", true));
     DPB_TRY(check_vec(sigma, "sigma", false));
+    DPB_TRY(check_rows(r, "r", false));
     DPB_TRY(check_rows(grad_y, "grad_y", true));
     DPB_TRY(check_rows(grad_x, "grad_x", true));
     DPB_TRY(check_vec(grad_val, "grad_val", true));
     DPB_TRY(check_workspace(workspace, workspace_bytes));
     DPB_TRY(check_device(plan));
-    return launched(dpb::launch_backward(plan, x, idx, val, T, sigma, grad_y, grad_x, grad_val,
+    return launched(dpb::launch_backward(plan, x, idx, val, T, sigma, r, grad_y, grad_x, grad_val,
                                          static_cast<int32_t *>(workspace),
                                          static_cast<cudaStream_t>(stream)),
                     "backward");

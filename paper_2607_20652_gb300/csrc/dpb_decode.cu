@@ -19,6 +19,7 @@ struct DecodeArgs {
     const int32_t *idx;
     const float *val, *xnorm;
     void *y;
+    float *R;  // nullable: r itself, fp32 [T][d], for a later backward
     int64_t T;
     int32_t *status;
     const uint32_t *M;
@@ -73,6 +74,8 @@ __global__ void __launch_bounds__(128) decode_warp_kernel(DecodeArgs a) {
             rb[i] = r;
             ss += r * r;
         }
+        if (a.R)
+            for (int i = lane; i < d; i += 32) a.R[t * d + i] = rb[i];
         float scale = 1.f;
         if (a.norm_match) {
             ss = warp_sum(ss);
@@ -108,6 +111,7 @@ __global__ void __launch_bounds__(256) decode_lut_kernel(DecodeArgs a, int t) {
         __syncwarp();
         const int nh = split_code(a.idx + tk * a.k, a.val + tk * a.k, a.k, d, a.m_mask, r, hl, a.status);
         synthesise<NKC>(sw, hl.c, hl.a, nh, t, d, koff, a.inv_sqrt_d, r);
+        if (a.R) RowOps<VEC>::store(a.R + tk * d, r, d, 1.f);
         float scale = 1.f;
         if (a.norm_match) {
             float ss = 0.f, unused = 0.f;
@@ -143,8 +147,9 @@ cudaError_t run_decode_lut(const dpb_plan *p, const DecodeArgs &a, int64_t T, cu
 
 template <typename Tio, int NKC>
 cudaError_t run_decode_lut(const dpb_plan *p, const DecodeArgs &a, int64_t T, cudaStream_t stream) {
-    // y can be written 4 elements at a time: d % 4 == 0 and y aligned to 4 elements
-    if (p->cfg.d % 4 == 0 && reinterpret_cast<uintptr_t>(a.y) % (4 * sizeof(Tio)) == 0)
+    // y (and r) can be written 4 elements at a time: d % 4 == 0 and both aligned to 4 elements
+    if (p->cfg.d % 4 == 0 && reinterpret_cast<uintptr_t>(a.y) % (4 * sizeof(Tio)) == 0 &&
+        reinterpret_cast<uintptr_t>(a.R) % 16 == 0)
         return run_decode_lut<Tio, NKC, true>(p, a, T, stream);
     return run_decode_lut<Tio, NKC, false>(p, a, T, stream);
 }
@@ -160,9 +165,9 @@ cudaError_t dispatch_decode_lut(const dpb_plan *p, const DecodeArgs &a, int64_t 
 }  // namespace
 
 cudaError_t launch_decode(const dpb_plan *p, const int32_t *idx, const float *val, int64_t T,
-                          const float *xnorm, void *y, int32_t *status, cudaStream_t stream) {
+                          const float *xnorm, void *y, float *r_out, int32_t *status, cudaStream_t stream) {
     const dpb_config &c = p->cfg;
-    DecodeArgs a{idx, val, xnorm, y, T, status, p->dM, c.d, p->code_len, c.norm_match, p->m_mask,
+    DecodeArgs a{idx, val, xnorm, y, r_out, T, status, p->dM, c.d, p->code_len, c.norm_match, p->m_mask,
                  p->inv_sqrt_d};
     if (c.d <= 2048) {
         return c.dtype == DPB_BF16 ? dispatch_decode_lut<__nv_bfloat16>(p, a, T, stream)

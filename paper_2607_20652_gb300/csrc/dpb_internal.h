@@ -108,10 +108,10 @@ inline size_t tab_bytes(const dpb_plan *p) {
     return m <= (1ull << 26) ? (size_t)((8 * m + 255) / 256 * 256) : 0;
 }
 cudaError_t launch_decode(const dpb_plan *p, const int32_t *idx, const float *val, int64_t T,
-                          const float *xnorm, void *y, int32_t *status, cudaStream_t stream);
+                          const float *xnorm, void *y, float *r_out, int32_t *status, cudaStream_t stream);
 cudaError_t launch_backward(const dpb_plan *p, const void *x, const int32_t *idx,
-                            const float *val, int64_t T, const float *sigma, const void *grad_y,
-                            void *grad_x, float *grad_val, int32_t *status,
+                            const float *val, int64_t T, const float *sigma, const float *r_in,
+                            const void *grad_y, void *grad_x, float *grad_val, int32_t *status,
                             cudaStream_t stream);
 
 // Standardisation moments (dpb_stats.cu): whether the sampled search fits

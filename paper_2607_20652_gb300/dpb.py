@@ -89,8 +89,8 @@ def load(path: Optional[str] = None):
     lib.dpb_code_length.argtypes = [vp, ctypes.POINTER(ctypes.c_int32)]
     lib.dpb_workspace_size.argtypes = [vp, i64, ctypes.POINTER(sz)]
     lib.dpb_encode.argtypes = [vp, vp, i64, vp, vp, vp, vp, vp, vp, sz, vp]
-    lib.dpb_decode.argtypes = [vp, vp, vp, i64, vp, vp, vp, sz, vp]
-    lib.dpb_backward.argtypes = [vp, vp, vp, vp, i64, vp, vp, vp, vp, vp, sz, vp]
+    lib.dpb_decode.argtypes = [vp, vp, vp, i64, vp, vp, vp, vp, sz, vp]
+    lib.dpb_backward.argtypes = [vp, vp, vp, vp, i64, vp, vp, vp, vp, vp, vp, sz, vp]
     lib.dpb_workspace_status.argtypes = [vp, ctypes.c_int, ctypes.POINTER(ctypes.c_int32), vp]
     lib.dpb_encode_noalloc.argtypes = [vp, vp, i64, vp, vp, vp, vp, vp, vp, vp]
     lib.dpb_stats_accumulate.argtypes = [vp, vp, i64, vp, vp, vp, ctypes.c_int32, vp, vp, sz, vp]
@@ -234,8 +234,9 @@ def encode(plan: Plan, x: torch.Tensor, mu=None, sigma=None, idx=None, val=None,
 
 
 def decode(plan: Plan, idx: torch.Tensor, val: torch.Tensor, xnorm=None, y=None, workspace=None,
-           stream=None):
-    """dpb_decode. Returns y [T, d] in the plan's dtype."""
+           stream=None, r_out: Optional[torch.Tensor] = None):
+    """dpb_decode. Returns y [T, d] in the plan's dtype; with ``r_out`` (fp32
+    [T, d]) also keeps r there for dpb_backward."""
     T = idx.shape[0]
     if idx.dtype != torch.int32 or val.dtype != torch.float32 or idx.shape != val.shape \
             or not idx.is_contiguous() or not val.is_contiguous():
@@ -244,21 +245,28 @@ def decode(plan: Plan, idx: torch.Tensor, val: torch.Tensor, xnorm=None, y=None,
         raise ValueError(f"code length {idx.shape[1]} != plan's {plan.code_len}")
     y = torch.empty((T, plan.d), dtype=plan.torch_dtype, device=idx.device) if y is None else y
     ws = plan.workspace(T, idx.device) if workspace is None else workspace
-    _check(plan._lib.dpb_decode(plan.handle, _ptr(idx), _ptr(val), T, _ptr(xnorm), _ptr(y), _ptr(ws),
-                                ws.numel() * ws.element_size(), _stream(stream)))
+    if r_out is not None and (r_out.dtype != torch.float32 or not r_out.is_contiguous()
+                              or tuple(r_out.shape) != (T, plan.d)):
+        raise ValueError(f"r_out must be a contiguous float32 tensor of shape [T, {plan.d}]")
+    _check(plan._lib.dpb_decode(plan.handle, _ptr(idx), _ptr(val), T, _ptr(xnorm), _ptr(y), _ptr(r_out),
+                                _ptr(ws), ws.numel() * ws.element_size(), _stream(stream)))
     return y
 
 
 def backward(plan: Plan, x: torch.Tensor, idx: torch.Tensor, val: torch.Tensor, grad_y: torch.Tensor,
-             sigma=None, grad_x=None, grad_val=None, workspace=None, stream=None):
-    """dpb_backward. Returns (grad_x [T, d] plan dtype, grad_val fp32 [T, k])."""
+             sigma=None, grad_x=None, grad_val=None, workspace=None, stream=None,
+             r: Optional[torch.Tensor] = None):
+    """dpb_backward. Returns (grad_x [T, d] plan dtype, grad_val fp32 [T, k]);
+    ``r`` is the r_out of the decode of this code (optional)."""
     _rows(x, plan, "x")
     _rows(grad_y, plan, "grad_y")
     T = x.shape[0]
     grad_x = torch.empty_like(x) if grad_x is None else grad_x
     grad_val = torch.empty(idx.shape, dtype=torch.float32, device=x.device) if grad_val is None else grad_val
     ws = plan.workspace(T, x.device) if workspace is None else workspace
-    _check(plan._lib.dpb_backward(plan.handle, _ptr(x), _ptr(idx), _ptr(val), T, _ptr(sigma),
+    if r is not None and (r.dtype != torch.float32 or not r.is_contiguous() or tuple(r.shape) != (T, plan.d)):
+        raise ValueError(f"r must be a contiguous float32 tensor of shape [T, {plan.d}]")
+    _check(plan._lib.dpb_backward(plan.handle, _ptr(x), _ptr(idx), _ptr(val), T, _ptr(sigma), _ptr(r),
                                   _ptr(grad_y), _ptr(grad_x), _ptr(grad_val), _ptr(ws),
                                   ws.numel() * ws.element_size(), _stream(stream)))
     return grad_x, grad_val

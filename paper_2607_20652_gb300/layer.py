@@ -1,8 +1,8 @@
 """The DPB as a PyTorch layer: autograd around the C-ABI calls.
 
-Forward runs dpb_encode then dpb_decode (the code and |x| are kept for the
-backward); backward runs dpb_backward, the gradient with the selected set
-held fixed. The layer has no trainable parameters: its dictionary is the
+Forward runs dpb_encode then dpb_decode (the code and the decode's r are
+kept for the backward); backward runs dpb_backward, the gradient with the
+selected set held fixed. The layer has no trainable parameters: its dictionary is the
 parity construction (§2.1). With ``ema`` set, the layer keeps live
 standardisation tables (§2.2 "Score Standardization"): forward adds the
 batch's moment sums (level 0 over every row, levels >= 1 over a 64-row
@@ -28,27 +28,28 @@ class _DPBFunction(torch.autograd.Function):
         stream = torch.cuda.current_stream(x.device)
         ev = layer._events("forward")
         idx, val, xn = dpb.encode(layer.plan, x, layer.mu, layer.sigma, workspace=ws, stream=stream)
-        y = dpb.decode(layer.plan, idx, val, xn, workspace=ws, stream=stream)
+        r = torch.empty((T, layer.d), dtype=torch.float32, device=x.device)  # kept for the backward
+        y = dpb.decode(layer.plan, idx, val, xn, workspace=ws, stream=stream, r_out=r)
         if layer.ema is not None and layer.training:
             rows = dpb.sample_rows(T, layer.ema_rows, layer._gen, x.device)
             dpb.stats_accumulate(layer.plan, x, rows, layer._acc, mu=layer.mu, sigma=layer.sigma, workspace=ws,
                                  stream=stream)
         if ev:
             ev[1].record(stream)
-        ctx.save_for_backward(x, idx, val)
+        ctx.save_for_backward(x, idx, val, r)
         ctx.layer = layer
         layer.last_code = (idx, val)
         return y
 
     @staticmethod
     def backward(ctx, gy):
-        x, idx, val = ctx.saved_tensors
+        x, idx, val, r = ctx.saved_tensors
         layer = ctx.layer
         gy = gy.contiguous().to(x.dtype)
         ws = layer._workspace(x.shape[0], x.device)
         stream = torch.cuda.current_stream(x.device)
         ev = layer._events("backward")
-        gx, gv = dpb.backward(layer.plan, x, idx, val, gy, layer.sigma, workspace=ws, stream=stream)
+        gx, gv = dpb.backward(layer.plan, x, idx, val, gy, layer.sigma, workspace=ws, stream=stream, r=r)
         if layer.ema is not None and layer.training:
             dpb.ema_step(lambda a: None,
                          lambda a: dpb.stats_update(layer.plan, a, layer.ema, layer.mu, layer.sigma, stream=stream),

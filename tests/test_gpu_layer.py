@@ -2,8 +2,8 @@
 ParityTransformer step built from it.
 
 The layer must give exactly the C-ABI calls' outputs (same kernels): forward
-= dpb_encode + dpb_decode, the input gradient = dpb_backward with the code of
-that forward. Its live tables must move like a direct dpb_stats_* sequence.
+= dpb_encode + dpb_decode (keeping r), the input gradient = dpb_backward with
+the code and r of that forward. Its live tables must move like a direct dpb_stats_* sequence.
 A small ParityTransformer must train (the loss falls on a fixed batch) with
 finite gradients everywhere.
 """
@@ -37,8 +37,9 @@ def test_layer_is_the_c_abi_calls():
     y = layer(x)
     y.backward(gy)
     idx, val, xn = dpb.encode(layer.plan, x0)
-    y_ref = dpb.decode(layer.plan, idx, val, xn)
-    gx_ref, gv_ref = dpb.backward(layer.plan, x0, idx, val, gy.view(-1, 768).contiguous())
+    r = torch.empty((600, 768), dtype=torch.float32, device=dev)
+    y_ref = dpb.decode(layer.plan, idx, val, xn, r_out=r)
+    gx_ref, gv_ref = dpb.backward(layer.plan, x0, idx, val, gy.view(-1, 768).contiguous(), r=r)
     torch.cuda.synchronize()
     assert torch.equal(y.view(-1, 768), y_ref)
     assert torch.equal(x.grad.view(-1, 768), gx_ref)

@@ -310,3 +310,36 @@ def test_empty_batch_is_a_no_op():
     assert idx.shape == (0, 8)
     y = dpb.decode(plan, idx, val, xn)
     assert y.shape == (0, 64)
+
+
+@pytest.mark.parametrize("d,dtype", [(768, "f32"), (768, "bf16"), (2304, "f32")])
+def test_kept_r_matches_the_oracle_and_the_rebuilt_backward(d, dtype):
+    # dpb_decode's r_out is r itself (the oracle's decode without norm
+    # matching); dpb_backward given that r gives the gradients of rebuilding it
+    # (fp32 sums in another order: within fp32 rounding).
+    plan = dpb.Plan(d=d, levels=4, m_bits=16, children=16, beam=8, k=32, dtype=dtype)
+    ref = _ref(plan)
+    dev = torch.device("cuda")
+    x_np = inputs.gaussian_rows(300, d, 70)
+    x_np = inputs.to_bf16(x_np) if dtype == "bf16" else x_np
+    gy_np = inputs.normal((300, d), 71)
+    gy_np = inputs.to_bf16(gy_np) if dtype == "bf16" else gy_np
+    x = torch.from_numpy(x_np).to(dev).to(plan.torch_dtype)
+    gy = torch.from_numpy(gy_np).to(dev).to(plan.torch_dtype)
+    idx, val, xn = dpb.encode(plan, x)
+    r = torch.empty((300, d), dtype=torch.float32, device=dev)
+    y_kept = dpb.decode(plan, idx, val, xn, r_out=r)
+    y = dpb.decode(plan, idx, val, xn)
+    gx0, gv0 = dpb.backward(plan, x, idx, val, gy)
+    gx1, gv1 = dpb.backward(plan, x, idx, val, gy, r=r)
+    torch.cuda.synchronize()
+    assert torch.equal(y, y_kept)
+    r_o = oracle.decode(ref, idx.cpu().numpy(), val.cpu().numpy().astype(np.float64), norm_match=0)
+    assert parity.rel_rows(r.cpu().numpy(), r_o).max() <= 1e-5
+    tol = parity.TOL[dtype]
+    assert parity.rel_rows(gx1.float().cpu().numpy(), gx0.float().cpu().numpy()).max() <= max(tol, 1e-5)
+    assert parity.rel_rows(gv1.cpu().numpy(), gv0.cpu().numpy()).max() <= 1e-5
+    gx_o, gv_o = oracle.backward(ref, x_np.astype(np.float64), idx.cpu().numpy(),
+                                 val.cpu().numpy().astype(np.float64), gy_np.astype(np.float64))
+    assert parity.rel_rows(gx1.float().cpu().numpy(), gx_o).max() <= tol
+    assert parity.rel_rows(gv1.cpu().numpy(), gv_o).max() <= 1e-5
