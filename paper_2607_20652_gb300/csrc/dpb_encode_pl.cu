@@ -483,8 +483,11 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
             const uint32_t G0 = G;
             // the level's first nbs - 1 tiles (every earlier MMA is done, so
             // every stage is free)
+            // the first tiles: every stage with three or more (all free here),
+            // one ahead of the first chunk with two
+            const int ahead = nbs >= 3 ? nbs : nbs - 1;
             if (tid == 0)
-                for (int c = 0; c < min(nbs - 1, nch); ++c)
+                for (int c = 0; c < min(ahead, nch); ++c)
                     copy_b(stage_b(G0 + c), gt + (int64_t)c * D * 32, D, full_b(G0 + c));
             for (int c = 0; c < nch; ++c) {
                 const uint32_t g = G0 + c;
@@ -545,12 +548,19 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
                     }
                     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
                         mma_done(g)));
-                    // the tile nbs - 1 chunks ahead goes to the stage chunk g - 1
-                    // read, once its MMAs are done
-                    if (c + nbs - 1 < nch) {
+                    if (nbs >= 3) {
+                        // the tile nbs - 2 chunks ahead goes to the stage chunk g - 2
+                        // read; its MMAs were waited for at the top of this chunk,
+                        // so thread 0 goes on to the next chunk without waiting
+                        if (c >= 2 && c + nbs - 2 < nch)
+                            copy_b(stage_b(g + nbs - 2), gt + (int64_t)(c + nbs - 2) * D * 32, D,
+                                   full_b(g + nbs - 2));
+                    } else if (c + 1 < nch) {
+                        // two stages: the next tile goes to the stage chunk g - 1
+                        // read, once its MMAs are done
                         const bool ok = c == 0 || mbar_wait(mma_done(g - 1), phase(g - 1));
                         if (ok)
-                            copy_b(stage_b(g + nbs - 1), gt + (int64_t)(c + nbs - 1) * D * 32, D, full_b(g + nbs - 1));
+                            copy_b(stage_b(g + 1), gt + (int64_t)(c + 1) * D * 32, D, full_b(g + 1));
                         else
                             set_status(a.status, DPB_DEV_TIMEOUT);
                     }
