@@ -42,11 +42,13 @@ INT_LOGIC_PER_SM = 64     # LOP3 per SM per clock (measured)
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic_wide_T65536.txt")
 # files whose contents define each timed kernel (traffic figures are dropped
 # when any of them changed after the counters were taken)
+# the files holding each kernel's device code (host-side plan code does not
+# change what a launch moves)
 KERNEL_SOURCES = {
     "encode": ["dpb_encode_mma.cuh", "dpb_encode_mma.cu", "dpb_encode_mma_n2.cu", "dpb_select.cuh",
-               "dpb_device.cuh", "dpb_internal.h", "dpb_plan.cu"],
-    "decode": ["dpb_decode.cu", "dpb_lut.cuh", "dpb_device.cuh", "dpb_internal.h", "dpb_plan.cu"],
-    "backward": ["dpb_backward.cu", "dpb_lut.cuh", "dpb_device.cuh", "dpb_internal.h", "dpb_plan.cu"],
+               "dpb_device.cuh"],
+    "decode": ["dpb_decode.cu", "dpb_lut.cuh", "dpb_device.cuh"],
+    "backward": ["dpb_backward.cu", "dpb_lut.cuh", "dpb_device.cuh"],
 }
 
 
@@ -352,8 +354,16 @@ def run_ours(args, world, rank, local):
         dist.init_process_group("nccl", device_id=device)
     w = workload_cfg()
     T, d = w["T"], w["d"]
-    plan = dpb.Plan(d=d, levels=w["levels"], m_bits=w["m_bits"], children=w["children"],
-                    beam=w["beam"], k=w["k"], dtype="bf16", norm_match=1)
+    plan_kw = dict(d=d, levels=w["levels"], m_bits=w["m_bits"], children=w["children"],
+                   beam=w["beam"], k=w["k"], dtype="bf16", norm_match=1)
+    if args.coset:
+        # the variant outside the paper: coset generators g0 ^ {0..15} per level,
+        # scored by the Walsh-Hadamard path or by the contraction
+        from paper_2607_20652_gb300 import inputs
+        bits = dpb.Plan(**plan_kw).config["bits"]
+        plan_kw.update(generators=inputs.coset_generators(bits, w["levels"], seed=5),
+                       scoring=dpb.SCORING_COSET_WHT if args.coset == "wht" else dpb.SCORING_CONTRACTION)
+    plan = dpb.Plan(**plan_kw)
     seed = shard_seed(w["seed"], rank)
     x, gy, idx_true = make_inputs_gpu(w, plan, seed, device)
     k = plan.code_len
@@ -455,7 +465,9 @@ def run_ours(args, world, rank, local):
         "metric": METRIC, "value": round(value, 1), "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_max / args.steps, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-        "data": "synthetic", "config": config_block(w, world, standardise=std, keep_r=rk is not None),
+        "data": "synthetic", "config": {**config_block(w, world, standardise=std, keep_r=rk is not None),
+                                         **({"generators": "coset g0 ^ {0..15} per level (variant outside the paper)",
+                                             "scoring": args.coset} if args.coset else {})},
         "roofline": roof,
         "step_roofline": {"t_roofline_us": round(step_roof_us, 2),
                           "t_measured_us": round(1e3 * ms_max / args.steps, 2),
@@ -768,6 +780,8 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-streams", type=int, default=4, help="streams of the host-buffer run")
     ap.add_argument("--no-keep-r", action="store_true", help="backward rebuilds r instead of reading the decode's")
+    ap.add_argument("--coset", choices=["wht", "contraction"],
+                    help="coset generators g0 ^ {0..15} per level, scored by a WHT or by the contraction")
     ap.add_argument("--e2e-chunks", type=int, default=8,
                     help="chunks of the batch in the host-buffer run (copies overlap kernels across streams)")
     ap.add_argument("--standardise", action="store_true",

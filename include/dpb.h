@@ -67,6 +67,9 @@ typedef enum { DPB_F32 = 0, DPB_BF16 = 1 } dpb_dtype;
  * code is every level's kept set, level by level. */
 typedef enum { DPB_SELECT_GLOBAL = 0, DPB_SELECT_PER_LEVEL = 1 } dpb_select;
 
+/* How child scores are computed (see dpb_config.scoring). */
+typedef enum { DPB_SCORING_CONTRACTION = 0, DPB_SCORING_COSET_WHT = 1 } dpb_scoring;
+
 /* Device status bits (sticky, OR-ed by kernels into the workspace word). */
 #define DPB_DEV_BAD_INDEX 0x1   /* an idx outside [0, 2^N) was skipped        */
 #define DPB_DEV_BAD_SIGMA 0x2   /* a sigma <= 0 or non-finite was met         */
@@ -92,6 +95,14 @@ typedef enum { DPB_SELECT_GLOBAL = 0, DPB_SELECT_PER_LEVEL = 1 } dpb_select;
  *               and z^11+z^2+1 (t = 11) as in App. A.4 Eq. 24, otherwise the
  *               smallest irreducible trinomial, else pentanomial
  *   generator_seed  seed of the generator draw (splitmix64, see the plan)
+ *   scoring     DPB_SCORING_CONTRACTION: child scores by the dense
+ *               contraction of Eq. 6 (any generators). DPB_SCORING_COSET_WHT:
+ *               a variant outside the paper, for generators given by the
+ *               caller where every level's 16 generators are one coset
+ *               g0 ^ {0, ..., 15} of the span of index bits 0..3: a parent's 16
+ *               child scores are then a 16-point Walsh-Hadamard transform of
+ *               16 bucket sums of x (.) phi~_{p ^ g0} (bucket = iota mod 16).
+ *               Global selection, bf16, beam 8, d a multiple of 32 up to 1024.
  */
 typedef struct dpb_config {
     int32_t d;
@@ -108,6 +119,8 @@ typedef struct dpb_config {
     int32_t field_t;
     uint32_t field_poly;
     uint64_t generator_seed;
+    int32_t scoring;
+    int32_t reserved;             /* 0 */
 } dpb_config;
 
 typedef struct dpb_plan dpb_plan;

@@ -228,7 +228,10 @@ def resolve(d: int, m_bits: int, levels: int, children: int | Sequence[int], bea
     if generators is None:
         cfg.G = generators_table(levels, bits, children, seed)
     else:
-        cfg.G = np.ascontiguousarray(generators, dtype=np.uint32)
+        # any [levels, n] table goes into the C side's [MAX_LEVELS, GSTRIDE] rows
+        src = np.asarray(generators, dtype=np.uint32)
+        cfg.G = np.zeros((MAX_LEVELS, GSTRIDE), dtype=np.uint32)
+        cfg.G[: src.shape[0], : src.shape[1]] = src[:, :GSTRIDE]
     return cfg
 
 

@@ -98,7 +98,7 @@ dpb_status dpb_plan_create(const dpb_config *cfg, const uint32_t *generators, dp
         uint32_t **dst;
         const std::vector<uint32_t> *src;
     } ups[] = {{&p->dM, &p->M}, {&p->dG, &p->G}, {&p->dVH, &p->VH}, {&p->dFRAG, &p->FRAG}, {&p->dDD, &p->DD},
-                {&p->dGT, &p->GT},     {&p->dVH2, &p->VH2}};
+                {&p->dGT, &p->GT},     {&p->dVH2, &p->VH2}, {&p->dCOSET, &p->COSET}};
     for (const Up &u : ups) {
         if (u.src->empty()) continue;
         const size_t bytes = sizeof(uint32_t) * u.src->size();
@@ -133,6 +133,7 @@ dpb_status dpb_plan_destroy(dpb_plan *plan) {
     cudaFree(plan->dDD);
     cudaFree(plan->dGT);
     cudaFree(plan->dVH2);
+    cudaFree(plan->dCOSET);
     if (cur >= 0 && cur != plan->device) cudaSetDevice(cur);
     delete plan;
     return DPB_OK;

@@ -28,6 +28,7 @@ cudaError_t launch_encode_mma(const dpb_plan *p, const void *x, int64_t T, const
     a.mu = mu;
     a.sigma = sigma;
     a.tab = tab;
+    a.coset = c.scoring == DPB_SCORING_COSET_WHT ? p->dCOSET : nullptr;
     a.idx = idx;
     a.val = val;
     a.xnorm = xnorm;

@@ -51,6 +51,7 @@ struct Args {
     int64_t T;
     const float *mu, *sigma;
     const float2 *tab;  // packed (mu, 1 / sigma), nullable
+    const uint32_t *coset;  // coset scoring tables (nullable): per level, g0's block sign words, then S_j
     int32_t *idx;
     float *val, *xnorm;
     int32_t *status;
@@ -572,7 +573,12 @@ __device__ __forceinline__ void level0_bisect(const Args &a, const uint16_t *xh,
 
 // ---- the kernel ---------------------------------------------------------------------
 
-template <int NKC, int KPL>
+// COSET: the generators of every level are one coset g0 ^ {0..15} (a variant
+// outside the paper), and a parent's 16 child scores are the 16-point
+// Walsh-Hadamard transform of its bucket sums B_u = sum over iota = u mod 16
+// of x (.) phi~_{p ^ g0}; the shared memory of the B fragments holds the coset
+// tables instead.
+template <int NKC, int KPL, bool COSET>
 __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
     extern __shared__ __align__(16) uint32_t smem[];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
@@ -586,9 +592,13 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
     uint32_t *s_dd = s_vh + NKC * 1024;
     uint32_t *s_g = s_dd + (L - 1) * kDedupSlots * 2;
     {
-        const uint4 *src = reinterpret_cast<const uint4 *>(a.frag);
-        uint4 *dst = reinterpret_cast<uint4 *>(s_frag);
-        for (int i = threadIdx.x; i < (L - 1) * nblk * 64; i += blockDim.x) dst[i] = src[i];
+        if (COSET) {
+            for (int i = threadIdx.x; i < (L - 1) * (nblk + 16); i += blockDim.x) s_frag[i] = a.coset[i];
+        } else {
+            const uint4 *src = reinterpret_cast<const uint4 *>(a.frag);
+            uint4 *dst = reinterpret_cast<uint4 *>(s_frag);
+            for (int i = threadIdx.x; i < (L - 1) * nblk * 64; i += blockDim.x) dst[i] = src[i];
+        }
         for (int v = threadIdx.x; v < 32; v += blockDim.x) {
             uint32_t word = 0;
             for (int l = 0; l < 32; ++l) word |= (uint32_t)(__popc(l & v) & 1) << l;
@@ -664,49 +674,89 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
                 for (int m = lane >> 4; m < nblk; m += 2) sw[m * 16 + row] = parent_signs<NKC>(po, s_pq, s_vh, m);
             }
             __syncwarp();
-            float acc[2][2][2][4];  // [m & 1][chunk][n-half][reg]
+            float sc[2][4];  // [token][2 h + (r & 1)]: this lane's children 8 h + 2 q4 + (r & 1)
+            if constexpr (COSET) {
+                // lane owns coordinates iota = 32 m + lane, all in bucket lane % 16;
+                // row (token tk, slot s) adds x_tk[iota] (-1)^{sign of p_s,tk ^ g0}
+                const uint32_t *cw = s_frag + (l - 1) * (nblk + 16);
+                const int wl = ((lane & 3) << 2) | (((lane & 15) >> 3) << 1) | ((lane >> 2) & 1), hl = lane >> 4;
+                float part[16];  // [tk * 8 + s]
 #pragma unroll
-            for (int u = 0; u < 2; ++u)
+                for (int r = 0; r < 16; ++r) part[r] = 0.f;
+#pragma unroll 1
+                for (int m = 0; m < nblk; ++m) {
+                    const uint32_t gw = cw[m];
+                    const float x0 = __uint_as_float((uint32_t)xh[(m * 16 + wl) * 2 + hl] << 16);
+                    const float x1 = __uint_as_float((uint32_t)xh[(nblk * 16 + m * 16 + wl) * 2 + hl] << 16);
 #pragma unroll
-                for (int c = 0; c < 2; ++c)
+                    for (int sl = 0; sl < 8; ++sl) {
+                        const uint2 sg = sgn[m * 8 + sl];
+                        part[sl] += flip(x0, ((sg.x ^ gw) << (31 - lane)) & 0x80000000u);
+                        part[8 + sl] += flip(x1, ((sg.y ^ gw) << (31 - lane)) & 0x80000000u);
+                    }
+                }
+                uint32_t sj[4];  // S of this lane's 4 children: the WHT index that scores each
 #pragma unroll
-                    for (int h = 0; h < 2; ++h)
+                for (int e = 0; e < 4; ++e) sj[e] = cw[nblk + 8 * (e >> 1) + 2 * q4 + (e & 1)];
 #pragma unroll
-                        for (int r = 0; r < 4; ++r) acc[u][c][h][r] = 0.f;
-            const uint4 *xa = reinterpret_cast<const uint4 *>(xt) + q4;
-            const uint4 *xb = reinterpret_cast<const uint4 *>(xt + nblk * 16) + q4;
-            const uint4 *fr = reinterpret_cast<const uint4 *>(frag) + lane * 2;
-            const int sh = 15 - q4;
+                for (int r = 0; r < 16; ++r) {
+                    float v = part[r] + __shfl_xor_sync(kFull, part[r], 16);  // bucket lane % 16
+#pragma unroll
+                    for (int b = 1; b < 16; b <<= 1) {
+                        const float o = __shfl_xor_sync(kFull, v, b);
+                        v = (lane & b) ? o - v : v + o;
+                    }
+                    // lane u now holds the score of child S = u of row r
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const float got = __shfl_sync(kFull, v, (int)sj[e]) * a.inv_sqrt_d;
+                        if ((r & 7) == slot) sc[r >> 3][e] = got;
+                    }
+                }
+            } else {
+                float acc[2][2][2][4];  // [m & 1][chunk][n-half][reg]
+#pragma unroll
+                for (int u = 0; u < 2; ++u)
+#pragma unroll
+                    for (int c = 0; c < 2; ++c)
+#pragma unroll
+                        for (int h = 0; h < 2; ++h)
+#pragma unroll
+                            for (int r = 0; r < 4; ++r) acc[u][c][h][r] = 0.f;
+                const uint4 *xa = reinterpret_cast<const uint4 *>(xt) + q4;
+                const uint4 *xb = reinterpret_cast<const uint4 *>(xt + nblk * 16) + q4;
+                const uint4 *fr = reinterpret_cast<const uint4 *>(frag) + lane * 2;
+                const int sh = 15 - q4;
 #pragma unroll 2
-            for (int m = 0; m < nblk; ++m) {
-                const uint4 va = xa[m * 4], vb = xb[m * 4];
-                const uint2 sg = sgn[m * 8 + slot];
-                const uint32_t s0 = sg.x, s1 = sg.y;
-                const uint4 f0 = fr[m * 64], f1 = fr[m * 64 + 1];
-                // chunk 0 holds pairs 0 and 1 of the block, chunk 1 pairs 2 and 3
-                const uint32_t a00 = va.x ^ ((s0 << sh) & 0x80008000u);
-                const uint32_t a01 = vb.x ^ ((s1 << sh) & 0x80008000u);
-                const uint32_t a02 = va.y ^ ((s0 << (sh - 4)) & 0x80008000u);
-                const uint32_t a03 = vb.y ^ ((s1 << (sh - 4)) & 0x80008000u);
-                const uint32_t a10 = va.z ^ ((s0 << (sh - 8)) & 0x80008000u);
-                const uint32_t a11 = vb.z ^ ((s1 << (sh - 8)) & 0x80008000u);
-                const uint32_t a12 = va.w ^ ((s0 << (sh - 12)) & 0x80008000u);
-                const uint32_t a13 = vb.w ^ ((s1 << (sh - 12)) & 0x80008000u);
-                float(&cc)[2][2][4] = acc[m & 1];
-                mma_bf16(cc[0][0], a00, a01, a02, a03, f0.x, f0.y);
-                mma_bf16(cc[0][1], a00, a01, a02, a03, f0.z, f0.w);
-                mma_bf16(cc[1][0], a10, a11, a12, a13, f1.x, f1.y);
-                mma_bf16(cc[1][1], a10, a11, a12, a13, f1.z, f1.w);
+                for (int m = 0; m < nblk; ++m) {
+                    const uint4 va = xa[m * 4], vb = xb[m * 4];
+                    const uint2 sg = sgn[m * 8 + slot];
+                    const uint32_t s0 = sg.x, s1 = sg.y;
+                    const uint4 f0 = fr[m * 64], f1 = fr[m * 64 + 1];
+                    // chunk 0 holds pairs 0 and 1 of the block, chunk 1 pairs 2 and 3
+                    const uint32_t a00 = va.x ^ ((s0 << sh) & 0x80008000u);
+                    const uint32_t a01 = vb.x ^ ((s1 << sh) & 0x80008000u);
+                    const uint32_t a02 = va.y ^ ((s0 << (sh - 4)) & 0x80008000u);
+                    const uint32_t a03 = vb.y ^ ((s1 << (sh - 4)) & 0x80008000u);
+                    const uint32_t a10 = va.z ^ ((s0 << (sh - 8)) & 0x80008000u);
+                    const uint32_t a11 = vb.z ^ ((s1 << (sh - 8)) & 0x80008000u);
+                    const uint32_t a12 = va.w ^ ((s0 << (sh - 12)) & 0x80008000u);
+                    const uint32_t a13 = vb.w ^ ((s1 << (sh - 12)) & 0x80008000u);
+                    float(&cc)[2][2][4] = acc[m & 1];
+                    mma_bf16(cc[0][0], a00, a01, a02, a03, f0.x, f0.y);
+                    mma_bf16(cc[0][1], a00, a01, a02, a03, f0.z, f0.w);
+                    mma_bf16(cc[1][0], a10, a11, a12, a13, f1.x, f1.y);
+                    mma_bf16(cc[1][1], a10, a11, a12, a13, f1.z, f1.w);
+                }
+                // accumulator (n-half h, register r): row slot (r < 2) or slot + 8
+                // (r >= 2), child 8 h + 2 q4 + (r & 1)
+#pragma unroll
+                for (int h = 0; h < 2; ++h)
+#pragma unroll
+                    for (int r = 0; r < 4; ++r)
+                        sc[r >> 1][2 * h + (r & 1)] =
+                            ((acc[0][0][h][r] + acc[0][1][h][r]) + (acc[1][0][h][r] + acc[1][1][h][r])) * a.inv_sqrt_d;
             }
-            // accumulator (n-half h, register r): row slot (r < 2) or slot + 8
-            // (r >= 2), child 8 h + 2 q4 + (r & 1)
-            float sc[2][4];  // [token][2 h + (r & 1)]
-#pragma unroll
-            for (int h = 0; h < 2; ++h)
-#pragma unroll
-                for (int r = 0; r < 4; ++r)
-                    sc[r >> 1][2 * h + (r & 1)] =
-                        ((acc[0][0][h][r] + acc[0][1][h][r]) + (acc[1][0][h][r] + acc[1][1][h][r])) * a.inv_sqrt_d;
             const uint32_t *gl = s_g + l * 16;
             const uint32_t *ddl = s_dd + (l - 1) * kDedupSlots * 2;
             uint32_t pcur = p0;
@@ -792,26 +842,32 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
     }
 }
 
-template <int NKC, int KPL>
+template <int NKC, int KPL, bool COSET>
 cudaError_t launch_kpl(const dpb_plan *p, const Args &a, int warps, cudaStream_t stream) {
     const size_t smem = encode_mma_smem(p, warps);
     const cudaError_t e =
-        cudaFuncSetAttribute(encode_kernel<NKC, KPL>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        cudaFuncSetAttribute(encode_kernel<NKC, KPL, COSET>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     int sms = 0;
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, p->device);
     const int64_t pairs = (a.T + 1) / 2;
     const int grid = (int)std::min<int64_t>((pairs + warps - 1) / warps, (int64_t)std::max(sms, 1));
-    encode_kernel<NKC, KPL><<<grid, warps * 32, smem, stream>>>(a);
+    encode_kernel<NKC, KPL, COSET><<<grid, warps * 32, smem, stream>>>(a);
     return cudaGetLastError();
 }
 
 template <int NKC>
 cudaError_t launch_nkc(const dpb_plan *p, const Args &a, int warps, cudaStream_t stream) {
-    if (a.k <= 32) return launch_kpl<NKC, 1>(p, a, warps, stream);
-    if (a.k <= 64) return launch_kpl<NKC, 2>(p, a, warps, stream);
-    if (a.k <= 128) return launch_kpl<NKC, 4>(p, a, warps, stream);
-    return launch_kpl<NKC, 8>(p, a, warps, stream);
+    if (a.coset) {
+        if (a.k <= 32) return launch_kpl<NKC, 1, true>(p, a, warps, stream);
+        if (a.k <= 64) return launch_kpl<NKC, 2, true>(p, a, warps, stream);
+        if (a.k <= 128) return launch_kpl<NKC, 4, true>(p, a, warps, stream);
+        return launch_kpl<NKC, 8, true>(p, a, warps, stream);
+    }
+    if (a.k <= 32) return launch_kpl<NKC, 1, false>(p, a, warps, stream);
+    if (a.k <= 64) return launch_kpl<NKC, 2, false>(p, a, warps, stream);
+    if (a.k <= 128) return launch_kpl<NKC, 4, false>(p, a, warps, stream);
+    return launch_kpl<NKC, 8, false>(p, a, warps, stream);
 }
 
 // One per table count, each in its own translation unit.

@@ -51,6 +51,12 @@ struct dpb_plan {
     uint32_t *dDD = nullptr;    // device copy of DD
     uint32_t *dGT = nullptr;    // device copy of GT
     uint32_t *dVH2 = nullptr;   // device copy of VH2
+    // Coset-generator scoring (DPB_SCORING_COSET_WHT), per level l >= 1:
+    //  COSET[(l-1) * (nblk + 16) + m] = sign word of g0 over 32-coordinate
+    //  block m (bit i = parity(M[32 m + i] AND g0)), then 16 words S_j with
+    //  g_j = g0 ^ S_j (S_j in 0..15).
+    std::vector<uint32_t> COSET;
+    uint32_t *dCOSET = nullptr;
 };
 
 namespace dpb {

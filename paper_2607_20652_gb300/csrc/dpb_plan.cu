@@ -332,6 +332,32 @@ dpb_status resolve_and_build(const dpb_config *in, const uint32_t *generators, d
     }
     p->cfg = c;
     build_mma_tables(p);
+    if (c.scoring == DPB_SCORING_COSET_WHT) {
+        // the variant outside the paper: every level's 16 generators one coset
+        // g0 ^ {0..15} (given by the caller), scored by a 16-point WHT
+        if (!generators) return fail(DPB_ERR_INVALID_ARG, "coset scoring needs the caller's generators");
+        if (!p->mma_encode)
+            return fail(DPB_ERR_UNSUPPORTED,
+                        "coset scoring needs global selection, bf16, beam 8, 16 children, d a multiple of 32 up to 1024");
+        const int nblk = c.d / 32;
+        p->COSET.assign((size_t)(c.levels - 1) * (nblk + 16), 0u);
+        for (int l = 1; l < c.levels; ++l) {
+            const uint32_t *g = &p->G[(size_t)l * DPB_MAX_CHILDREN];
+            uint32_t *row = &p->COSET[(size_t)(l - 1) * (nblk + 16)];
+            for (int j = 0; j < 16; ++j) {
+                if ((g[j] ^ g[0]) > 15u)
+                    return fail(DPB_ERR_INVALID_ARG, "level %d: generator %u is not in the coset of %u", l, g[j], g[0]);
+                row[nblk + j] = g[j] ^ g[0];
+            }
+            for (int m = 0; m < nblk; ++m) {
+                uint32_t w = 0;
+                for (int i = 0; i < 32; ++i) w |= (uint32_t)(__builtin_popcount(p->M[32 * m + i] & g[0]) & 1) << i;
+                row[m] = w;
+            }
+        }
+    } else if (c.scoring != DPB_SCORING_CONTRACTION) {
+        return fail(DPB_ERR_INVALID_ARG, "scoring=%d unknown", c.scoring);
+    }
     if (c.select_mode == DPB_SELECT_PER_LEVEL) build_per_level_tables(p);
     p->t = c.field_t;
     p->poly = c.field_poly;

@@ -20,6 +20,7 @@ MAX_LEVELS = 8
 MAX_CHILDREN = 256
 F32, BF16 = 0, 1
 SELECT_GLOBAL, SELECT_PER_LEVEL = 0, 1
+SCORING_CONTRACTION, SCORING_COSET_WHT = 0, 1
 DEV_BAD_INDEX, DEV_BAD_SIGMA, DEV_SHORT_CODE = 0x1, 0x2, 0x4
 
 _STATUS = {0: "ok", 1: "invalid argument", 2: "unsupported configuration", 3: "CUDA error",
@@ -48,6 +49,8 @@ class Config(ctypes.Structure):
         ("field_t", ctypes.c_int32),
         ("field_poly", ctypes.c_uint32),
         ("generator_seed", ctypes.c_uint64),
+        ("scoring", ctypes.c_int32),
+        ("reserved", ctypes.c_int32),
     ]
 
     def as_dict(self) -> dict:
@@ -56,7 +59,7 @@ class Config(ctypes.Structure):
                 "children": list(self.children[:L]), "beam": self.beam, "k": self.k,
                 "k_per_level": list(self.k_per_level[:L]), "select_mode": self.select_mode,
                 "norm_match": self.norm_match, "dtype": self.dtype, "field_t": self.field_t,
-                "field_poly": self.field_poly, "generator_seed": self.generator_seed}
+                "field_poly": self.field_poly, "generator_seed": self.generator_seed, "scoring": self.scoring}
 
 
 _lib = None
@@ -137,7 +140,8 @@ class Plan:
                  beam: int = 8, k: int = 64, dtype: str = "bf16", norm_match: int = 1,
                  seed: int = 0, field_t: int = 0, field_poly: int = 0,
                  bits: Optional[Sequence[int]] = None, generators=None,
-                 select_mode: int = SELECT_GLOBAL, k_per_level: Optional[Sequence[int]] = None):
+                 select_mode: int = SELECT_GLOBAL, k_per_level: Optional[Sequence[int]] = None,
+                 scoring: int = SCORING_CONTRACTION):
         lib = load()
         c = Config()
         c.d, c.levels, c.m_bits = d, levels, m_bits
@@ -155,6 +159,7 @@ class Plan:
         c.select_mode, c.norm_match = select_mode, norm_match
         c.dtype = _DTYPES[dtype][0]
         c.field_t, c.field_poly, c.generator_seed = field_t, field_poly, seed & (2**64 - 1)
+        c.scoring = scoring
         gen_buf = None
         if generators is not None:
             import numpy as np

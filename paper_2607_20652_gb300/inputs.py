@@ -61,6 +61,21 @@ def sample_rows(T: int, n: int, seed: int) -> np.ndarray:
     return rng(seed).permutation(T)[: min(n, T)].astype(np.int32)
 
 
+def coset_generators(bits, levels: int, seed: int, max_children: int = 256) -> np.ndarray:
+    """Generator table [8, max_children] uint32 where level l >= 1 holds one
+    coset g0 ^ {0, ..., 15}: g0 drawn uniformly from [2^{r_{l-1}}, 2^{r_l})
+    with its low 4 bits cleared, g_j = g0 | j (every g_j keeps g0's level bit)."""
+    g = rng(seed)
+    out = np.zeros((8, max_children), dtype=np.uint32)
+    for l in range(1, levels):
+        lo, hi = 1 << bits[l - 1], 1 << bits[l]
+        g0 = int(g.integers(lo, hi)) & ~15
+        if g0 < lo:
+            g0 = lo
+        out[l, :16] = [g0 | j for j in range(16)]
+    return out
+
+
 def moment_tables(m: int, seed: int, mean_scale: float = 0.2, sigma_range=(0.5, 2.0)):
     """Standardisation tables (mu, sigma) fp32 [m]: mu ~ N(0, mean_scale^2),
     sigma uniform in sigma_range."""

@@ -166,3 +166,28 @@ def test_workspace_holds_the_packed_tables(lib):
     for m_bits in (12, 20):
         plan = dpb.Plan(d=64, levels=3, m_bits=m_bits, children=16, beam=4, k=8, dtype="f32")
         assert plan.workspace_size(1) == 256 + 8 * (1 << m_bits)
+
+
+def test_coset_scoring_is_checked(lib):
+    # DPB_SCORING_COSET_WHT: every level's 16 generators one coset g0 ^ {0..15},
+    # given by the caller, on the tensor-core layout (bf16, beam 8, 16 children)
+    from paper_2607_20652_gb300 import inputs
+    bits = [10, 12, 15, 17, 20]
+    G = inputs.coset_generators(bits, 5, seed=3)
+    kw = dict(d=768, levels=5, bits=bits, children=16, beam=8, k=64, dtype="bf16",
+              scoring=dpb.SCORING_COSET_WHT)
+    plan = dpb.Plan(generators=G, **kw)
+    assert plan.config["scoring"] == dpb.SCORING_COSET_WHT
+    _, Gp = plan.tables()
+    assert np.array_equal(Gp[1:5, :16], G[1:5, :16])
+    with pytest.raises(dpb.DPBError) as e:
+        dpb.Plan(**kw)                                        # the plan's own random generators
+    assert e.value.status == 1
+    bad = G.copy()
+    bad[2, 5] ^= 1 << 13                                      # not in the coset of g0
+    with pytest.raises(dpb.DPBError) as e:
+        dpb.Plan(generators=bad, **kw)
+    assert e.value.status == 1
+    with pytest.raises(dpb.DPBError) as e:
+        dpb.Plan(generators=G, **dict(kw, dtype="f32"))       # outside the tensor-core layout
+    assert e.value.status == 2

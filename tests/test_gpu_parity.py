@@ -343,3 +343,30 @@ def test_kept_r_matches_the_oracle_and_the_rebuilt_backward(d, dtype):
                                  val.cpu().numpy().astype(np.float64), gy_np.astype(np.float64))
     assert parity.rel_rows(gx1.float().cpu().numpy(), gx_o).max() <= tol
     assert parity.rel_rows(gv1.cpu().numpy(), gv_o).max() <= 1e-5
+
+
+@pytest.mark.parametrize("T", [300, 4099])
+def test_coset_scoring_matches_the_oracle(T):
+    # The coset-generator variant (outside the paper): the 16 child scores of
+    # a parent by a warp-shuffle Walsh-Hadamard transform of bucket sums. Same
+    # generators through the contraction path as a second check.
+    bits = [10, 12, 15, 17, 20]
+    G = inputs.coset_generators(bits, 5, seed=9)
+    kw = dict(d=768, levels=5, bits=bits, children=16, beam=8, k=64, dtype="bf16", generators=G)
+    wht = dpb.Plan(scoring=dpb.SCORING_COSET_WHT, **kw)
+    mma = dpb.Plan(**kw)
+    c = wht.config
+    ref = oracle.resolve(d=768, m_bits=20, levels=5, children=16, beam=8, k=64, bits=bits, generators=G,
+                         t=c["field_t"], poly=c["field_poly"], norm_match=c["norm_match"])
+    x = inputs.to_bf16(inputs.gaussian_rows(T, 768, 80))
+    rows = np.arange(T) if T <= 300 else inputs.sample_rows(T, 160, 81)
+    idx_o, val_o, xn_o, gap = oracle.encode(ref, x[rows].astype(np.float64))
+    reports = []
+    for plan in (wht, mma):
+        g = _gpu(plan, x)
+        assert g["status"] == 0
+        parity.check_code_order(g["idx"][rows], g["val"][rows])
+        near, worst = parity.compare_codes(g["idx"][rows], g["val"][rows], idx_o, val_o, gap, xn_o)
+        assert near <= max(2, len(rows) // 10)
+        reports.append((near, worst))
+    print(reports)

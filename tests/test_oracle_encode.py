@@ -143,3 +143,22 @@ def test_per_level_mode_levels():
         top1 = sorted(kids, key=lambda c: (-abs(s[c]), c))[:6]
         assert idx[t, 4:].tolist() == top1
         assert np.allclose(val[t, 4:], [s[c] for c in top1])
+
+
+def test_coset_children_scores_are_a_walsh_transform():
+    # The coset-generator variant (outside the paper): with g_j = g0 ^ j for
+    # j < 16, the 16 child scores of a parent p are the 16-point Walsh-
+    # Hadamard transform (scipy's Sylvester matrix) of the bucket sums
+    # B_u = sum over iota = u mod 16 of phi~_{p ^ g0}[iota] x[iota].
+    import scipy.linalg
+    cfg = _tiny()
+    rng = np.random.default_rng(8)
+    H = scipy.linalg.hadamard(16)
+    for _ in range(5):
+        g0 = int(rng.integers(1 << 6, 1 << 9)) & ~15
+        p = int(rng.integers(0, 1 << 6))
+        x = rng.standard_normal(cfg.d)
+        y = oracle.phi_tilde(cfg.d, cfg.M, p ^ g0) * x
+        B = np.array([y[u::16].sum() for u in range(16)])
+        s = np.array([oracle.phi(cfg.d, cfg.M, p ^ g0 ^ j) @ x for j in range(16)])
+        assert np.allclose(H @ B, s, atol=1e-12)
