@@ -631,7 +631,7 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
         for (int tk = 0; tk < ntok; ++tk) {
             const uint4 *row = reinterpret_cast<const uint4 *>(a.x + (t0 + tk) * d);
             float ss = 0.f;
-#pragma unroll 1
+#pragma unroll 3  // the row's loads in flight together (3 chunks per lane at d = 768)
             for (int ch = lane; ch < nch; ch += 32) {
                 const uint4 v = row[ch];
                 const int m = ch >> 2, l0 = (ch & 3) * 8, half = l0 >> 4, pb = (l0 & 15) >> 2;

@@ -215,6 +215,28 @@ class Plan:
         n = self.workspace_size(T)
         return torch.zeros(n, dtype=torch.uint8, device=device or "cuda")
 
+    def _stream_workspace(self, T: int, device, stream) -> torch.Tensor:
+        """The workspace of calls made without one: one per (device, stream),
+        kept with the plan (calls on one stream run in order, so they may
+        share it; its status bits accumulate until read and cleared)."""
+        dev = torch.device(device)
+        s = stream if stream is not None else torch.cuda.current_stream(dev)
+        key = (dev.index if dev.index is not None else torch.cuda.current_device(), s.cuda_stream)
+        cache = self.__dict__.setdefault("_ws_cache", {})
+        ws = cache.get(key)
+        if ws is None or ws.numel() < self.workspace_size(T):
+            ws = cache[key] = self.workspace(T, dev)
+        return ws
+
+    def status(self, device=None, stream=None, clear: bool = True) -> int:
+        """The DPB_DEV_* bits that calls made without a workspace left on
+        ``stream`` (synchronises it); cleared by default."""
+        dev = torch.device(device or "cuda")
+        s = stream if stream is not None else torch.cuda.current_stream(dev)
+        key = (dev.index if dev.index is not None else torch.cuda.current_device(), s.cuda_stream)
+        ws = self.__dict__.get("_ws_cache", {}).get(key)
+        return 0 if ws is None else workspace_status(ws, clear=clear, stream=s)
+
 
 def _rows(t: torch.Tensor, plan: Plan, name: str):
     if t.dtype != plan.torch_dtype or not t.is_cuda or not t.is_contiguous() or t.dim() != 2 \
@@ -232,7 +254,7 @@ def encode(plan: Plan, x: torch.Tensor, mu=None, sigma=None, idx=None, val=None,
     val = torch.empty((T, k), dtype=torch.float32, device=dev) if val is None else val
     if xnorm is None and want_xnorm:
         xnorm = torch.empty((T,), dtype=torch.float32, device=dev)
-    ws = plan.workspace(T, dev) if workspace is None else workspace
+    ws = plan._stream_workspace(T, dev, stream) if workspace is None else workspace
     _check(plan._lib.dpb_encode(plan.handle, _ptr(x), T, _ptr(mu), _ptr(sigma), _ptr(idx), _ptr(val),
                                 _ptr(xnorm), _ptr(ws), ws.numel() * ws.element_size(), _stream(stream)))
     return idx, val, xnorm
@@ -249,7 +271,7 @@ def decode(plan: Plan, idx: torch.Tensor, val: torch.Tensor, xnorm=None, y=None,
     if idx.shape[1] != plan.code_len:
         raise ValueError(f"code length {idx.shape[1]} != plan's {plan.code_len}")
     y = torch.empty((T, plan.d), dtype=plan.torch_dtype, device=idx.device) if y is None else y
-    ws = plan.workspace(T, idx.device) if workspace is None else workspace
+    ws = plan._stream_workspace(T, idx.device, stream) if workspace is None else workspace
     if r_out is not None and (r_out.dtype != torch.float32 or not r_out.is_contiguous()
                               or tuple(r_out.shape) != (T, plan.d)):
         raise ValueError(f"r_out must be a contiguous float32 tensor of shape [T, {plan.d}]")
@@ -268,7 +290,7 @@ def backward(plan: Plan, x: torch.Tensor, idx: torch.Tensor, val: torch.Tensor, 
     T = x.shape[0]
     grad_x = torch.empty_like(x) if grad_x is None else grad_x
     grad_val = torch.empty(idx.shape, dtype=torch.float32, device=x.device) if grad_val is None else grad_val
-    ws = plan.workspace(T, x.device) if workspace is None else workspace
+    ws = plan._stream_workspace(T, x.device, stream) if workspace is None else workspace
     if r is not None and (r.dtype != torch.float32 or not r.is_contiguous() or tuple(r.shape) != (T, plan.d)):
         raise ValueError(f"r must be a contiguous float32 tensor of shape [T, {plan.d}]")
     _check(plan._lib.dpb_backward(plan.handle, _ptr(x), _ptr(idx), _ptr(val), T, _ptr(sigma), _ptr(r),
@@ -292,7 +314,7 @@ def stats_accumulate(plan: Plan, x: torch.Tensor, sample: torch.Tensor, acc: tor
     if acc.dtype != torch.float64 or not acc.is_contiguous() or acc.numel() != 3 * plan.n_features:
         raise ValueError("acc must be a contiguous float64 tensor of 3 * 2^N entries (stats_buffer)")
     T = x.shape[0]
-    ws = plan.workspace(T, x.device) if workspace is None else workspace
+    ws = plan._stream_workspace(T, x.device, stream) if workspace is None else workspace
     _check(plan._lib.dpb_stats_accumulate(plan.handle, _ptr(x), T, _ptr(mu), _ptr(sigma),
                                           _ptr(sample) if sample.numel() else None, sample.numel(),
                                           _ptr(acc), _ptr(ws), ws.numel() * ws.element_size(),

@@ -370,3 +370,15 @@ def test_coset_scoring_matches_the_oracle(T):
         assert near <= max(2, len(rows) // 10)
         reports.append((near, worst))
     print(reports)
+
+
+def test_calls_without_a_workspace_share_one_per_stream():
+    plan = dpb.Plan(d=64, levels=3, m_bits=12, children=16, beam=4, k=8, dtype="f32")
+    dev = torch.device("cuda")
+    x = torch.from_numpy(inputs.gaussian_rows(40, 64, 90)).to(dev)
+    idx, val, xn = dpb.encode(plan, x)
+    bad = idx.clone()
+    bad[3, 2] = 1 << 12                                  # outside [0, 2^N): flagged, skipped
+    dpb.decode(plan, bad, val, xn)
+    assert len(plan._ws_cache) == 1
+    assert plan.status() == dpb.DEV_BAD_INDEX and plan.status() == 0
