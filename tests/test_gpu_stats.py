@@ -246,3 +246,40 @@ def test_packed_tables_give_the_same_codes(layout):
     torch.cuda.synchronize()
     assert torch.equal(a[0], b[0]) and torch.equal(a[1], b[1])
     assert dpb.workspace_status(full) == 0 and dpb.workspace_status(small) == 0
+
+
+def test_bad_sigma_is_flagged_not_faulted():
+    # sigma <= 0 (or not finite) for a feature that is used: every path sets
+    # DPB_DEV_BAD_SIGMA and carries on
+    dev = torch.device("cuda")
+    x = torch.from_numpy(inputs.to_bf16(inputs.gaussian_rows(64, 768, 95))).to(dev).to(torch.bfloat16)
+    plan = dpb.Plan(d=768, levels=5, m_bits=20, children=16, beam=8, k=64, dtype="bf16")
+    mu = torch.zeros(plan.n_features, device=dev)
+    for bad in (0.0, -1.0, float("inf")):
+        sg = torch.ones(plan.n_features, device=dev)
+        sg[5] = bad                                            # a basis coordinate: every token reads it
+        for ws in (plan.workspace(64, dev), torch.zeros(256, dtype=torch.uint8, device=dev)):
+            idx, val, xn = dpb.encode(plan, x, mu, sg, workspace=ws)
+            assert dpb.workspace_status(ws) & dpb.DEV_BAD_SIGMA
+        ws = plan.workspace(64, dev)
+        acc = dpb.stats_buffer(plan, dev)
+        dpb.stats_accumulate(plan, x, torch.arange(8, dtype=torch.int32, device=dev), acc, mu=mu, sigma=sg,
+                             workspace=ws)
+        assert dpb.workspace_status(ws) & dpb.DEV_BAD_SIGMA
+    # the backward divides grad_val by sigma of each code entry
+    idx, val, xn = dpb.encode(plan, x)
+    sg = torch.ones(plan.n_features, device=dev)
+    sg[idx[0, 0].long()] = 0.0
+    ws = plan.workspace(64, dev)
+    gy = torch.ones_like(x)
+    dpb.backward(plan, x, idx, val, gy, sg, workspace=ws)
+    assert dpb.workspace_status(ws) & dpb.DEV_BAD_SIGMA
+    # per-level layout
+    pl = dpb.Plan(d=64, levels=3, bits=[6, 9, 12], children=[0, 16, 32], dtype="bf16",
+                  select_mode=dpb.SELECT_PER_LEVEL, k_per_level=[4, 8, 8])
+    x2 = torch.from_numpy(inputs.to_bf16(inputs.gaussian_rows(16, 64, 96))).to(dev).to(torch.bfloat16)
+    sg2 = torch.ones(pl.n_features, device=dev)
+    sg2[3] = -2.0
+    ws = pl.workspace(16, dev)
+    dpb.encode(pl, x2, torch.zeros(pl.n_features, device=dev), sg2, workspace=ws)
+    assert dpb.workspace_status(ws) & dpb.DEV_BAD_SIGMA
