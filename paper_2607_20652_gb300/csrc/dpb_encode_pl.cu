@@ -314,9 +314,21 @@ __device__ __forceinline__ int select_level(Scan scan, int nlive, int K, const W
             if (drank[r] == target) mine = top[r];
         uint32_t tau = __reduce_max_sync(kFull, mine);
         if (tau == 0u) tau = 1u;
-        int cnt = 0;
-        scan([&](float z, uint32_t, bool live) { cnt += live && akey(z) + 1u >= tau; });
-        int n = __reduce_add_sync(kFull, cnt);
+        // gather every candidate at or above tau, warp-interleaved in scan
+        // order (one pass: positions come from the running ballot counts)
+        int n = 0;
+        scan([&](float z, uint32_t ci, bool live) {
+            const bool take = live && akey(z) + 1u >= tau;
+            const unsigned mb = __ballot_sync(kFull, take);
+            if (mb) {  // rare: most candidates fall short of tau
+                const int pos = n + __popc(mb & ((1u << lane) - 1u));
+                if (take && pos < kSelCap) {
+                    w.z[pos] = z;
+                    w.id[pos] = ci;
+                }
+                n += __popc(mb);
+            }
+        });
         if (n > kSelCap) {
             if (attempt == 0 && target > K) {
                 target = min(K, nd);
@@ -325,23 +337,6 @@ __device__ __forceinline__ int select_level(Scan scan, int nlive, int K, const W
             set_status(a.status, DPB_DEV_SHORT_CODE);
             n = kSelCap;
         }
-        int off = cnt;  // exclusive prefix over the lanes
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int t = __shfl_up_sync(kFull, off, o);
-            if (lane >= o) off += t;
-        }
-        off -= cnt;
-        scan([&](float z, uint32_t ci, bool live) {
-            const bool take = live && akey(z) + 1u >= tau;
-            if (__any_sync(kFull, take)) {  // rare: most candidates fall short of tau
-                if (take && off < kSelCap) {
-                    w.z[off] = z;
-                    w.id[off] = ci;
-                }
-                off += take;
-            }
-        });
         __syncwarp();
         distinct = n <= 128 ? sort_keep<4>(n, K, w, a, tok, col, par_out, true)
                             : sort_keep<8>(n, K, w, a, tok, col, par_out, true);
