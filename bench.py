@@ -675,6 +675,84 @@ def run_per_level(args, world, rank, local):
 
 
 # ---------------------------------------------------------------------------
+# the sweep at d = 768, T = 32768: tokens/s and roofline fraction per point
+# ---------------------------------------------------------------------------
+
+def run_sweep(args, world, rank, local):
+    import torch
+    from paper_2607_20652_gb300 import configs, dpb
+
+    device = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(device)
+    stream = torch.cuda.current_stream(device)
+    peaks, src = load_peaks()
+    points = []
+    steps = max(3, args.steps // 4)
+    for w in configs.SWEEP:
+        T, d = w["T"], w["d"]
+        plan = dpb.Plan(d=d, levels=w["levels"], m_bits=w["m_bits"], children=w["children"], beam=w["beam"],
+                        k=w["k"], dtype="bf16")
+        g = torch.Generator(device=device).manual_seed(shard_seed(w["seed"], rank) + w["m_bits"] * 100 + w["k"])
+        x = torch.randn((T, d), generator=g, device=device).to(torch.bfloat16)
+        gy = torch.randn((T, d), generator=g, device=device).to(torch.bfloat16)
+        k = plan.code_len
+        idx = torch.empty((T, k), dtype=torch.int32, device=device)
+        val = torch.empty((T, k), dtype=torch.float32, device=device)
+        xn = torch.empty((T,), dtype=torch.float32, device=device)
+        y, gx = torch.empty_like(x), torch.empty_like(x)
+        gv = torch.empty((T, k), dtype=torch.float32, device=device)
+        rk = torch.empty((T, d), dtype=torch.float32, device=device)
+        ws = plan.workspace(T, device)
+
+        def step(ev=None):
+            if ev:
+                ev[0].record(stream)
+            dpb.encode(plan, x, idx=idx, val=val, xnorm=xn, workspace=ws, stream=stream)
+            if ev:
+                ev[1].record(stream)
+            dpb.decode(plan, idx, val, xn, y=y, workspace=ws, stream=stream, r_out=rk)
+            if ev:
+                ev[2].record(stream)
+            dpb.backward(plan, x, idx, val, gy, grad_x=gx, grad_val=gv, workspace=ws, stream=stream, r=rk)
+            if ev:
+                ev[3].record(stream)
+
+        for _ in range(2):
+            step()
+        torch.cuda.synchronize(device)
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(steps)]
+        barrier(world)
+        for e in evs:
+            step(e)
+        torch.cuda.synchronize(device)
+        kern = {n: statistics.mean(e[j].elapsed_time(e[j + 1]) for e in evs)
+                for j, n in enumerate(("encode", "decode", "backward"))}
+        ms = max_over_ranks(sum(kern.values()), world, device)
+        k_hash = float(np.mean(np.sum(idx.cpu().numpy() >= d, axis=1)))
+        work = algorithmic_work(plan.config, T, k_hash, 2)
+        roofs = {n: roofline_for(n, work[n], kern[n] / 1e3, peaks, src) for n in kern}
+        step_roof = sum(r["t_roofline_us"] for r in roofs.values())
+        points.append({"features": 2 ** w["m_bits"], "k": w["k"], "beam": w["beam"],
+                       "encoder": "tensor-core" if w["beam"] <= 8 else "general",
+                       "tokens_per_s": round(whole_job_rate(T, world, 1, ms / 1e3), 1),
+                       "ms": {n: round(v, 4) for n, v in kern.items()},
+                       "frac": {n: r["frac"] for n, r in roofs.items()},
+                       "step_roofline_frac": round(step_roof / (1e3 * ms), 4),
+                       "device_status": dpb.workspace_status(ws)})
+        del x, gy, idx, val, xn, y, gx, gv, rk, ws, plan
+        torch.cuda.empty_cache()
+    line = {"metric": "DPB sweep at d=768, T=32768: tokens/s (encode+decode+bwd) and roofline fraction per point",
+            "unit": "tokens/s", "n_gpus": world, "steps": steps, "warmup": 2, "higher_is_better": True,
+            "scaling": "weak", "dtype": "bf16", "data": "synthetic (x, grad_y ~ N(0, 1), bf16)",
+            "config": {"workload": "sweep", "T_per_gpu": 32768, "d": 768, "levels": 5, "children": 16,
+                       "r_kept": "decode keeps r (fp32) for the backward"},
+            "points": points}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    return 0
+
+
+# ---------------------------------------------------------------------------
 # the ParityTransformer step (GPT-2 small shape): the DPB's share of a step
 # ---------------------------------------------------------------------------
 
@@ -787,7 +865,7 @@ def main(argv=None):
     ap.add_argument("--standardise", action="store_true",
                     help="live standardisation tables and the per-step EMA update in the timed step")
     ap.add_argument("--no-dense", action="store_true", help="gpt2small: skip the dense model of the same shape")
-    ap.add_argument("--workload", default=WORKLOAD, choices=[WORKLOAD, "paper3l", "paper2l", "gpt2small"],
+    ap.add_argument("--workload", default=WORKLOAD, choices=[WORKLOAD, "paper3l", "paper2l", "gpt2small", "sweep"],
                     help="wide (the headline, global selection) or one of the paper's per-level layouts")
     args = ap.parse_args(argv)
     world, rank, local = dist_env()
@@ -798,6 +876,8 @@ def main(argv=None):
         return run_reference(args, world, rank)
     if args.workload == "gpt2small":
         return run_transformer(args, world, rank, local)
+    if args.workload == "sweep":
+        return run_sweep(args, world, rank, local)
     if args.workload != WORKLOAD:
         return run_per_level(args, world, rank, local)
     return run_ours(args, world, rank, local)

@@ -102,7 +102,7 @@ typedef enum { DPB_SCORING_CONTRACTION = 0, DPB_SCORING_COSET_WHT = 1 } dpb_scor
  *               g0 ^ {0, ..., 15} of the span of index bits 0..3: a parent's 16
  *               child scores are then a 16-point Walsh-Hadamard transform of
  *               16 bucket sums of x (.) phi~_{p ^ g0} (bucket = iota mod 16).
- *               Global selection, bf16, beam 8, d a multiple of 32 up to 1024.
+ *               Global selection, bf16, beam <= 8, d a multiple of 32 up to 1024.
  */
 typedef struct dpb_config {
     int32_t d;

@@ -41,6 +41,7 @@ cudaError_t launch_encode_mma(const dpb_plan *p, const void *x, int64_t T, const
     a.nblk = c.d / 32;
     a.levels = c.levels;
     a.k = c.k;
+    a.beam = c.beam;
     a.t = p->t;
     a.ecap = mmaenc::entrant_cap(c.k, c.d / 32);
     a.inv_sqrt_d = p->inv_sqrt_d;

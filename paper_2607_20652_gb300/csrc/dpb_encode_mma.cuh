@@ -1,5 +1,5 @@
 // dpb_encode_mma.cuh -- the §2.2 encoder with the child scoring of Eq. 6 on the
-// tensor cores (bf16 inputs, beam 8, 16 children per parent). Instantiated
+// tensor cores (bf16 inputs, beam up to 8, 16 children per parent). Instantiated
 // per count of inverse-coordinate sign tables (dpb_encode_mma_n*.cu).
 //
 // Scoring. A warp owns two tokens at a time. At level l its 16 tensor-core
@@ -57,6 +57,7 @@ struct Args {
     int32_t *status;
     const uint32_t *frag, *G, *VH, *DD;
     int d, nblk, levels, k, t, ecap;
+    int beam;  // B <= 8: beam slots B..7 hold no parent
     float inv_sqrt_d;
 };
 
@@ -769,7 +770,7 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
                 {
                     uint32_t delta = 0u;
                     bool hit = false;
-                    if (lane < 28) {
+                    if (lane < 28 && ps < a.beam) {  // both slots hold parents
                         delta = bt[ps] ^ bt[psp];
                         uint32_t h = dedup_hash(delta);
                         for (int probe = 0; probe < kDedupSlots; ++probe) {
@@ -813,7 +814,7 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
                 for (int e = 0; e < 4; ++e) {
                     const uint32_t ci = pcur ^ gl[8 * (e >> 1) + 2 * q4 + (e & 1)];
                     const float z = standardise(sc[0][e], ci, a, a.status);
-                    c[e] = ((dmask >> e) & 1u) ? 0ull : cword(z, ci);
+                    c[e] = ((dmask >> e) & 1u) || slot >= a.beam ? 0ull : cword(z, ci);
                     sc[0][e] = sc[1][e];
                 }
                 pcur = p1;
