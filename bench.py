@@ -733,7 +733,7 @@ def run_sweep(args, world, rank, local):
         roofs = {n: roofline_for(n, work[n], kern[n] / 1e3, peaks, src) for n in kern}
         step_roof = sum(r["t_roofline_us"] for r in roofs.values())
         points.append({"features": 2 ** w["m_bits"], "k": w["k"], "beam": w["beam"],
-                       "encoder": "tensor-core" if w["beam"] <= 8 else "general",
+                       "encoder": "tensor-core" if w["beam"] <= 16 else "general",
                        "tokens_per_s": round(whole_job_rate(T, world, 1, ms / 1e3), 1),
                        "ms": {n: round(v, 4) for n, v in kern.items()},
                        "frac": {n: r["frac"] for n, r in roofs.items()},

@@ -235,7 +235,7 @@ cudaError_t launch_encode(const dpb_plan *p, const void *x, int64_t T, const flo
     // the paper's per-level selection: tcgen05 scoring
     if (p->cfg.select_mode == DPB_SELECT_PER_LEVEL)
         return launch_encode_pl(p, x, T, mu, sigma, tab, idx, val, xnorm, status, stream);
-    // bf16 rows on 16-byte boundaries, beam <= 8, 16 children: tensor-core scoring
+    // bf16 rows on 16-byte boundaries, beam <= 16, 16 children: tensor-core scoring
     if (p->mma_encode && (reinterpret_cast<uintptr_t>(x) & 15u) == 0)
         return launch_encode_mma(p, x, T, mu, sigma, tab, idx, val, xnorm, status, stream);
     const dpb_config &c = p->cfg;

@@ -1,5 +1,5 @@
 // dpb_encode_mma.cuh -- the §2.2 encoder with the child scoring of Eq. 6 on the
-// tensor cores (bf16 inputs, beam up to 8, 16 children per parent). Instantiated
+// tensor cores (bf16 inputs, beam up to 16, 16 children per parent). Instantiated
 // per count of inverse-coordinate sign tables (dpb_encode_mma_n*.cu).
 //
 // Scoring. A warp owns two tokens at a time. At level l its 16 tensor-core
@@ -251,6 +251,45 @@ __device__ __forceinline__ void beam_tournament(uint64_t (&c)[4], uint32_t *beam
             c[1] = c[2];
             c[2] = c[3];
             c[3] = 0ull;
+        }
+    }
+    __syncwarp();
+}
+
+// The first nb (<= 16) of up to 256 distinct candidate words held 8 per lane
+// (two groups of 4, 0 = none), by nb rounds of a warp tournament over the
+// heads of the lanes' two sorted groups.
+__device__ __forceinline__ void beam_tournament16(uint64_t (&c)[4], uint64_t (&d)[4], uint32_t *beam, int nb) {
+    cas_desc(c[0], c[1]);
+    cas_desc(c[2], c[3]);
+    cas_desc(c[0], c[2]);
+    cas_desc(c[1], c[3]);
+    cas_desc(c[1], c[2]);
+    cas_desc(d[0], d[1]);
+    cas_desc(d[2], d[3]);
+    cas_desc(d[0], d[2]);
+    cas_desc(d[1], d[3]);
+    cas_desc(d[1], d[2]);
+#pragma unroll 1
+    for (int r = 0; r < nb; ++r) {
+        const bool fc = c[0] > d[0];
+        const uint64_t head = fc ? c[0] : d[0];
+        const uint32_t hi = (uint32_t)(head >> 32), lo = (uint32_t)head;
+        const uint32_t mh = __reduce_max_sync(kFull, hi);
+        const uint32_t ml = __reduce_max_sync(kFull, hi == mh ? lo : 0u);
+        if (hi == mh && lo == ml && (mh | ml) != 0u) {
+            beam[r] = cword_idx(head);
+            if (fc) {
+                c[0] = c[1];
+                c[1] = c[2];
+                c[2] = c[3];
+                c[3] = 0ull;
+            } else {
+                d[0] = d[1];
+                d[1] = d[2];
+                d[2] = d[3];
+                d[3] = 0ull;
+            }
         }
     }
     __syncwarp();
@@ -579,7 +618,11 @@ __device__ __forceinline__ void level0_bisect(const Args &a, const uint16_t *xh,
 // Walsh-Hadamard transform of its bucket sums B_u = sum over iota = u mod 16
 // of x (.) phi~_{p ^ g0}; the shared memory of the B fragments holds the coset
 // tables instead.
-template <int NKC, int KPL, bool COSET>
+// WIDE: beams of 9 to 16. A warp then owns one token, whose beam slots
+// 0..7 and 8..15 take the places of the two tokens (same x, one code list);
+// repeats are found over all 120 slot pairs and the next beam is the top of
+// both halves' children.
+template <int NKC, int KPL, bool COSET, bool WIDE>
 __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
     extern __shared__ __align__(16) uint32_t smem[];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
@@ -622,11 +665,12 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
     // the lane-th slot pair (sp, s), sp < s, of the beam
     const int ps = 1 + (lane >= 1) + (lane >= 3) + (lane >= 6) + (lane >= 10) + (lane >= 15) + (lane >= 21);
     const int psp = lane - ps * (ps - 1) / 2;
-    const int64_t npairs = (a.T + 1) / 2;
+    const int64_t npairs = WIDE ? a.T : (a.T + 1) / 2;
 
     for (int64_t pr = (int64_t)blockIdx.x * nwarps + warp; pr < npairs; pr += (int64_t)gridDim.x * nwarps) {
-        const int64_t t0 = 2 * pr;
-        const int ntok = t0 + 1 < a.T ? 2 : 1;
+        const int64_t t0 = WIDE ? pr : 2 * pr;
+        const int ntok = WIDE ? 1 : (t0 + 1 < a.T ? 2 : 1);
+        const int nhalf = WIDE ? 2 : ntok;  // row groups of 8 beam slots
 
         // ---- each row into the permuted tile; |x|; level 0 ----
         for (int tk = 0; tk < ntok; ++tk) {
@@ -657,6 +701,10 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
             if (!done)
                 level0_bisect(a, xh + tk * nblk * 32, reinterpret_cast<float *>(E),
                               reinterpret_cast<uint32_t *>(E) + a.ecap, a.ecap, Lt, bt);
+            if constexpr (WIDE) {  // the beam: the first 16 of the sorted list (k >= beam)
+                if (lane < 16) beams[lane] = cword_idx(Lt[lane]);
+                __syncwarp();
+            }
         }
 
         // ---- levels 1 .. L-1 ----
@@ -664,12 +712,12 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
             const uint32_t *frag = s_frag + (l - 1) * nblk * 256;
             // this lane's tensor-core rows: (token 0, slot) and (token 1, slot)
             const uint32_t p0 = beams[slot];
-            const uint32_t p1 = ntok > 1 ? beams[kBeam + slot] : 0u;
+            const uint32_t p1 = nhalf > 1 ? beams[kBeam + slot] : 0u;
             // sign words of the 16 rows' parents over every block, row 2 slot + token
             uint2 *sgn = reinterpret_cast<uint2 *>(E);  // [nblk][8] (token 0, token 1)
             {
                 const int row = lane & 15;
-                const uint32_t pr = (row & 1) && ntok < 2 ? 0u : beams[(row & 1) * kBeam + (row >> 1)];
+                const uint32_t pr = (row & 1) && nhalf < 2 ? 0u : beams[(row & 1) * kBeam + (row >> 1)];
                 const ParentOff po = parent_offsets(pr, t, s_w5);
                 uint32_t *sw = reinterpret_cast<uint32_t *>(E);
                 for (int m = lane >> 4; m < nblk; m += 2) sw[m * 16 + row] = parent_signs<NKC>(po, s_pq, s_vh, m);
@@ -688,7 +736,7 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
                 for (int m = 0; m < nblk; ++m) {
                     const uint32_t gw = cw[m];
                     const float x0 = __uint_as_float((uint32_t)xh[(m * 16 + wl) * 2 + hl] << 16);
-                    const float x1 = __uint_as_float((uint32_t)xh[(nblk * 16 + m * 16 + wl) * 2 + hl] << 16);
+                    const float x1 = __uint_as_float((uint32_t)xh[((WIDE ? 0 : nblk * 16) + m * 16 + wl) * 2 + hl] << 16);
 #pragma unroll
                     for (int sl = 0; sl < 8; ++sl) {
                         const uint2 sg = sgn[m * 8 + sl];
@@ -725,7 +773,7 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
 #pragma unroll
                             for (int r = 0; r < 4; ++r) acc[u][c][h][r] = 0.f;
                 const uint4 *xa = reinterpret_cast<const uint4 *>(xt) + q4;
-                const uint4 *xb = reinterpret_cast<const uint4 *>(xt + nblk * 16) + q4;
+                const uint4 *xb = reinterpret_cast<const uint4 *>(xt + (WIDE ? 0 : nblk * 16)) + q4;
                 const uint4 *fr = reinterpret_cast<const uint4 *>(frag) + lane * 2;
                 const int sh = 15 - q4;
 #pragma unroll 2
@@ -761,13 +809,46 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
             const uint32_t *gl = s_g + l * 16;
             const uint32_t *ddl = s_dd + (l - 1) * kDedupSlots * 2;
             uint32_t pcur = p0;
-            for (int tk = 0; tk < ntok; ++tk) {
+            if constexpr (WIDE) {
+                // repeats over all pairs S' < S < beam of the 16 slots: pair q = lane + 32 r
+                if (lane < 8) dup[lane] = 0u;
+                __syncwarp();
+#pragma unroll 1
+                for (int q = lane; q < 120; q += 32) {
+                    int S = (int)((1.f + sqrtf(8.f * (float)q + 1.f)) * 0.5f);
+                    while (S * (S - 1) / 2 > q) --S;
+                    while ((S + 1) * S / 2 <= q) ++S;
+                    const int Sp = q - S * (S - 1) / 2;
+                    if (S >= a.beam) continue;
+                    const uint32_t delta = beams[S] ^ beams[Sp];
+                    uint32_t h = dedup_hash(delta);
+                    for (int probe = 0; probe < kDedupSlots; ++probe) {
+                        const uint32_t key = ddl[2 * h];
+                        if (key == 0u) break;
+                        if (key == delta + 1u) {
+                            const uint32_t bit = (uint32_t)S * 16u + (ddl[2 * h + 1] & 0xffu);
+                            atomicOr(&dup[bit >> 5], 1u << (bit & 31u));
+                        }
+                        h = (h + 1u) & (kDedupSlots - 1);
+                    }
+                }
+                __syncwarp();
+            }
+            uint64_t cw0[4] = {0ull, 0ull, 0ull, 0ull};  // WIDE: the first half's candidate words
+            for (int tk = 0; tk < nhalf; ++tk) {
                 uint32_t *bt = beams + tk * kBeam;
-                uint64_t *Lt = codes + tk * k;
+                uint64_t *Lt = codes + (WIDE ? 0 : tk * k);
                 // ---- duplicate children (R8): p_s ^ g_j' == p_s' ^ g_j with s' < s
                 // exactly when p_s ^ p_s' == g_j ^ g_j'; slot s's copy is dropped
                 uint32_t dmask = 0u;
-                {
+                if constexpr (WIDE) {
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const uint32_t bit =
+                            (uint32_t)(8 * tk + slot) * 16u + (uint32_t)(8 * (e >> 1) + 2 * q4 + (e & 1));
+                        dmask |= ((dup[bit >> 5] >> (bit & 31u)) & 1u) << e;
+                    }
+                } else {
                     uint32_t delta = 0u;
                     bool hit = false;
                     if (lane < 28 && ps < a.beam) {  // both slots hold parents
@@ -814,13 +895,23 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
                 for (int e = 0; e < 4; ++e) {
                     const uint32_t ci = pcur ^ gl[8 * (e >> 1) + 2 * q4 + (e & 1)];
                     const float z = standardise(sc[0][e], ci, a, a.status);
-                    c[e] = ((dmask >> e) & 1u) || slot >= a.beam ? 0ull : cword(z, ci);
+                    // (WIDE: tk is the half of the beam; otherwise the token)
+                    c[e] = ((dmask >> e) & 1u) || (WIDE ? 8 * tk + slot : slot) >= a.beam ? 0ull : cword(z, ci);
                     sc[0][e] = sc[1][e];
                 }
                 pcur = p1;
                 const bool next = l + 1 < L;
-                const int m = merge_entrants<KPL>(Lt, k, E, c, next ? bt : nullptr);
-                if (next && (m < kBeam || m > 32)) beam_tournament(c, bt);
+                const int m = merge_entrants<KPL>(Lt, k, E, c, next && !WIDE ? bt : nullptr);
+                if constexpr (WIDE) {
+                    if (tk == 0) {
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) cw0[e] = c[e];
+                    } else if (next) {
+                        beam_tournament16(cw0, c, beams, a.beam);
+                    }
+                } else {
+                    if (next && (m < kBeam || m > 32)) beam_tournament(c, bt);
+                }
                 __syncwarp();
             }
         }
@@ -843,22 +934,29 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
     }
 }
 
-template <int NKC, int KPL, bool COSET>
+template <int NKC, int KPL, bool COSET, bool WIDE = false>
 cudaError_t launch_kpl(const dpb_plan *p, const Args &a, int warps, cudaStream_t stream) {
     const size_t smem = encode_mma_smem(p, warps);
     const cudaError_t e =
-        cudaFuncSetAttribute(encode_kernel<NKC, KPL, COSET>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        cudaFuncSetAttribute(encode_kernel<NKC, KPL, COSET, WIDE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
     if (e != cudaSuccess) return e;
     int sms = 0;
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, p->device);
-    const int64_t pairs = (a.T + 1) / 2;
+    const int64_t pairs = WIDE ? a.T : (a.T + 1) / 2;
     const int grid = (int)std::min<int64_t>((pairs + warps - 1) / warps, (int64_t)std::max(sms, 1));
-    encode_kernel<NKC, KPL, COSET><<<grid, warps * 32, smem, stream>>>(a);
+    encode_kernel<NKC, KPL, COSET, WIDE><<<grid, warps * 32, smem, stream>>>(a);
     return cudaGetLastError();
 }
 
 template <int NKC>
 cudaError_t launch_nkc(const dpb_plan *p, const Args &a, int warps, cudaStream_t stream) {
+    if (a.beam > kBeam) {
+        if (a.k <= 32) return launch_kpl<NKC, 1, false, true>(p, a, warps, stream);
+        if (a.k <= 64) return launch_kpl<NKC, 2, false, true>(p, a, warps, stream);
+        if (a.k <= 128) return launch_kpl<NKC, 4, false, true>(p, a, warps, stream);
+        return launch_kpl<NKC, 8, false, true>(p, a, warps, stream);
+    }
     if (a.coset) {
         if (a.k <= 32) return launch_kpl<NKC, 1, true>(p, a, warps, stream);
         if (a.k <= 64) return launch_kpl<NKC, 2, true>(p, a, warps, stream);

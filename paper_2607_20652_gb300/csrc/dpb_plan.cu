@@ -152,7 +152,7 @@ int ceil_log2(int v) {
 void build_mma_tables(dpb_plan *p) {
     const dpb_config &c = p->cfg;
     bool ok = c.dtype == DPB_BF16 && c.d % 32 == 0 && c.d >= 32 && c.d <= 1024 && c.levels >= 2 &&
-              c.select_mode == DPB_SELECT_GLOBAL && c.beam >= 1 && c.beam <= 8 && c.k >= c.beam && c.k <= 256;
+              c.select_mode == DPB_SELECT_GLOBAL && c.beam >= 1 && c.beam <= 16 && c.k >= c.beam && c.k <= 256;
     for (int l = 1; l < c.levels && ok; ++l) ok = c.children[l] == 16;
     const int nblk = c.d / 32;
     // every level's fragments, the tables and the warps' lists share one block
@@ -336,7 +336,7 @@ dpb_status resolve_and_build(const dpb_config *in, const uint32_t *generators, d
         // the variant outside the paper: every level's 16 generators one coset
         // g0 ^ {0..15} (given by the caller), scored by a 16-point WHT
         if (!generators) return fail(DPB_ERR_INVALID_ARG, "coset scoring needs the caller's generators");
-        if (!p->mma_encode)
+        if (!p->mma_encode || c.beam > 8)
             return fail(DPB_ERR_UNSUPPORTED,
                         "coset scoring needs global selection, bf16, beam <= 8, 16 children, d a multiple of 32 up to 1024");
         const int nblk = c.d / 32;

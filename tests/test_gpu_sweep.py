@@ -3,9 +3,10 @@ k in {16, 32, 64, 128}, beam in {4, 8, 16}; bf16 x ~ N(0, 1)): every point
 runs at its full size through the C ABI, in the launch configuration the
 benchmark uses, and a sample of its tokens is compared with the oracle under
 the rules of ``tests/parity.py`` (indices as sets except near-ties; values,
-decode and both gradients on the GPU's own code). Beams 4 and 8 run the
-tensor-core encoder (beam slots past the beam hold no parent), beam 16 the
-general one.
+decode and both gradients on the GPU's own code). Every point runs the
+tensor-core encoder: beam slots past the beam hold no parent, and a beam of
+16 gives a warp one token whose two halves of 8 slots fill the tensor-core
+rows.
 """
 import numpy as np
 import pytest
