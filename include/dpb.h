@@ -262,6 +262,16 @@ dpb_status dpb_stats_accumulate(const dpb_plan *plan, const void *x, int64_t T, 
 dpb_status dpb_stats_update(const dpb_plan *plan, double *acc, float alpha, float *mu, float *sigma,
                             void *stream);
 
+/*
+ * dpb_forward -- dpb_encode then dpb_decode of the same rows in one call
+ * (two kernels on `stream`; the code is written out, as the backward needs
+ * it). Arguments as in those two calls; xnorm is required when the plan has
+ * norm_match. Errors: those of either call.
+ */
+dpb_status dpb_forward(const dpb_plan *plan, const void *x, int64_t T, const float *mu, const float *sigma,
+                       int32_t *idx, float *val, float *xnorm, void *y, float *r_out, void *workspace,
+                       size_t workspace_bytes, void *stream);
+
 /* Read (and with clear != 0, zero) the workspace status word: synchronises
  * `stream`, writes the sticky DPB_DEV_* bits to host *status_out, and returns
  * DPB_ERR_DEVICE if any bit is set, else DPB_OK. */

@@ -234,6 +234,16 @@ dpb_status dpb_backward(const dpb_plan *plan, const void *x, const int32_t *idx,
                     "backward");
 }
 
+dpb_status dpb_forward(const dpb_plan *plan, const void *x, int64_t T, const float *mu, const float *sigma,
+                       int32_t *idx, float *val, float *xnorm, void *y, float *r_out, void *workspace,
+                       size_t workspace_bytes, void *stream) {
+    DPB_TRY(check_plan(plan));
+    if (plan->cfg.norm_match && T > 0 && !xnorm)
+        return dpb::fail(DPB_ERR_INVALID_ARG, "xnorm is required with norm_match");
+    DPB_TRY(dpb_encode(plan, x, T, mu, sigma, idx, val, xnorm, workspace, workspace_bytes, stream));
+    return dpb_decode(plan, idx, val, T, xnorm, y, r_out, workspace, workspace_bytes, stream);
+}
+
 dpb_status dpb_stats_accumulate(const dpb_plan *plan, const void *x, int64_t T, const float *mu,
                                 const float *sigma, const int32_t *sample, int32_t n_sample, double *acc,
                                 void *workspace, size_t workspace_bytes, void *stream) {

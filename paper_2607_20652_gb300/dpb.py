@@ -66,7 +66,7 @@ _lib = None
 EXPORTS = ("dpb_plan_create", "dpb_plan_destroy", "dpb_plan_config", "dpb_plan_tables",
            "dpb_code_length", "dpb_workspace_size", "dpb_encode", "dpb_decode", "dpb_backward",
            "dpb_workspace_status", "dpb_status_string", "dpb_last_error", "dpb_encode_noalloc",
-           "dpb_stats_accumulate", "dpb_stats_update")
+           "dpb_stats_accumulate", "dpb_stats_update", "dpb_forward")
 
 
 def library_path() -> str:
@@ -98,6 +98,7 @@ def load(path: Optional[str] = None):
     lib.dpb_encode_noalloc.argtypes = [vp, vp, i64, vp, vp, vp, vp, vp, vp, vp]
     lib.dpb_stats_accumulate.argtypes = [vp, vp, i64, vp, vp, vp, ctypes.c_int32, vp, vp, sz, vp]
     lib.dpb_stats_update.argtypes = [vp, vp, ctypes.c_float, vp, vp, vp]
+    lib.dpb_forward.argtypes = [vp, vp, i64, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
     lib.dpb_status_string.argtypes = [st]
     lib.dpb_status_string.restype = ctypes.c_char_p
     lib.dpb_last_error.argtypes = []
@@ -278,6 +279,25 @@ def decode(plan: Plan, idx: torch.Tensor, val: torch.Tensor, xnorm=None, y=None,
     _check(plan._lib.dpb_decode(plan.handle, _ptr(idx), _ptr(val), T, _ptr(xnorm), _ptr(y), _ptr(r_out),
                                 _ptr(ws), ws.numel() * ws.element_size(), _stream(stream)))
     return y
+
+
+def forward(plan: Plan, x: torch.Tensor, mu=None, sigma=None, workspace=None, stream=None,
+            r_out: Optional[torch.Tensor] = None):
+    """dpb_forward (encode then decode). Returns (idx, val, xnorm, y)."""
+    _rows(x, plan, "x")
+    T, k, dev = x.shape[0], plan.code_len, x.device
+    idx = torch.empty((T, k), dtype=torch.int32, device=dev)
+    val = torch.empty((T, k), dtype=torch.float32, device=dev)
+    xnorm = torch.empty((T,), dtype=torch.float32, device=dev)
+    y = torch.empty_like(x)
+    if r_out is not None and (r_out.dtype != torch.float32 or not r_out.is_contiguous()
+                              or tuple(r_out.shape) != (T, plan.d)):
+        raise ValueError(f"r_out must be a contiguous float32 tensor of shape [T, {plan.d}]")
+    ws = plan._stream_workspace(T, dev, stream) if workspace is None else workspace
+    _check(plan._lib.dpb_forward(plan.handle, _ptr(x), T, _ptr(mu), _ptr(sigma), _ptr(idx), _ptr(val),
+                                 _ptr(xnorm), _ptr(y), _ptr(r_out), _ptr(ws), ws.numel() * ws.element_size(),
+                                 _stream(stream)))
+    return idx, val, xnorm, y
 
 
 def backward(plan: Plan, x: torch.Tensor, idx: torch.Tensor, val: torch.Tensor, grad_y: torch.Tensor,

@@ -382,3 +382,16 @@ def test_calls_without_a_workspace_share_one_per_stream():
     dpb.decode(plan, bad, val, xn)
     assert len(plan._ws_cache) == 1
     assert plan.status() == dpb.DEV_BAD_INDEX and plan.status() == 0
+
+
+def test_forward_is_encode_then_decode():
+    plan = dpb.Plan(d=768, levels=5, m_bits=20, children=16, beam=8, k=64, dtype="bf16")
+    dev = torch.device("cuda")
+    x = torch.from_numpy(inputs.to_bf16(inputs.gaussian_rows(500, 768, 97))).to(dev).to(torch.bfloat16)
+    r = torch.empty((500, 768), dtype=torch.float32, device=dev)
+    idx, val, xn, y = dpb.forward(plan, x, r_out=r)
+    i2, v2, xn2 = dpb.encode(plan, x)
+    y2 = dpb.decode(plan, i2, v2, xn2)
+    torch.cuda.synchronize()
+    assert torch.equal(idx, i2) and torch.equal(val, v2) and torch.equal(xn, xn2) and torch.equal(y, y2)
+    assert plan.status() == 0
