@@ -155,16 +155,19 @@ __global__ void __launch_bounds__(128) backward_warp_kernel(BackwardArgs a) {
 constexpr int kChunkBlocks = 4;                       // 32-coordinate blocks per analysis chunk
 constexpr int kTabStride = 17;                        // 16 entries + 1 pad (bank spread)
 constexpr int kChunkTables = kChunkBlocks * 8 * kTabStride;  // nibble tables of a chunk (words)
+constexpr int kScratchWords = pad64(kSweepWords > kChunkTables ? kSweepWords : kChunkTables);
 constexpr int kBwdWarps = 8;
-static_assert(kChunkBlocks == 4, "analyse() maps items to blocks with three compares");
+static_assert(kChunkBlocks == 4, "the analysis gives a code 4 lanes, one per block of a chunk");
 
+// Per-warp words: the scratch (a sweep's tables, or a chunk's nibble tables;
+// first, so that it keeps the region's 256-byte alignment), then r / dL/dr /
+// grad_x (d) and the code's lists (list, map, sums, offsets).
 __host__ __device__ constexpr int bwd_warp_words(int d, int k) {
-    return pad4(d) /* r, then dL/dr, then grad_x */ + 6 * pad4(k) /* list, map, sums, offsets */ +
-           (kSweepWords > kChunkTables ? kSweepWords : pad4(kChunkTables));
+    return pad64(kScratchWords + pad4(d) + 6 * pad4(k));
 }
 
 __host__ __device__ constexpr int bwd_block_words(int d, int nkc) {
-    return pad4(d) /* koff */ + 32 /* W5 */ + nkc * ((d + 31) / 32) * 32 /* VH2 */;
+    return pad64(pad4(d) /* koff */ + 32 /* W5 */ + nkc * ((d + 31) / 32) * 32 /* VH2 */);
 }
 
 struct BwdWarp {
@@ -178,18 +181,74 @@ struct BwdWarp {
     uint32_t *scratch;
 };
 
+// The 4 nibble offsets (times 4, one per byte) of the even (ev) and odd (od)
+// nibbles of a sign word: nibble n of s indexes table n of its block.
+__device__ __forceinline__ void nibble_offsets(uint32_t s, uint32_t &ev, uint32_t &od) {
+    ev = (s << 2) & 0x3C3C3C3Cu;  // nibbles 0, 2, 4, 6
+    od = (s >> 2) & 0x3C3C3C3Cu;  // nibbles 1, 3, 5, 7
+}
+
+// The 8 table entries of one (code, block) term as a pair of partial sums.
+// A table's address is its block's base with the entry offset in the low
+// byte: base_s must be 256-byte aligned, the table offsets OFF + n 68 come
+// as immediates.
+template <int OFF>
+__device__ __forceinline__ float2 nibble_sum(uint32_t base_s, uint32_t s) {
+    constexpr int S4 = 4 * kTabStride;  // bytes per table
+    uint32_t ev, od;
+    nibble_offsets(s, ev, od);
+    const float p0 = lds_f32<OFF + 0 * S4>(__byte_perm(ev, base_s, 0x7650));
+    const float p1 = lds_f32<OFF + 1 * S4>(__byte_perm(od, base_s, 0x7650));
+    const float p2 = lds_f32<OFF + 2 * S4>(__byte_perm(ev, base_s, 0x7651));
+    const float p3 = lds_f32<OFF + 3 * S4>(__byte_perm(od, base_s, 0x7651));
+    const float p4 = lds_f32<OFF + 4 * S4>(__byte_perm(ev, base_s, 0x7652));
+    const float p5 = lds_f32<OFF + 5 * S4>(__byte_perm(od, base_s, 0x7652));
+    const float p6 = lds_f32<OFF + 6 * S4>(__byte_perm(ev, base_s, 0x7653));
+    const float p7 = lds_f32<OFF + 7 * S4>(__byte_perm(od, base_s, 0x7653));
+    return __fadd2_rn(__fadd2_rn(make_float2(p0, p1), make_float2(p2, p3)),
+                      __fadd2_rn(make_float2(p4, p5), make_float2(p6, p7)));
+}
+
+// The same with the block's base in a register (any 4-byte alignment).
+__device__ __forceinline__ float nibble_sum_at(uint32_t blk_s, uint32_t s) {
+    constexpr int S4 = 4 * kTabStride;
+    uint32_t ev, od;
+    nibble_offsets(s, ev, od);
+    const float p0 = lds_f32<0 * S4>(blk_s + __byte_perm(ev, 0, 0x4440));
+    const float p1 = lds_f32<1 * S4>(blk_s + __byte_perm(od, 0, 0x4440));
+    const float p2 = lds_f32<2 * S4>(blk_s + __byte_perm(ev, 0, 0x4441));
+    const float p3 = lds_f32<3 * S4>(blk_s + __byte_perm(od, 0, 0x4441));
+    const float p4 = lds_f32<4 * S4>(blk_s + __byte_perm(ev, 0, 0x4442));
+    const float p5 = lds_f32<5 * S4>(blk_s + __byte_perm(od, 0, 0x4442));
+    const float p6 = lds_f32<6 * S4>(blk_s + __byte_perm(ev, 0, 0x4443));
+    const float p7 = lds_f32<7 * S4>(blk_s + __byte_perm(od, 0, 0x4443));
+    const float2 r = __fadd2_rn(__fadd2_rn(make_float2(p0, p1), make_float2(p2, p3)),
+                                __fadd2_rn(make_float2(p4, p5), make_float2(p6, p7)));
+    return r.x + r.y;
+}
+
+// Block QQ of the chunk at q0 (if the chunk has it) added into a code's sums.
+template <int NKC, int QQ>
+__device__ __forceinline__ void add_block(float2 &acc, const uint32_t *vh2, int qn, int q0, int cq, uint32_t o1,
+                                          uint32_t o2, uint32_t th_s) {
+    if (QQ < cq)
+        acc = __fadd2_rn(acc, nibble_sum<QQ * 8 * kTabStride * 4>(th_s, block_signs<NKC>(vh2, qn, q0 + QQ, o1, o2)));
+}
+
 // gv[p] += sum_i h[i] (-1)^{parity(M[i] AND hc_p)} for the nh hashed codes.
-// Per chunk of 8 blocks: nibble tables TH[b][n][v] = sum_j (-1)^{v_j}
-// h[32b + 4n + j] (16 entries per 4 coordinates), then one (code, block) item
-// per lane: the code's sign word over the block indexes 8 nibble tables.
-// Items of one warp step have distinct codes, so the shared-memory
-// accumulation order is fixed.
+// Per chunk of 4 blocks: nibble tables TH[b][n][v] = sum_j (-1)^{v_j}
+// h[32b + 4n + j] (16 entries per 4 coordinates); a code's sign word over a
+// block indexes that block's 8 tables. The first nh - nh % 32 codes go one
+// per lane through all blocks of the chunk; each of the others gets 4 lanes,
+// one block each, summed by shuffles. Every code's sum is taken in a fixed
+// order.
 template <int NKC>
 __device__ __forceinline__ void analyse(const BwdWarp &w, int nh, int d, const uint32_t *vh2) {
     const int lane = threadIdx.x & 31;
     const int qn = (d + 31) / 32;
-    const int nhp = nh > 32 ? nh : 32;
+    const int full = nh & ~31, tail = nh - full;
     float *TH = reinterpret_cast<float *>(w.scratch);
+    const uint32_t th_s = smem_u32(TH);  // 256-byte aligned
     for (int q0 = 0; q0 < qn; q0 += kChunkBlocks) {
         const int cq = min(kChunkBlocks, qn - q0);
         // both loops stay rolled: this kernel's hot code is at the instruction caches' size
@@ -216,23 +275,25 @@ __device__ __forceinline__ void analyse(const BwdWarp &w, int nh, int d, const u
         }
         __syncwarp();
 #pragma unroll 1
-        for (int it = lane; it < cq * nhp; it += 32) {
-            // block of the chunk and code of this item (cq <= 4 blocks)
-            const int qq = (it >= nhp) + (it >= 2 * nhp) + (it >= 3 * nhp), e = it - qq * nhp;
-            if (e < nh) {
-                const uint32_t s = block_signs<NKC>(vh2, qn, q0 + qq, w.o1[e], w.o2[e]);
-                const char *T = reinterpret_cast<const char *>(TH + qq * 8 * kTabStride);
-                constexpr int S4 = 4 * kTabStride;  // bytes per table
-                float p0 = *reinterpret_cast<const float *>(T + ((s << 2) & 0x3Cu));
-                float p1 = *reinterpret_cast<const float *>(T + 1 * S4 + ((s >> 2) & 0x3Cu));
-                float p2 = *reinterpret_cast<const float *>(T + 2 * S4 + ((s >> 6) & 0x3Cu));
-                float p3 = *reinterpret_cast<const float *>(T + 3 * S4 + ((s >> 10) & 0x3Cu));
-                float p4 = *reinterpret_cast<const float *>(T + 4 * S4 + ((s >> 14) & 0x3Cu));
-                float p5 = *reinterpret_cast<const float *>(T + 5 * S4 + ((s >> 18) & 0x3Cu));
-                float p6 = *reinterpret_cast<const float *>(T + 6 * S4 + ((s >> 22) & 0x3Cu));
-                float p7 = *reinterpret_cast<const float *>(T + 7 * S4 + ((s >> 26) & 0x3Cu));
-                atomicAdd(&w.gv[e], ((p0 + p1) + (p2 + p3)) + ((p4 + p5) + (p6 + p7)));
-            }
+        for (int e = lane; e < full; e += 32) {  // full is a multiple of 32: no lane drops out
+            const uint32_t o1 = w.o1[e], o2 = w.o2[e];
+            float2 acc = make_float2(0.f, 0.f);
+            add_block<NKC, 0>(acc, vh2, qn, q0, cq, o1, o2, th_s);
+            add_block<NKC, 1>(acc, vh2, qn, q0, cq, o1, o2, th_s);
+            add_block<NKC, 2>(acc, vh2, qn, q0, cq, o1, o2, th_s);
+            add_block<NKC, 3>(acc, vh2, qn, q0, cq, o1, o2, th_s);
+            w.gv[e] += acc.x + acc.y;  // this lane's own code
+        }
+#pragma unroll 1
+        for (int it0 = 0; it0 < 4 * tail; it0 += 32) {
+            const int it = it0 + lane, e = full + (it >> 2), qq = it & 3;
+            float v = 0.f;
+            if (it < 4 * tail && qq < cq)
+                v = nibble_sum_at(th_s + qq * (8 * kTabStride * 4),
+                                  block_signs<NKC>(vh2, qn, q0 + qq, w.o1[e], w.o2[e]));
+            v += __shfl_xor_sync(kFull, v, 1);
+            v += __shfl_xor_sync(kFull, v, 2);
+            if (it < 4 * tail && qq == 0) w.gv[e] += v;  // the code's 4 lanes are lanes 4j .. 4j+3
         }
         __syncwarp();
     }
@@ -240,7 +301,8 @@ __device__ __forceinline__ void analyse(const BwdWarp &w, int nh, int d, const u
 
 template <typename Tio, int NKC, bool VEC>
 __global__ void __launch_bounds__(kBwdWarps * 32, 3) backward_lut_kernel(BackwardArgs a, int t) {
-    extern __shared__ __align__(16) uint32_t smem[];
+    extern __shared__ __align__(16) uint32_t smem_raw[];
+    uint32_t *smem = aligned_smem<256>(smem_raw);
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
     const int d = a.d, k = a.k;
     const int dp = pad4(d), kp = pad4(k);
@@ -257,14 +319,14 @@ __global__ void __launch_bounds__(kBwdWarps * 32, 3) backward_lut_kernel(Backwar
 
     uint32_t *base = smem + bwd_block_words(d, NKC) + (size_t)warp * bwd_warp_words(d, k);
     BwdWarp w;
-    w.buf = reinterpret_cast<float *>(base);
+    w.scratch = base;
+    w.buf = reinterpret_cast<float *>(base + kScratchWords);
     w.hc = reinterpret_cast<uint32_t *>(w.buf + dp);
     w.ha = reinterpret_cast<float *>(w.hc + kp);
     w.cmap = reinterpret_cast<int *>(w.ha + kp);
     w.gv = reinterpret_cast<float *>(w.cmap + kp);
     w.o1 = reinterpret_cast<uint32_t *>(w.gv + kp);
     w.o2 = w.o1 + kp;
-    w.scratch = w.o2 + kp;
     float *bterm = reinterpret_cast<float *>(w.o2);  // basis grad_x terms, after the analysis
     Sweep sw = sweep_at(w.scratch);
 
@@ -392,7 +454,8 @@ int grid_for(const dpb_plan *p, int64_t T, int warps) {
 template <typename Tio, int NKC, bool VEC>
 cudaError_t run_backward_lut(const dpb_plan *p, const BackwardArgs &a, int64_t T, cudaStream_t stream) {
     const int warps = kBwdWarps;
-    const size_t smem = sizeof(uint32_t) * ((size_t)bwd_block_words(p->cfg.d, NKC) +
+    const size_t smem = 256 /* alignment */ +
+                        sizeof(uint32_t) * ((size_t)bwd_block_words(p->cfg.d, NKC) +
                                             (size_t)warps * bwd_warp_words(p->cfg.d, p->code_len));
     const cudaError_t e = cudaFuncSetAttribute(backward_lut_kernel<Tio, NKC, VEC>,
                                                cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);

@@ -89,22 +89,26 @@ __global__ void __launch_bounds__(128) decode_warp_kernel(DecodeArgs a) {
 
 // ---- table-driven decoder (d <= 2048) -----------------------------------------
 
-// Per-warp shared memory of the decoder, in 4-byte words: r (d), the hashed
-// list (indices, coefficients) and one sweep's tables.
-__host__ __device__ constexpr int decode_warp_words(int d, int k) { return pad4(d) + 2 * pad4(k) + kSweepWords; }
+// Per-warp shared memory of the decoder, in 4-byte words: one sweep's tables
+// (first, so that they keep the region's 128-byte alignment), r (d) and the
+// hashed list (indices, coefficients).
+__host__ __device__ constexpr int decode_warp_words(int d, int k) {
+    return pad32(kSweepWords + pad4(d) + 2 * pad4(k));
+}
 
 template <typename Tio, int NKC, bool VEC>
 __global__ void __launch_bounds__(256) decode_lut_kernel(DecodeArgs a, int t) {
-    extern __shared__ __align__(16) uint32_t smem[];
+    extern __shared__ __align__(16) uint32_t smem_raw[];
+    uint32_t *smem = aligned_smem<128>(smem_raw);
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
     const int d = a.d;
     uint32_t *koff = smem;
     load_koff(a.M, d, t, koff);
     const int dp = pad4(d), kp = pad4(a.k);
-    uint32_t *base = smem + dp + (size_t)warp * decode_warp_words(d, a.k);
-    float *r = reinterpret_cast<float *>(base);
-    HashedList hl{base + dp, reinterpret_cast<float *>(base + dp + kp), nullptr};
-    Sweep sw = sweep_at(base + dp + 2 * kp);
+    uint32_t *base = smem + pad32(d) + (size_t)warp * decode_warp_words(d, a.k);
+    Sweep sw = sweep_at(base);
+    float *r = reinterpret_cast<float *>(base + kSweepWords);
+    HashedList hl{base + kSweepWords + dp, reinterpret_cast<float *>(base + kSweepWords + dp + kp), nullptr};
     Tio *Y = static_cast<Tio *>(a.y);
     for (int64_t tk = (int64_t)blockIdx.x * nwarps + warp; tk < a.T; tk += (int64_t)gridDim.x * nwarps) {
         RowOps<VEC>::fill(r, d, 0.f);
@@ -137,7 +141,8 @@ namespace {
 template <typename Tio, int NKC, bool VEC>
 cudaError_t run_decode_lut(const dpb_plan *p, const DecodeArgs &a, int64_t T, cudaStream_t stream) {
     const int warps = 8;
-    const size_t smem = sizeof(uint32_t) * ((size_t)pad4(p->cfg.d) + (size_t)warps * decode_warp_words(p->cfg.d, p->code_len));
+    const size_t smem = 128 /* alignment */ +
+                        sizeof(uint32_t) * ((size_t)pad32(p->cfg.d) + (size_t)warps * decode_warp_words(p->cfg.d, p->code_len));
     const cudaError_t e = cudaFuncSetAttribute(decode_lut_kernel<Tio, NKC, VEC>,
                                                cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;

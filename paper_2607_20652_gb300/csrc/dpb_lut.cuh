@@ -17,7 +17,9 @@
 //     runs are held one entry per lane and read with a shuffle (which uses
 //     only the low 5 bits of its index); odd runs live in shared memory (a
 //     32-word table spans all banks: every lookup is conflict-free). The two
-//     kinds of lookup go down different pipes.
+//     kinds of lookup go down different pipes. The odd tables are 128-byte
+//     aligned, so a lookup's address is the table's address OR the run's 5
+//     bits times 4, one logic instruction.
 #pragma once
 
 #include <cstdint>
@@ -43,15 +45,39 @@ struct Sweep {
     uint2 *zh;                // [kMaxKChunks][32] (shared)
     float *vto;               // [6][32] odd runs (shared)
     float *coef;              // [64] (shared)
+    uint32_t vto_s;           // shared-window address of vto (128-byte aligned)
     int runs;                 // ceil(codes / 5)
 };
 
+// Shared-window (32-bit) address of a pointer into this block's shared memory.
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+// fp32 load from shared memory at byte address addr + OFF.
+template <int OFF>
+__device__ __forceinline__ float lds_f32(uint32_t addr) {
+    float v;
+    asm volatile("ld.shared.f32 %0, [%1+%2];" : "=f"(v) : "r"(addr), "n"(OFF));
+    return v;
+}
+
+// The first A-byte aligned word of a dynamic shared-memory buffer (the
+// launch allocates A bytes more than the layout needs).
+template <int A>
+__device__ __forceinline__ uint32_t *aligned_smem(uint32_t *raw) {
+    return raw + ((A - (smem_u32(raw) & (A - 1))) & (A - 1)) / 4;
+}
+
+// A sweep's tables at base, which must be 128-byte aligned (the odd value
+// tables are addressed by OR).
 __device__ __forceinline__ Sweep sweep_at(uint32_t *base) {
     Sweep s;
     s.zq = reinterpret_cast<uint2 *>(base);
     s.zh = s.zq + kMaxBlocks;
     s.vto = reinterpret_cast<float *>(s.zh + 32 * kMaxKChunks);
     s.coef = s.vto + 32 * (kMaxRuns - kShflRuns);
+    s.vto_s = smem_u32(s.vto);
     return s;
 }
 
@@ -177,14 +203,35 @@ __device__ __forceinline__ uint32_t run_offset(uint2 z) {
 }
 
 template <int G, int RUNS>
-__device__ __forceinline__ void run_lookups(const Sweep &s, uint2 z, const char *vto, float *p) {
+__device__ __forceinline__ void run_lookups(const Sweep &s, uint2 z, float *p) {
     if constexpr (G < RUNS) {
         if constexpr (G % 2 == 0) {
             p[G] = __shfl_sync(kFull, s.vt[G / 2], run_field<G>(z));
         } else {
-            p[G] = *reinterpret_cast<const float *>(vto + (G / 2) * 128 + run_offset<G>(z));
+            p[G] = lds_f32<(G / 2) * 128>(s.vto_s | run_offset<G>(z));
         }
-        run_lookups<G + 1, RUNS>(s, z, vto, p);
+        run_lookups<G + 1, RUNS>(s, z, p);
+    }
+}
+
+// Sum of n floats: pairs added two at a time (packed fp32x2 adds), then the
+// two halves and an odd last one.
+template <int N>
+__device__ __forceinline__ float sum_packed(const float *p) {
+    if constexpr (N == 1) {
+        return p[0];
+    } else {
+        constexpr int NP = N / 2;
+        float2 q[NP];
+#pragma unroll
+        for (int i = 0; i < NP; ++i) q[i] = make_float2(p[2 * i], p[2 * i + 1]);
+#pragma unroll
+        for (int w = 1; w < NP; w *= 2)
+#pragma unroll
+            for (int g = 0; g + w < NP; g += 2 * w) q[g] = __fadd2_rn(q[g], q[g + w]);
+        const float h = q[0].x + q[0].y;
+        if constexpr (N % 2 == 1) return h + p[N - 1];
+        return h;
     }
 }
 
@@ -192,17 +239,17 @@ __device__ __forceinline__ void run_lookups(const Sweep &s, uint2 z, const char 
 template <int RUNS>
 __device__ __forceinline__ float sweep_sum(const Sweep &s, uint2 z) {
     float p[RUNS];
-    run_lookups<0, RUNS>(s, z, reinterpret_cast<const char *>(s.vto), p);
-#pragma unroll
-    for (int w = 1; w < RUNS; w *= 2)
-#pragma unroll
-        for (int g = 0; g + w < RUNS; g += 2 * w) p[g] += p[g + w];
-    return p[0];
+    run_lookups<0, RUNS>(s, z, p);
+    return sum_packed<RUNS>(p);
 }
 
 // Sizes rounded up to 4 words, so that every per-warp array of the kernels'
 // shared-memory layouts starts 16-byte aligned.
 __host__ __device__ constexpr int pad4(int v) { return (v + 3) & ~3; }
+// Sizes rounded up to 32 words (128 bytes) and 64 words (256 bytes).
+__host__ __device__ constexpr int pad32(int v) { return (v + 31) & ~31; }
+__host__ __device__ constexpr int pad64(int v) { return (v + 63) & ~63; }
+static_assert(kSweepWords % 32 == 0, "a sweep's tables keep the 128-byte alignment of what follows");
 
 // ---- a token's code -----------------------------------------------------------
 
