@@ -336,16 +336,49 @@ __global__ void __launch_bounds__(kBwdWarps * 32, 3) backward_lut_kernel(Backwar
     for (int64_t tk = (int64_t)blockIdx.x * nwarps + warp; tk < a.T; tk += (int64_t)gridDim.x * nwarps) {
         const int32_t *it = a.idx + tk * k;
         const float *vt = a.val + tk * k;
-        // ---- split the code: basis entries into buf (r), hashed entries listed ----
         const Tio *xr = X + tk * d, *gr = GY + tk * d;
-        RowOps<VEC>::fill(w.buf, d, 0.f);
+        // the code's first 64 entries, loaded ahead of the rows so that the
+        // two loads overlap
+        int32_t ci_pre[2] = {-1, -1};
+        float v_pre[2] = {0.f, 0.f};
+#pragma unroll
+        for (int j = 0; j < 2; ++j)
+            if (32 * j + lane < k) {
+                ci_pre[j] = it[32 * j + lane];
+                v_pre[j] = vt[32 * j + lane];
+            }
+        // With norm matching and the decode's r, dL/dr comes first, from one
+        // sweep over x, grad_y and r; otherwise buf starts as the basis part
+        // of r (rebuilt below) or as grad_y.
+        const bool kept_r = a.norm_match && a.R;
+        float nx, direct = 0.f;  // direct: coefficient of x / |x| in grad_x
+        if (kept_r) {
+            float sxx = 0.f, srr = 0.f, sgr = 0.f;
+            RowOps<VEC>::rows3(w.buf, xr, gr, a.R + tk * d, d, sxx, srr, sgr);
+            nx = sqrtf(warp_sum(sxx));
+            srr = warp_sum(srr);
+            sgr = warp_sum(sgr);
+            const float nr = sqrtf(srr);
+            if (nr > 0.f) {
+                RowOps<VEC>::project(w.buf, gr, d, nx / nr, sgr / srr);  // this lane's own coordinates
+                direct = nx > 0.f ? sgr / nr : 0.f;
+            } else {
+                RowOps<VEC>::fill(w.buf, d, 0.f);
+            }
+        } else {
+            RowOps<VEC>::fill(w.buf, d, 0.f);
+        }
         __syncwarp();
+        // ---- split the code: hashed entries listed (basis entries into buf when r is rebuilt) ----
         int nh = 0;
         for (int e0 = 0; e0 < k; e0 += 32) {
             const int e = e0 + lane;
             int32_t ci = -1;
             float v = 0.f;
-            if (e < k) {
+            if (e0 < 64) {
+                ci = ci_pre[e0 >> 5];
+                v = v_pre[e0 >> 5];
+            } else if (e < k) {
                 ci = it[e];
                 v = vt[e];
             }
@@ -356,7 +389,7 @@ __global__ void __launch_bounds__(kBwdWarps * 32, 3) backward_lut_kernel(Backwar
                 w.cmap[e] = INT_MIN;
             }
             if (valid && !hashed) {
-                atomicAdd(&w.buf[ci], v);
+                if (a.norm_match && !kept_r) atomicAdd(&w.buf[ci], v);
                 w.cmap[e] = -(ci + 1);
             }
             const unsigned m = __ballot_sync(kFull, hashed);
@@ -371,8 +404,7 @@ __global__ void __launch_bounds__(kBwdWarps * 32, 3) backward_lut_kernel(Backwar
             nh += __popc(m);
         }
         __syncwarp();
-        const float nx = sqrtf(warp_sum(RowOps<VEC>::sumsq(xr, d)));
-        float direct = 0.f;  // coefficient of x / |x| in grad_x
+        if (!kept_r) nx = sqrtf(warp_sum(RowOps<VEC>::sumsq(xr, d)));
         if (!a.norm_match) {
             RowOps<VEC>::scale_in(w.buf, gr, d, 1.f);
             __syncwarp();
@@ -381,7 +413,7 @@ __global__ void __launch_bounds__(kBwdWarps * 32, 3) backward_lut_kernel(Backwar
         // matching only) and turns it into dL/dr; pass 1 adds the hashed
         // entries' sum to grad_x.
 #pragma unroll 1
-        for (int pass = a.norm_match ? 0 : 1;; ++pass) {
+        for (int pass = a.norm_match && !kept_r ? 0 : 1;; ++pass) {
             if (pass == 1) {
                 // ---- grad_val = <phi_e, dL/dr> ----
                 analyse<NKC>(w, nh, d, vh2);
@@ -421,10 +453,7 @@ __global__ void __launch_bounds__(kBwdWarps * 32, 3) backward_lut_kernel(Backwar
                 }
                 __syncwarp();
             }
-            if (pass == 0 && a.R)
-                RowOps<VEC>::scale_in(w.buf, a.R + tk * d, d, 1.f);  // r as the decode left it
-            else
-                synthesise<NKC, kSweepCompact>(sw, w.hc, w.ha, nh, t, d, koff, a.inv_sqrt_d, w.buf);
+            synthesise<NKC, kSweepCompact>(sw, w.hc, w.ha, nh, t, d, koff, a.inv_sqrt_d, w.buf);
             if (pass == 1) break;
             // ---- dL/dr = c (g - (<g,r>/|r|^2) r) in place of r ----
             float srr = 0.f, sgr = 0.f;

@@ -106,6 +106,31 @@ struct RowOps {
             }
         }
     }
+    // buf[i] = r[i]; sxx += x[i]^2, srr += r[i]^2, sgr += g[i] r[i] (this
+    // lane's share): the three rows in one sweep
+    template <typename T>
+    __device__ __forceinline__ static void rows3(float *buf, const T *x, const T *g, const float *r, int d,
+                                                 float &sxx, float &srr, float &sgr) {
+        const int lane = threadIdx.x & 31;
+        if (VEC) {
+            for (int i = 4 * lane; i < d; i += 128) {
+                const float4 xv = ld4(x + i), gv = ld4(g + i);
+                const float4 rv = *reinterpret_cast<const float4 *>(r + i);
+                sxx += xv.x * xv.x + xv.y * xv.y + xv.z * xv.z + xv.w * xv.w;
+                srr += rv.x * rv.x + rv.y * rv.y + rv.z * rv.z + rv.w * rv.w;
+                sgr += gv.x * rv.x + gv.y * rv.y + gv.z * rv.z + gv.w * rv.w;
+                *reinterpret_cast<float4 *>(buf + i) = rv;
+            }
+        } else {
+            for (int i = lane; i < d; i += 32) {
+                const float xv = ld_elem(x, i), gv = ld_elem(g, i), rv = r[i];
+                sxx += xv * xv;
+                srr += rv * rv;
+                sgr += gv * rv;
+                buf[i] = rv;
+            }
+        }
+    }
     // buf[i] = c (row[i] - beta buf[i])
     template <typename T>
     __device__ __forceinline__ static void project(float *buf, const T *row, int d, float c, float beta) {

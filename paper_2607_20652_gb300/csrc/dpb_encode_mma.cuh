@@ -190,12 +190,12 @@ template <int R, typename W>
 __device__ __forceinline__ void sort_stage(W (&v)[R], int size, int stride) {
     const int lane = threadIdx.x & 31;
     if (stride >= R) {
-        const bool lower = (lane & (stride / R)) == 0;
+        // size >= 2 stride >= 2R: r never reaches the size bit of lane R + r
+        const bool keep_hi = ((lane & (stride / R)) == 0) == (((lane * R) & size) == 0);
 #pragma unroll
         for (int r = 0; r < R; ++r) {
-            const bool desc = (((lane * R + r) & size) == 0);
             const W o = __shfl_xor_sync(kFull, v[r], stride / R);
-            v[r] = (lower == desc) ? whi(v[r], o) : wlo(v[r], o);
+            v[r] = keep_hi ? whi(v[r], o) : wlo(v[r], o);
         }
     } else {
 #pragma unroll
@@ -293,6 +293,25 @@ __device__ __forceinline__ void beam_tournament16(uint64_t (&c)[4], uint64_t (&d
         }
     }
     __syncwarp();
+}
+
+// The same for lanes whose R words are already sorted descending: odd lanes
+// reverse theirs (a bitonic merge of size 2R wants them ascending) and the
+// sort starts at size 2R.
+template <int R, typename W>
+__device__ __forceinline__ void warp_sort_desc_runs(W (&v)[R]) {
+    if (threadIdx.x & 1) {
+#pragma unroll
+        for (int r = 0; r < R / 2; ++r) {
+            const W t = v[r];
+            v[r] = v[R - 1 - r];
+            v[R - 1 - r] = t;
+        }
+    }
+#pragma unroll 1
+    for (int size = 2 * R; size <= 32 * R; size <<= 1)
+#pragma unroll 1
+        for (int stride = size / 2; stride > 0; stride >>= 1) sort_stage<R, W>(v, size, stride);
 }
 
 // ---- merging entrants into a code list -------------------------------------------
@@ -393,7 +412,7 @@ __device__ __forceinline__ bool level0_union(const uint4 *row, int nch, int k, u
         }
     }
     const uint32_t kept_min = top[R - 1];  // every word of this lane below it was not kept
-    warp_sort_desc<R>(top);
+    warp_sort_desc_runs<R>(top);
     uint32_t mine = 0u;
 #pragma unroll
     for (int r = 0; r < R; ++r)
@@ -468,7 +487,7 @@ __device__ __forceinline__ bool level0_union_std(const Args &a, const uint16_t *
         }
     }
     const uint64_t kept_min = top[R - 1];  // every word of this lane below it was not kept
-    warp_sort_desc<R>(top);
+    warp_sort_desc_runs<R>(top);
     uint64_t mine = 0ull;
 #pragma unroll
     for (int r = 0; r < R; ++r)
