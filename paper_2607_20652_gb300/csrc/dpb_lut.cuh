@@ -42,7 +42,7 @@ struct Sweep {
     uint2 zl;                 // ZL(lane) for codes 0..31 (x) and 32..63 (y)
     float vt[kShflRuns];      // lane v holds the table of run 2i at v
     uint2 *zq;                // [kMaxBlocks] (shared)
-    uint2 *zh;                // [kMaxKChunks][32] (shared)
+    uint32_t *zh;             // [kMaxKChunks][2][32]: codes 0..31, then 32..63 (shared)
     float *vto;               // [6][32] odd runs (shared)
     float *coef;              // [64] (shared)
     uint32_t vto_s;           // shared-window address of vto (128-byte aligned)
@@ -74,18 +74,18 @@ __device__ __forceinline__ uint32_t *aligned_smem(uint32_t *raw) {
 __device__ __forceinline__ Sweep sweep_at(uint32_t *base) {
     Sweep s;
     s.zq = reinterpret_cast<uint2 *>(base);
-    s.zh = s.zq + kMaxBlocks;
-    s.vto = reinterpret_cast<float *>(s.zh + 32 * kMaxKChunks);
+    s.zh = reinterpret_cast<uint32_t *>(s.zq + kMaxBlocks);
+    s.vto = reinterpret_cast<float *>(s.zh + 64 * kMaxKChunks);
     s.coef = s.vto + 32 * (kMaxRuns - kShflRuns);
     s.vto_s = smem_u32(s.vto);
     return s;
 }
 
-// Byte offsets (x8, for uint2 tables) of the 5-bit chunks of kappa = inv(iota).
-__device__ __forceinline__ uint32_t kappa_offsets8(uint32_t kappa) {
+// Byte offsets (x4, for 32-bit tables) of the 5-bit chunks of kappa = inv(iota).
+__device__ __forceinline__ uint32_t kappa_offsets4(uint32_t kappa) {
     uint32_t off = 0;
 #pragma unroll
-    for (int k = 0; k < kMaxKChunks; ++k) off |= (((kappa >> (5 * k)) & 31u) * 8u) << (8 * k);
+    for (int k = 0; k < kMaxKChunks; ++k) off |= (((kappa >> (5 * k)) & 31u) * 4u) << (8 * k);
     return off;
 }
 
@@ -134,7 +134,8 @@ __device__ __forceinline__ void sweep_build_signs(uint32_t ca, uint32_t cb, int 
                 acc.y ^= xb;
             }
         }
-        s.zh[k * 32 + lane] = acc;
+        s.zh[k * 64 + lane] = acc.x;
+        s.zh[k * 64 + 32 + lane] = acc.y;
     }
 }
 
@@ -160,16 +161,18 @@ __device__ __forceinline__ void sweep_build_values(Sweep &s) {
     }
 }
 
-// Z(iota) of a sweep; koff = kappa_offsets8(inv iota), zq = ZQ(iota >> 5).
+// Z(iota) of a sweep; koff = kappa_offsets4(inv iota), zq = ZQ(iota >> 5).
+// Each half of a ZH entry is its own 32-word table, so that a lookup of
+// random entries by the 32 lanes is free of bank conflicts.
 template <int NKC>
 __device__ __forceinline__ uint2 sweep_signs(const Sweep &s, uint2 zq, uint32_t koff) {
     const char *zh = reinterpret_cast<const char *>(s.zh);
     uint2 z = make_uint2(s.zl.x ^ zq.x, s.zl.y ^ zq.y);
 #pragma unroll
     for (int k = 0; k < NKC; ++k) {
-        const uint2 h = *reinterpret_cast<const uint2 *>(zh + k * 256 + __byte_perm(koff, 0, 0x4440 + k));
-        z.x ^= h.x;
-        z.y ^= h.y;
+        const uint32_t o = __byte_perm(koff, 0, 0x4440 + k);
+        z.x ^= *reinterpret_cast<const uint32_t *>(zh + k * 256 + o);
+        z.y ^= *reinterpret_cast<const uint32_t *>(zh + k * 256 + 128 + o);
     }
     return z;
 }
@@ -339,7 +342,7 @@ __device__ __forceinline__ void sweep_accumulate_runs(const Sweep &s, float *out
 
 // out[i] += scale * sum_e coef_e (-1)^{parity(M[i] AND c_e)} over n codes
 // (indices c, coefficients coef), 64 codes per sweep. koff[i] holds the
-// packed chunk offsets of inv(i) (kappa_offsets8).
+// packed chunk offsets of inv(i) (kappa_offsets4).
 template <int NKC, SweepShape SHAPE = kSweepWide>
 __device__ __forceinline__ void synthesise(Sweep &s, const uint32_t *c, const float *coef, int n, int t, int d,
                                            const uint32_t *koff, float scale, float *out) {
@@ -363,7 +366,7 @@ __device__ __forceinline__ void synthesise(Sweep &s, const uint32_t *c, const fl
 
 // Packed chunk offsets of inv(i) = M[i] >> t for the block's coordinates.
 __device__ __forceinline__ void load_koff(const uint32_t *M, int d, int t, uint32_t *koff) {
-    for (int i = threadIdx.x; i < d; i += blockDim.x) koff[i] = kappa_offsets8(M[i] >> t);
+    for (int i = threadIdx.x; i < d; i += blockDim.x) koff[i] = kappa_offsets4(M[i] >> t);
     __syncthreads();
 }
 

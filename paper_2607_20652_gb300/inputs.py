@@ -76,6 +76,25 @@ def coset_generators(bits, levels: int, seed: int, max_children: int = 256) -> n
     return out
 
 
+def mixed_codes(T: int, d: int, m_bits: int, k: int, hashed_counts, seed: int):
+    """Codes idx int32 [T, k] and val float32 [T, k] ~ N(0, 1) in which token t
+    has hashed_counts[t % len] distinct entries in [d, 2^m_bits) and the rest
+    distinct entries below d (basis), in random order."""
+    g = rng(seed)
+    counts = list(hashed_counts)
+    idx = np.zeros((T, k), dtype=np.int32)
+    for t in range(T):
+        nh = counts[t % len(counts)]
+        if nh > k or k - nh > d:
+            raise ValueError("a code of %d entries cannot hold %d hashed ones at d = %d" % (k, nh, d))
+        ids = np.concatenate([g.choice(d, k - nh, replace=False),
+                              d + g.choice((1 << m_bits) - d, nh, replace=False)])
+        g.shuffle(ids)
+        idx[t] = ids
+    val = g.standard_normal((T, k), dtype=np.float32)
+    return idx, val
+
+
 def moment_tables(m: int, seed: int, mean_scale: float = 0.2, sigma_range=(0.5, 2.0)):
     """Standardisation tables (mu, sigma) fp32 [m]: mu ~ N(0, mean_scale^2),
     sigma uniform in sigma_range."""
