@@ -263,10 +263,18 @@ dpb_status dpb_stats_update(const dpb_plan *plan, double *acc, float alpha, floa
                             void *stream);
 
 /*
- * dpb_forward -- dpb_encode then dpb_decode of the same rows in one call
- * (two kernels on `stream`; the code is written out, as the backward needs
- * it). Arguments as in those two calls; xnorm is required when the plan has
- * norm_match. Errors: those of either call.
+ * dpb_forward -- the layer's forward pass: the §2.2 encoder (dpb_encode) and
+ * then the §2.1 decoder with on-chip signs (Eq. 1-2, App. A.4 Eq. 26-27;
+ * dpb_decode) over the same T rows, as two kernels on `stream`.
+ *   x, mu, sigma, idx, val, xnorm  as in dpb_encode (device; idx/val [T, k]
+ *                                  are written, as the backward needs them;
+ *                                  xnorm [T] is required with norm_match)
+ *   y                              [T, d] in the plan's dtype (device, out)
+ *   r_out                          optional fp32 [T, d] r before norm matching
+ *                                  (device, out; NULL to skip), as in dpb_decode
+ * The caller owns every buffer; the workspace is that of dpb_encode.
+ * Errors: those of either call (the decode is not launched when the encode
+ * fails).
  */
 dpb_status dpb_forward(const dpb_plan *plan, const void *x, int64_t T, const float *mu, const float *sigma,
                        int32_t *idx, float *val, float *xnorm, void *y, float *r_out, void *workspace,
