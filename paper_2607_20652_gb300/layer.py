@@ -1,7 +1,7 @@
 """The DPB as a PyTorch layer: autograd around the C-ABI calls.
 
-Forward runs dpb_encode then dpb_decode (the code and the decode's r are
-kept for the backward); backward runs dpb_backward, the gradient with the
+Forward runs dpb_forward, i.e. dpb_encode then dpb_decode (the code and the
+decode's r are kept for the backward); backward runs dpb_backward, the gradient with the
 selected set held fixed. The layer has no trainable parameters: its dictionary is the
 parity construction (§2.1). With ``ema`` set, the layer keeps live
 standardisation tables (§2.2 "Score Standardization"): forward adds the
@@ -27,9 +27,8 @@ class _DPBFunction(torch.autograd.Function):
         ws = layer._workspace(T, x.device)
         stream = torch.cuda.current_stream(x.device)
         ev = layer._events("forward")
-        idx, val, xn = dpb.encode(layer.plan, x, layer.mu, layer.sigma, workspace=ws, stream=stream)
         r = torch.empty((T, layer.d), dtype=torch.float32, device=x.device)  # kept for the backward
-        y = dpb.decode(layer.plan, idx, val, xn, workspace=ws, stream=stream, r_out=r)
+        idx, val, xn, y = dpb.forward(layer.plan, x, layer.mu, layer.sigma, workspace=ws, stream=stream, r_out=r)
         if layer.ema is not None and layer.training:
             rows = dpb.sample_rows(T, layer.ema_rows, layer._gen, x.device)
             dpb.stats_accumulate(layer.plan, x, rows, layer._acc, mu=layer.mu, sigma=layer.sigma, workspace=ws,
