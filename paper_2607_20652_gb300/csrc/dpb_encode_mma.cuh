@@ -826,6 +826,15 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
                             ((acc[0][0][h][r] + acc[0][1][h][r]) + (acc[1][0][h][r] + acc[1][1][h][r])) * a.inv_sqrt_d;
             }
             const uint32_t *gl = s_g + l * 16;
+            if (a.mu) {  // standardise both rows' children now: their table loads go out together
+#pragma unroll
+                for (int tk = 0; tk < 2; ++tk)
+#pragma unroll
+                    for (int e = 0; e < 4; ++e)
+                        if (tk < nhalf)
+                            sc[tk][e] = standardise(sc[tk][e], (tk ? p1 : p0) ^ gl[8 * (e >> 1) + 2 * q4 + (e & 1)],
+                                                    a, a.status);
+            }
             const uint32_t *ddl = s_dd + (l - 1) * kDedupSlots * 2;
             uint32_t pcur = p0;
             if constexpr (WIDE) {
@@ -913,7 +922,7 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
                     const uint32_t ci = pcur ^ gl[8 * (e >> 1) + 2 * q4 + (e & 1)];
-                    const float z = standardise(sc[0][e], ci, a, a.status);
+                    const float z = sc[0][e];  // standardised above
                     // (WIDE: tk is the half of the beam; otherwise the token)
                     c[e] = ((dmask >> e) & 1u) || (WIDE ? 8 * tk + slot : slot) >= a.beam ? 0ull : cword(z, ci);
                     sc[0][e] = sc[1][e];
