@@ -27,11 +27,14 @@
 // DPB_DEV_TIMEOUT, and the block drains its MMAs and frees its TMEM.
 //
 // Selection of a level (one warp per token, lane = parent slot): each lane
-// keeps the 4 largest keys |z| of its row, the warp sorts the union and takes
-// a threshold tau at rank K + K/2 of it; every candidate at or above tau is
-// gathered (a count pass, a prefix sum and a write pass), sorted, and its
-// repeated indices (two parents can share a child) are dropped. When K
-// distinct candidates reach tau they are exactly the level's top K.
+// keeps the 4 largest of its row's group maxima (the largest key |z| of each
+// 8 consecutive children; every key at level 0), the warp sorts the union and
+// takes a threshold tau at rank K + K/2 of its distinct keys. Each of those
+// keys is a candidate's, so at least K + K/2 distinct candidates reach tau.
+// Every candidate at or above tau is gathered (one pass with running ballot
+// positions), sorted, and its repeated indices (two parents can share a
+// child) are dropped. When K distinct candidates reach tau they are exactly
+// the level's top K.
 #include <algorithm>
 
 #include "dpb_encode_mma.cuh"
@@ -252,8 +255,9 @@ __device__ __forceinline__ int sort_keep(int n, int K, const WarpBufs &w, const 
 }
 
 // The top K distinct candidates of one token, as explained in the header.
-// `scan(f)` calls f(z, index, live) for every candidate of this lane, in the
-// same order each time and in step across the warp. Writes code columns
+// `scan(f)` calls f(z, index, live, gend) for every candidate of this lane, in
+// the same order each time and in step across the warp; gend marks the last
+// candidate of a group. Writes code columns
 // [col, col + K) of row `tok` and, when `par_out`, the kept indices as the
 // next level's parents. Returns the number of distinct candidates kept
 // (< K only with the status bit set).
@@ -261,47 +265,62 @@ template <class Scan>
 __device__ __forceinline__ int select_level(Scan scan, int nlive, int K, const WarpBufs &w, const Args &a,
                                             int64_t tok, int col, bool par_out) {
     const int lane = threadIdx.x & 31;
-    uint32_t top[4] = {0u, 0u, 0u, 0u};
-    scan([&](float z, uint32_t, bool live) {
-        uint32_t c = live ? akey(z) + 1u : 0u;
-#pragma unroll
-        for (int r = 0; r < 4; ++r) {
-            const uint32_t hi = max(top[r], c);
-            c = min(top[r], c);
-            top[r] = hi;
-        }
-    });
-    mmaenc::warp_sort_desc<4>(top);
-    // distinct keys of the sorted union (copies of one child share a key):
-    // drank[r] = rank among them, 0 for a repeat or an empty slot
+    uint32_t top[4];
     int drank[4];
-    {
-        uint32_t prev = __shfl_up_sync(kFull, top[3], 1);
-        int cnt = 0;
-        bool first[4];
-#pragma unroll
-        for (int r = 0; r < 4; ++r) {
-            first[r] = top[r] != 0u && ((r == 0 && lane == 0) || top[r] != prev);
-            prev = top[r];
-            cnt += first[r];
-        }
-        int base = cnt;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int t = __shfl_up_sync(kFull, base, o);
-            if (lane >= o) base += t;
-        }
-        base -= cnt;
-#pragma unroll
-        for (int r = 0; r < 4; ++r) {
-            drank[r] = first[r] ? base + 1 : 0;
-            base += first[r];
-        }
-    }
     int nd = 0;  // distinct keys in the union
+    // Group maxima first; when they hold fewer than K distinct keys (rows of
+    // few children, or copies), every candidate's key instead.
+#pragma unroll 1
+    for (int pass = 0; pass < 2; ++pass) {
+        const bool group = pass == 0;
 #pragma unroll
-    for (int r = 0; r < 4; ++r) nd = max(nd, drank[r]);
-    nd = __reduce_max_sync(kFull, (uint32_t)nd);
+        for (int r = 0; r < 4; ++r) top[r] = 0u;
+        uint32_t gm = 0u;  // the largest key of the current group
+        scan([&](float z, uint32_t, bool live, bool gend) {
+            gm = max(gm, live ? akey(z) + 1u : 0u);
+            if (gend || !group) {
+                uint32_t c = gm;
+                gm = 0u;
+#pragma unroll
+                for (int r = 0; r < 4; ++r) {
+                    const uint32_t hi = max(top[r], c);
+                    c = min(top[r], c);
+                    top[r] = hi;
+                }
+            }
+        });
+        mmaenc::warp_sort_desc<4>(top);
+        // distinct keys of the sorted union (copies of one child share a key):
+        // drank[r] = rank among them, 0 for a repeat or an empty slot
+        {
+            uint32_t prev = __shfl_up_sync(kFull, top[3], 1);
+            int cnt = 0;
+            bool first[4];
+#pragma unroll
+            for (int r = 0; r < 4; ++r) {
+                first[r] = top[r] != 0u && ((r == 0 && lane == 0) || top[r] != prev);
+                prev = top[r];
+                cnt += first[r];
+            }
+            int base = cnt;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int t = __shfl_up_sync(kFull, base, o);
+                if (lane >= o) base += t;
+            }
+            base -= cnt;
+#pragma unroll
+            for (int r = 0; r < 4; ++r) {
+                drank[r] = first[r] ? base + 1 : 0;
+                base += first[r];
+            }
+        }
+        nd = 0;
+#pragma unroll
+        for (int r = 0; r < 4; ++r) nd = max(nd, drank[r]);
+        nd = (int)__reduce_max_sync(kFull, (uint32_t)nd);
+        if (nd >= K) break;
+    }
     (void)nlive;
     int distinct = 0;
     // tau = the union's distinct key of rank K + K/2 (so that at least that many
@@ -317,7 +336,7 @@ __device__ __forceinline__ int select_level(Scan scan, int nlive, int K, const W
         // gather every candidate at or above tau, warp-interleaved in scan
         // order (one pass: positions come from the running ballot counts)
         int n = 0;
-        scan([&](float z, uint32_t ci, bool live) {
+        scan([&](float z, uint32_t ci, bool live, bool) {
             const bool take = live && akey(z) + 1u >= tau;
             const unsigned mb = __ballot_sync(kFull, take);
             if (mb) {  // rare: most candidates fall short of tau
@@ -437,7 +456,7 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
                 for (int i = lane; i < d; i += 32) {
                     const int m = i >> 5, wl = i & 31;
                     const float xv = __uint_as_float((uint32_t)xh[(m * 16 + (wl & 15)) * 2 + (wl >> 4)] << 16);
-                    f(standardise(xv, (uint32_t)i, a, nullptr), (uint32_t)i, true);
+                    f(standardise(xv, (uint32_t)i, a, nullptr), (uint32_t)i, true, true);
                 }
             };
             if (a.mu)
@@ -620,7 +639,7 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
 #pragma unroll
                         for (int j = 0; j < 32; ++j) {
                             const uint32_t ci = p ^ gl[c0 + j];
-                            f(__uint_as_float(v[j]) * scale, ci, rv && c0 + j < D);
+                            f(__uint_as_float(v[j]) * scale, ci, rv && c0 + j < D, (j & 7) == 7);
                         }
                     }
                 };
