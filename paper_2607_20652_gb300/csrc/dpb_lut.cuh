@@ -54,7 +54,11 @@ __device__ __forceinline__ uint32_t smem_u32(const void *p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
 
-// fp32 load from shared memory at byte address addr + OFF.
+// fp32 load from shared memory at byte address addr + OFF (a 32-bit
+// shared-window address the caller composed by OR or byte permute, with the
+// offset as an immediate). Every table read this way was written before a
+// __syncwarp() of the same warp; the asm is volatile, so the compiler keeps it
+// after that barrier.
 template <int OFF>
 __device__ __forceinline__ float lds_f32(uint32_t addr) {
     float v;
