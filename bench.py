@@ -142,7 +142,11 @@ def roofline_for(name: str, work: dict, seconds: float, peaks: dict, src: str, t
     else:
         achieved, peak, unit = achieved / 1e12, rate["int"] / 1e12, "Tops/s"
         psrc = "152 SMs x 64 LOP3/clock x max SM clock"
-    return {"kernel": name, "bound": bound, "achieved": round(achieved, 3), "peak": round(peak, 3),
+    # integer logic and FP32 adds are both plain ALU arithmetic ("alu"); "pipe"
+    # says which of the two peaks the fraction is taken against
+    return {"kernel": name, "bound": "alu" if bound == "int" else bound,
+            "pipe": {"alu": "fp32", "int": "integer logic"}.get(bound),
+            "achieved": round(achieved, 3), "peak": round(peak, 3),
             "unit": unit, "frac": round(achieved / peak, 4), "traffic": traffic,
             "algorithmic_bytes": int(work["bytes"]),
             "peak_source": f"{src} ({psrc})",
@@ -451,7 +455,7 @@ def run_ours(args, world, rank, local):
     dom = max(kern_ms, key=kern_ms.get)
     roof = roofline_for(dom, work[dom], kern_ms[dom] / 1e3, peaks, src, measured_traffic(dom, T))
     kernels = {n: {"ms": round(v, 4), **{kk: vv for kk, vv in roofline_for(n, work[n], v / 1e3, peaks, src).items()
-                                          if kk in ("bound", "frac", "t_roofline_us")}}
+                                          if kk in ("bound", "pipe", "frac", "t_roofline_us")}}
                for n, v in kern_ms.items()}
     step_roof_us = sum(kernels[n]["t_roofline_us"] for n in kernels)
 
@@ -648,7 +652,7 @@ def run_per_level(args, world, rank, local):
     if std:
         work["stats"] = {"bytes": T * d * 2 + 8 * plan.n_features}
     kernels = {n: {"ms": round(v, 4), **{kk: vv for kk, vv in roofline_for(n, work[n], v / 1e3, peaks, src).items()
-                                          if kk in ("bound", "frac", "t_roofline_us", "achieved", "unit")}}
+                                          if kk in ("bound", "pipe", "frac", "t_roofline_us", "achieved", "unit")}}
                for n, v in kern_ms.items()}
     dom = max(kern_ms, key=kern_ms.get)
     line = {

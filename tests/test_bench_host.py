@@ -61,11 +61,11 @@ def test_roofline_arithmetic():
     # encode: 24,576 sign applications per token at 152 x 64 logic ops per clock
     # bind before its 786,432 tensor flops at 1714.8 TFLOP/s
     r = bench.roofline_for("encode", work["encode"], 200e-6, peaks, "measured")
-    assert r["bound"] == "int" and abs(r["peak"] - 152 * 64 * 2070e6 / 1e12) < 1e-3
+    assert r["bound"] == "alu" and r["pipe"] == "integer logic" and abs(r["peak"] - 152 * 64 * 2070e6 / 1e12) < 1e-3
     assert abs(r["frac"] - work["encode"]["int_ops"] / 200e-6 / (152 * 64 * 2070e6)) < 1e-3
     assert abs(r["t_roofline_us"] - 1e6 * work["encode"]["int_ops"] / (152 * 64 * 2070e6)) < 0.01
     r = bench.roofline_for("decode", work["decode"], 100e-6, peaks, "measured")
-    assert r["bound"] == "alu" and abs(r["peak"] - 152 * 128 * 2070e6 / 1e12) < 1e-3
+    assert r["bound"] == "alu" and r["pipe"] == "fp32" and abs(r["peak"] - 152 * 128 * 2070e6 / 1e12) < 1e-3
     # a pure-HBM call picks the copy bandwidth
     r = bench.roofline_for("copy", {"bytes": 6781.4e9 * 1e-3}, 2e-3, peaks, "measured")
     assert r["bound"] == "hbm" and abs(r["frac"] - 0.5) < 1e-6 and r["unit"] == "GB/s"
