@@ -37,6 +37,7 @@ EMA_ALPHA = 0.01       # EMA weight of one batch
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
                   "sm_max_mhz": 2070.0}
 GB300_SMS = 152
+NOMINAL_HBM_GBS = 7900.0  # GB300 HBM3e, nominal (the measured copy rate is the roofline's peak)
 FP32_LANES_PER_SM = 128   # FADD/FFMA per SM per clock (measured; packed f32x2 gave no more)
 INT_LOGIC_PER_SM = 64     # LOP3 per SM per clock (measured)
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic_wide_T65536.txt")
@@ -142,9 +143,10 @@ def roofline_for(name: str, work: dict, seconds: float, peaks: dict, src: str, t
     else:
         achieved, peak, unit = achieved / 1e12, rate["int"] / 1e12, "Tops/s"
         psrc = "152 SMs x 64 LOP3/clock x max SM clock"
+    extra = {"frac_nominal": round(achieved / NOMINAL_HBM_GBS, 4)} if bound == "hbm" else {}
     # integer logic and FP32 adds are both plain ALU arithmetic ("alu"); "pipe"
     # says which of the two peaks the fraction is taken against
-    return {"kernel": name, "bound": "alu" if bound == "int" else bound,
+    return {**extra, "kernel": name, "bound": "alu" if bound == "int" else bound,
             "pipe": {"alu": "fp32", "int": "integer logic"}.get(bound),
             "achieved": round(achieved, 3), "peak": round(peak, 3),
             "unit": unit, "frac": round(achieved / peak, 4), "traffic": traffic,

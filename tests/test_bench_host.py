@@ -69,3 +69,4 @@ def test_roofline_arithmetic():
     # a pure-HBM call picks the copy bandwidth
     r = bench.roofline_for("copy", {"bytes": 6781.4e9 * 1e-3}, 2e-3, peaks, "measured")
     assert r["bound"] == "hbm" and abs(r["frac"] - 0.5) < 1e-6 and r["unit"] == "GB/s"
+    assert abs(r["frac_nominal"] - 6781.4 / 2 / 7900.0) < 1e-4  # and the nominal 7.9 TB/s beside it
