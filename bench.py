@@ -103,6 +103,13 @@ def load_peaks():
         return dict(FALLBACK_PEAKS), "fallback"
 
 
+def sign_ops(signs: int, s: int) -> float:
+    """Integer-logic operations that apply `signs` sign flips to stored
+    elements of s bytes: a bf16 pair shares one 32-bit word, so one LOP3
+    (XOR with the masked sign bits) flips two; an fp32 element takes one."""
+    return signs / 2 if s == 2 else float(signs)
+
+
 def algorithmic_work(cfg: dict, T: int, k_hash: float, s: int):
     """Per-launch algorithmic bytes and operations of each call (the method's
     own sums, not implementation overhead). s = bytes per stored element;
@@ -111,22 +118,33 @@ def algorithmic_work(cfg: dict, T: int, k_hash: float, s: int):
     mma = sum(2 * B * cfg["children"][l] * d for l in range(1, cfg["levels"]))
     signs = (cfg["levels"] - 1) * B * d  # the x (.) phi~_p products of Eq. 6
     return {
-        "encode": {"bytes": T * (d * s + 8 * k + 4), "tensor_flops": T * mma, "int_ops": T * signs},
+        "encode": {"bytes": T * (d * s + 8 * k + 4), "tensor_flops": T * mma, "int_ops": T * sign_ops(signs, s)},
         "decode": {"bytes": T * (8 * k + 4 + d * s), "fp_ops": T * (k_hash * d + 3 * d)},
         "backward": {"bytes": T * (3 * d * s + 12 * k), "fp_ops": T * (2 * k_hash * d + 6 * d)},
     }
 
 
-def peak_rates(peaks: dict):
+def alu_clock(peaks: dict, clocks: dict | None):
+    """SM clock (MHz) for the ALU peaks: the median sampled while the kernels
+    ran, else the maximum SM clock; and a note saying which."""
+    if clocks and clocks.get("sm_mhz"):
+        return float(clocks["sm_mhz"]), f"median SM clock sampled under load, {clocks['sm_mhz']:.0f} MHz"
     mhz = peaks.get("sm_max_mhz", 2070.0)
+    return float(mhz), f"maximum SM clock {mhz:.0f} MHz (no clock samples)"
+
+
+def peak_rates(peaks: dict, mhz: float | None = None):
+    mhz = mhz or peaks.get("sm_max_mhz", 2070.0)
     return {"hbm": peaks["hbm_gbs"] * 1e9, "tensor": peaks["bf16_tflops_sustained"] * 1e12,
             "alu": GB300_SMS * FP32_LANES_PER_SM * mhz * 1e6, "int": GB300_SMS * INT_LOGIC_PER_SM * mhz * 1e6}
 
 
-def roofline_for(name: str, work: dict, seconds: float, peaks: dict, src: str, traffic=None):
+def roofline_for(name: str, work: dict, seconds: float, peaks: dict, src: str, traffic=None, clocks=None):
     """The slowest of the call's terms at peak (HBM bytes, tensor flops, FP32
-    adds, integer logic ops) is its roofline; achieved = that term's work / time."""
-    rate = peak_rates(peaks)
+    adds, integer logic ops) is its roofline; achieved = that term's work / time.
+    The ALU peaks are taken at the SM clock sampled during the run."""
+    mhz, clk_note = alu_clock(peaks, clocks)
+    rate = peak_rates(peaks, mhz)
     keys = {"hbm": "bytes", "tensor": "tensor_flops", "alu": "fp_ops", "int": "int_ops"}
     terms = {b: work[kk] / rate[b] for b, kk in keys.items() if kk in work}
     bound = max(terms, key=terms.get)
@@ -139,10 +157,11 @@ def roofline_for(name: str, work: dict, seconds: float, peaks: dict, src: str, t
         psrc = "bf16 sustained"
     elif bound == "alu":
         achieved, peak, unit = achieved / 1e12, rate["alu"] / 1e12, "TFLOP/s"
-        psrc = "152 SMs x 128 FP32 adds/clock x max SM clock"
+        psrc = f"152 SMs x 128 FP32 adds/clock x {clk_note}"
     else:
         achieved, peak, unit = achieved / 1e12, rate["int"] / 1e12, "Tops/s"
-        psrc = "152 SMs x 64 LOP3/clock x max SM clock"
+        psrc = (f"152 SMs x 64 LOP3/clock x {clk_note}; one LOP3 flips the signs of a packed bf16 pair, "
+                "so the work is half the sign applications")
     extra = {"frac_nominal": round(achieved / NOMINAL_HBM_GBS, 4)} if bound == "hbm" else {}
     # integer logic and FP32 adds are both plain ALU arithmetic ("alu"); "pipe"
     # says which of the two peaks the fraction is taken against
@@ -263,11 +282,12 @@ def make_inputs_gpu(w, plan, seed, device):
                    beam=w["beam"], k=w["k"], dtype="f32", norm_match=0)
     y = dpb.decode(syn, torch.from_numpy(idx_true).to(device),
                    torch.from_numpy(tree.coef.astype(np.float32)).to(device))
-    noise = torch.from_numpy(inputs.normal((T, d), seed + 1000, w["noise"])).to(device)
-    x = (y + noise).to(torch.bfloat16).contiguous()
-    gy = torch.from_numpy(inputs.normal((T, d), seed + w["grad_seed"])).to(device).to(torch.bfloat16)
+    noise_h = inputs.normal((T, d), seed + 1000, w["noise"])
+    x = (y + torch.from_numpy(noise_h).to(device)).to(torch.bfloat16).contiguous()
+    gy_h = inputs.to_bf16(inputs.normal((T, d), seed + w["grad_seed"]))
+    gy = torch.from_numpy(gy_h).to(device).to(torch.bfloat16)
     torch.cuda.synchronize(device)
-    return x, gy, idx_true
+    return x, gy, idx_true, {"tree": tree, "noise": noise_h, "gy": gy_h}
 
 
 def oracle_sample(w, n_tokens, seed):
@@ -282,6 +302,63 @@ def oracle_sample(w, n_tokens, seed):
     x = inputs.to_bf16((clean + inputs.normal((n_tokens, w["d"]), seed + 1000, w["noise"])).astype(np.float32))
     gy = inputs.to_bf16(inputs.normal((n_tokens, w["d"]), seed + w["grad_seed"]))
     return ref, x.astype(np.float64), gy.astype(np.float64)
+
+
+PARITY_ROWS = 256  # sampled tokens of the timed batch checked against the oracle
+
+
+def parity_rows(w, host, T, seed):
+    """Oracle leg, before timing: a seeded sample of rows of the timed batch
+    and their x built by the oracle alone (its own generator table and decode
+    of the planted code, plus the same noise), which then replace those rows
+    on the GPU, so that no input of the check comes from the CUDA path."""
+    import oracle
+    from paper_2607_20652_gb300 import inputs
+    ref = oracle.resolve(d=w["d"], m_bits=w["m_bits"], levels=w["levels"], children=w["children"],
+                         beam=w["beam"], k=w["k"])
+    rows = np.unique(np.concatenate([inputs.sample_rows(T, PARITY_ROWS, seed + 77), [0, T - 1]]))
+    idx_true = compose(host["tree"], ref.G, w["levels"])[rows]
+    clean = oracle.decode(ref, idx_true, host["tree"].coef[rows], norm_match=0)
+    x_rows = inputs.to_bf16((clean + host["noise"][rows]).astype(np.float32))
+    return ref, rows, x_rows
+
+
+def parity_check(ref, rows, x_rows, gy_rows, out):
+    """Oracle leg, after timing: the sampled rows' outputs of the last timed
+    step against the oracle, by the rules of the -m gpu parity tests (codes as
+    sets with near-ties counted, decode / r / gradients element by element on
+    the GPU's own code)."""
+    import oracle
+    from tests import parity
+    tol = parity.TOL["bf16"]
+    xr = x_rows.astype(np.float64)
+    gi, gvl, gxn = out["idx"], out["val"], out["xnorm"]
+    res = {"tokens": int(len(rows)), "sample": f"{len(rows)} seeded rows of the timed batch (oracle-built x)",
+           "rule": "indices as sets except near-ties (gap < 1e-5 relative, counted); val within 1e-5 |x|; "
+                   "y, grad_x within 2e-2 max(|ref_i|, row rms) + 1 bf16 spacing, r and grad_val within 1e-5, "
+                   "element by element, decode and backward on the GPU's own code"}
+    try:
+        idx_o, val_o, xn_o, gap = oracle.encode(ref, xr)
+        parity.check_code_order(gi, gvl)
+        near, worst_val = parity.compare_codes(gi, gvl, idx_o, val_o, gap, xn_o)
+        res.update(near_ties=near, near_tie_tokens=[int(r) for r in np.asarray(rows)[gap < parity.NEAR_TIE]][:16],
+                   val_err=worst_val)
+        assert np.all(np.abs(gxn - xn_o) <= 1e-5 * np.maximum(xn_o, 1e-30)), "|x| differs"
+        y_o = oracle.decode(ref, gi, gvl.astype(np.float64), gxn.astype(np.float64))
+        res["y_err"] = parity.check_elementwise(out["y"], y_o, tol, True, "decode y")
+        if out.get("r") is not None:
+            r_o = oracle.decode(ref, gi, gvl.astype(np.float64), norm_match=0)
+            res["r_err"] = parity.check_elementwise(out["r"], r_o, 1e-5, False, "kept r")
+        gx_o, gv_o = oracle.backward(ref, xr, gi, gvl.astype(np.float64), gy_rows.astype(np.float64))
+        res["gx_err"] = parity.check_elementwise(out["gx"], gx_o, tol, True, "grad_x")
+        res["gv_err"] = parity.check_elementwise(out["gv"], gv_o, 1e-5, False, "grad_val")
+        res["ok"] = True
+    except AssertionError as e:
+        res.update(ok=False, failure=str(e)[:300])
+    for kk in ("val_err", "y_err", "r_err", "gx_err", "gv_err"):
+        if kk in res:
+            res[kk] = float(f"{res[kk]:.3e}")
+    return res
 
 
 def time_oracle(ref, x, gy):
@@ -363,14 +440,12 @@ def run_reference(args, world, rank):
     return 0
 
 
-def config_block(w, world, n_tokens=None, standardise=False, keep_r=False):
+def config_block(w, world, n_tokens=None, standardise=False):
     c = {"workload": WORKLOAD, "T_per_gpu": n_tokens or w["T"], "d": w["d"], "features": 2 ** w["m_bits"],
          "levels": w["levels"], "children": w["children"], "beam": w["beam"], "k": w["k"],
          "accumulate": "fp32", "inputs": "planted tree of 64 parity directions + N(0,0.1^2), bf16",
          "l2": "working set ~450 MB > 129 MB L2 (no flush needed)",
          "parallelism": f"dp{world} (independent token shards)"}
-    if keep_r:
-        c["r_kept"] = "decode keeps r (fp32 [T, d]) for the backward"
     if standardise:
         c["standardise"] = {"tables": "live fp32 mu/sigma (2^N each)", "ema_sample_rows": EMA_SAMPLE,
                             "ema_alpha": EMA_ALPHA,
@@ -400,7 +475,14 @@ def run_ours(args, world, rank, local):
                        scoring=dpb.SCORING_COSET_WHT if args.coset == "wht" else dpb.SCORING_CONTRACTION)
     plan = dpb.Plan(**plan_kw)
     seed = shard_seed(w["seed"], rank)
-    x, gy, idx_true = make_inputs_gpu(w, plan, seed, device)
+    x, gy, idx_true, host = make_inputs_gpu(w, plan, seed, device)
+    # oracle leg: seeded rows of the batch rebuilt by the oracle alone, checked after timing
+    check = rank == 0 and world == 1 and not args.no_parity and not std and not args.coset
+    if check:
+        pref, prows, px = parity_rows(w, host, T, seed)
+        x[torch.from_numpy(prows).to(device)] = torch.from_numpy(px).to(device).to(torch.bfloat16)
+        pgy = host["gy"][prows]
+    del host
     k = plan.code_len
     idx = torch.empty((T, k), dtype=torch.int32, device=device)
     val = torch.empty((T, k), dtype=torch.float32, device=device)
@@ -439,7 +521,8 @@ def run_ours(args, world, rank, local):
         if ev:
             ev[3].record(stream)
         if std:
-            dpb.stats_step(plan, x, mu_t, sg_t, EMA_ALPHA, samples[i], acc=acc, workspace=ws, stream=stream)
+            dpb.stats_step(plan, x, mu_t, sg_t, EMA_ALPHA, samples[i % len(samples)], acc=acc, workspace=ws,
+                           stream=stream)
             if ev:
                 ev[4].record(stream)
 
@@ -467,8 +550,25 @@ def run_ours(args, world, rank, local):
     end.record(stream)
     torch.cuda.synchronize(device)
     barrier(world)
-    clk = clocks.stop()
     ms = start.elapsed_time(end)
+    # A timed region shorter than the clock window is followed by the same
+    # step for the rest of the window, so that the sampler (200 ms period)
+    # sees the clock these kernels run at; its per-kernel times are reported
+    # beside the timed ones.
+    sustained = None
+    if ms < 1e3 * args.clock_seconds:
+        n_more = max(1, int((1e3 * args.clock_seconds - ms) / max(ms / args.steps, 1e-3)))
+        sev = [[torch.cuda.Event(enable_timing=True) for _ in range(len(stages) + 1)] for _ in range(n_more)]
+        for i in range(n_more):
+            step(sev[i], args.steps + i)
+        torch.cuda.synchronize(device)
+        sustained = {"steps": n_more, "ms_per_step": round(sum(e[0].elapsed_time(e[-1]) for e in sev) / n_more, 4),
+                     "kernels_ms": {n: round(statistics.mean(e[j].elapsed_time(e[j + 1]) for e in sev), 4)
+                                    for j, n in enumerate(stages)}}
+    clk = clocks.stop()
+    clk["window"] = ("the timed steps" if sustained is None else
+                     f"the timed steps and {sustained['steps']} more of the same step right after "
+                     f"({args.clock_seconds:.1f} s in all)")
     ms_max = max_over_ranks(ms, world, device)
     kern_ms = {n: statistics.mean(e[j].elapsed_time(e[j + 1]) for e in evs) for j, n in enumerate(stages)}
     if std:
@@ -484,11 +584,20 @@ def run_ours(args, world, rank, local):
         # the column pass reads x once; the update scans the 2^N counts
         work["stats"] = {"bytes": T * d * 2 + 8 * plan.n_features}
     dom = max(kern_ms, key=kern_ms.get)
-    roof = roofline_for(dom, work[dom], kern_ms[dom] / 1e3, peaks, src, measured_traffic(dom, T))
-    kernels = {n: {"ms": round(v, 4), **{kk: vv for kk, vv in roofline_for(n, work[n], v / 1e3, peaks, src).items()
-                                          if kk in ("bound", "pipe", "frac", "t_roofline_us")}}
+    roof = roofline_for(dom, work[dom], kern_ms[dom] / 1e3, peaks, src, measured_traffic(dom, T), clocks=clk)
+    kernels = {n: {"ms": round(v, 4), **{kk: vv for kk, vv in
+                                         roofline_for(n, work[n], v / 1e3, peaks, src, clocks=clk).items()
+                                         if kk in ("bound", "pipe", "frac", "t_roofline_us")}}
                for n, v in kern_ms.items()}
     step_roof_us = sum(kernels[n]["t_roofline_us"] for n in kernels)
+
+    par = None
+    if check:
+        pr = torch.from_numpy(prows).to(device)
+        out = {"idx": idx[pr].cpu().numpy(), "val": val[pr].cpu().numpy(), "xnorm": xn[pr].cpu().numpy(),
+               "y": y[pr].float().cpu().numpy(), "gx": gx[pr].float().cpu().numpy(), "gv": gv[pr].cpu().numpy(),
+               "r": None if rk is None else rk[pr].cpu().numpy()}
+        par = parity_check(pref, prows, px, pgy, out)
 
     # end to end through the public API with host buffers
     e2e = None
@@ -500,7 +609,7 @@ def run_ours(args, world, rank, local):
         "metric": METRIC, "value": round(value, 1), "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_max / args.steps, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-        "data": "synthetic", "config": {**config_block(w, world, standardise=std, keep_r=rk is not None),
+        "data": "synthetic", "config": {**config_block(w, world, standardise=std),
                                          **({"generators": "coset g0 ^ {0..15} per level (variant outside the paper)",
                                              "scoring": args.coset} if args.coset else {})},
         "roofline": roof,
@@ -508,8 +617,13 @@ def run_ours(args, world, rank, local):
                           "t_measured_us": round(1e3 * ms_max / args.steps, 2),
                           "frac": round(step_roof_us / (1e3 * ms_max / args.steps), 4)},
         "kernels": kernels, "k_hash": round(k_hash, 2), "planted_recovery": round(recovered, 4),
+        "r_kept": rk is not None,
         "gpu_launches": (3 + (3 if std else 0)) * args.steps, "clocks": clk, "device_status": status,
     }
+    if sustained:
+        line["sustained"] = sustained
+    if par is not None:
+        line["parity"] = par
     if e2e:
         line["e2e"] = e2e
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -573,7 +687,7 @@ def run_e2e(plan, x, gy, args, device, stream, world):
         for _ in range(max(1, args.warmup)):
             fn()
         torch.cuda.synchronize(device)
-        n = max(3, args.steps // 2)
+        n = max(3, min(args.steps // 2, 400))
         barrier(world)
         t0 = time.perf_counter()
         for _ in range(n):
@@ -604,7 +718,7 @@ def per_level_work(w, T: int, k_hash: float, s: int):
     mma = sum(2 * kl[l - 1] * ch[l] * d for l in range(1, w["levels"]))
     signs = sum(kl[l - 1] * d for l in range(1, w["levels"]))
     return {
-        "encode": {"bytes": T * (d * s + 8 * code + 4), "tensor_flops": T * mma, "int_ops": T * signs},
+        "encode": {"bytes": T * (d * s + 8 * code + 4), "tensor_flops": T * mma, "int_ops": T * sign_ops(signs, s)},
         "decode": {"bytes": T * (8 * code + 4 + d * s), "fp_ops": T * (k_hash * d + 3 * d)},
         "backward": {"bytes": T * (3 * d * s + 12 * code), "fp_ops": T * (2 * k_hash * d + 6 * d)},
     }
@@ -682,8 +796,9 @@ def run_per_level(args, world, rank, local):
     work = per_level_work(w, T, k_hash, 2)
     if std:
         work["stats"] = {"bytes": T * d * 2 + 8 * plan.n_features}
-    kernels = {n: {"ms": round(v, 4), **{kk: vv for kk, vv in roofline_for(n, work[n], v / 1e3, peaks, src).items()
-                                          if kk in ("bound", "pipe", "frac", "t_roofline_us", "achieved", "unit")}}
+    kernels = {n: {"ms": round(v, 4), **{kk: vv for kk, vv in
+                                         roofline_for(n, work[n], v / 1e3, peaks, src, clocks=clk).items()
+                                         if kk in ("bound", "pipe", "frac", "t_roofline_us", "achieved", "unit")}}
                for n, v in kern_ms.items()}
     dom = max(kern_ms, key=kern_ms.get)
     line = {
@@ -699,7 +814,7 @@ def run_per_level(args, world, rank, local):
                    "l2": "inputs (2 x 128 MiB) larger than the 129 MB L2 (no flush needed)",
                    **({"standardise": {"tables": "live fp32 mu/sigma (2^N each)", "ema_sample_rows": EMA_SAMPLE,
                                        "ema_alpha": EMA_ALPHA}} if std else {})},
-        "roofline": roofline_for(dom, work[dom], kern_ms[dom] / 1e3, peaks, src),
+        "roofline": roofline_for(dom, work[dom], kern_ms[dom] / 1e3, peaks, src, clocks=clk),
         "kernels": kernels, "k_hash": round(k_hash, 2), "gpu_launches": (3 + (3 if std else 0)) * args.steps,
         "clocks": clk,
         "device_status": dpb.workspace_status(ws),
@@ -723,6 +838,8 @@ def run_sweep(args, world, rank, local):
     peaks, src = load_peaks()
     points = []
     steps = max(3, args.steps // 4)
+    clocks = ClockSampler(None)
+    clocks.start()
     for w in configs.SWEEP:
         T, d = w["T"], w["d"]
         plan = dpb.Plan(d=d, levels=w["levels"], m_bits=w["m_bits"], children=w["children"], beam=w["beam"],
@@ -765,23 +882,26 @@ def run_sweep(args, world, rank, local):
         ms = max_over_ranks(sum(kern.values()), world, device)
         k_hash = float(np.mean(np.sum(idx.cpu().numpy() >= d, axis=1)))
         work = algorithmic_work(plan.config, T, k_hash, 2)
-        roofs = {n: roofline_for(n, work[n], kern[n] / 1e3, peaks, src) for n in kern}
-        step_roof = sum(r["t_roofline_us"] for r in roofs.values())
         points.append({"features": 2 ** w["m_bits"], "k": w["k"], "beam": w["beam"],
                        "encoder": "tensor-core" if w["beam"] <= 16 else "general",
                        "tokens_per_s": round(whole_job_rate(T, world, 1, ms / 1e3), 1),
                        "ms": {n: round(v, 4) for n, v in kern.items()},
-                       "frac": {n: r["frac"] for n, r in roofs.items()},
-                       "step_roofline_frac": round(step_roof / (1e3 * ms), 4),
+                       "_work": work, "_kern": kern, "_ms": ms,
                        "device_status": dpb.workspace_status(ws)})
         del x, gy, idx, val, xn, y, gx, gv, rk, ws, plan
         torch.cuda.empty_cache()
+    clk = clocks.stop()
+    for pt in points:
+        work, kern, ms = pt.pop("_work"), pt.pop("_kern"), pt.pop("_ms")
+        roofs = {n: roofline_for(n, work[n], kern[n] / 1e3, peaks, src, clocks=clk) for n in kern}
+        pt["frac"] = {n: r["frac"] for n, r in roofs.items()}
+        pt["step_roofline_frac"] = round(sum(r["t_roofline_us"] for r in roofs.values()) / (1e3 * ms), 4)
     line = {"metric": "DPB sweep at d=768, T=32768: tokens/s (encode+decode+bwd) and roofline fraction per point",
             "unit": "tokens/s", "n_gpus": world, "steps": steps, "warmup": 2, "higher_is_better": True,
             "scaling": "weak", "dtype": "bf16", "data": "synthetic (x, grad_y ~ N(0, 1), bf16)",
             "config": {"workload": "sweep", "T_per_gpu": 32768, "d": 768, "levels": 5, "children": 16,
                        "r_kept": "decode keeps r (fp32) for the backward"},
-            "points": points}
+            "clocks": clk, "points": points}
     if rank == 0:
         print(json.dumps(line), flush=True)
     return 0
@@ -884,13 +1004,19 @@ def run_transformer(args, world, rank, local):
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=None,
+                    help="timed steps (default: 1500 for the wide workload, about 2 s; 200 for the "
+                         "per-level layouts; 20 for the sweep and the transformer step)")
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--ref-tokens", type=int, default=2048)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-parity", action="store_true", help="skip the oracle check of sampled rows")
+    ap.add_argument("--clock-seconds", type=float, default=2.0,
+                    help="a shorter timed region is followed by the same step up to this many seconds, "
+                         "so that the clock sampler sees the kernels run")
     ap.add_argument("--e2e-streams", type=int, default=4, help="streams of the host-buffer run")
     ap.add_argument("--no-keep-r", action="store_true", help="backward rebuilds r instead of reading the decode's")
     ap.add_argument("--coset", choices=["wht", "contraction"],
@@ -903,6 +1029,8 @@ def main(argv=None):
     ap.add_argument("--workload", default=WORKLOAD, choices=[WORKLOAD, "paper3l", "paper2l", "gpt2small", "sweep"],
                     help="wide (the headline, global selection) or one of the paper's per-level layouts")
     args = ap.parse_args(argv)
+    if args.steps is None:
+        args.steps = {WORKLOAD: 1500, "paper3l": 200, "paper2l": 200}.get(args.workload, 20)
     world, rank, local = dist_env()
     if args.warmup < 3 and args.impl == "ours":
         print("note: at least 3 warm-up steps are used", file=sys.stderr)

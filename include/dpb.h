@@ -299,8 +299,12 @@ dpb_status dpb_workspace_status(const void *workspace, int clear, int32_t *statu
  * library routine.
  *   status_out  device int32 (nullable): receives the DPB_DEV_* bits of this
  *               call (the scratch word is cleared at the start of each call)
- * Plans whose scratch need (dpb_workspace_size) exceeds 4096 bytes are
- * rejected with DPB_ERR_UNSUPPORTED. The first call on a device looks up the
+ * The status word is all the scratch this call needs, for every plan and
+ * every T, so no plan is rejected for its size: the packed (mu, 1/sigma)
+ * table copy that dpb_encode keeps in a workspace of dpb_workspace_size
+ * bytes is not made here, and a standardised call reads mu and sigma from
+ * the two caller tables instead (same results, one more load per candidate,
+ * so slower with tables). The first call on a device looks up the
  * array's device address (cudaGetSymbolAddress); make that first call before
  * any stream capture. Every call on a device shares the one array, so calls
  * whose kernels overlap on the GPU (different streams, or several host

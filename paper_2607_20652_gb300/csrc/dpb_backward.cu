@@ -475,9 +475,7 @@ __global__ void __launch_bounds__(kBwdWarps * 32, 3) backward_lut_kernel(Backwar
 }
 
 int grid_for(const dpb_plan *p, int64_t T, int warps) {
-    int sms = 0;
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, p->device);
-    return (int)std::min<int64_t>((T + warps - 1) / warps, (int64_t)sms * 16);
+    return (int)std::min<int64_t>((T + warps - 1) / warps, (int64_t)std::max(p->sms, 1) * 16);
 }
 
 template <typename Tio, int NKC, bool VEC>
@@ -486,8 +484,7 @@ cudaError_t run_backward_lut(const dpb_plan *p, const BackwardArgs &a, int64_t T
     const size_t smem = 256 /* alignment */ +
                         sizeof(uint32_t) * ((size_t)bwd_block_words(p->cfg.d, NKC) +
                                             (size_t)warps * bwd_warp_words(p->cfg.d, p->code_len));
-    const cudaError_t e = cudaFuncSetAttribute(backward_lut_kernel<Tio, NKC, VEC>,
-                                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    const cudaError_t e = allow_smem((const void *)backward_lut_kernel<Tio, NKC, VEC>, smem);
     if (e != cudaSuccess) return e;
     backward_lut_kernel<Tio, NKC, VEC><<<grid_for(p, T, warps), warps * 32, smem, stream>>>(a, p->t);
     return cudaGetLastError();
@@ -534,12 +531,12 @@ cudaError_t launch_backward(const dpb_plan *p, const void *x, const int32_t *idx
     const size_t smem = sizeof(uint32_t) * ((size_t)c.d + (size_t)warps * 4 * c.d);
     const int grid = grid_for(p, T, warps);
     if (c.dtype == DPB_BF16) {
-        cudaFuncSetAttribute(backward_warp_kernel<__nv_bfloat16>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        const cudaError_t e = allow_smem((const void *)backward_warp_kernel<__nv_bfloat16>, smem);
+        if (e != cudaSuccess) return e;
         backward_warp_kernel<__nv_bfloat16><<<grid, warps * 32, smem, stream>>>(a);
     } else {
-        cudaFuncSetAttribute(backward_warp_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)smem);
+        const cudaError_t e = allow_smem((const void *)backward_warp_kernel<float>, smem);
+        if (e != cudaSuccess) return e;
         backward_warp_kernel<float><<<grid, warps * 32, smem, stream>>>(a);
     }
     return cudaGetLastError();

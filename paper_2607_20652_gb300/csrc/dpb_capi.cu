@@ -3,13 +3,31 @@
 // stream. No allocation happens in encode/decode/backward.
 #include <cstdint>
 #include <cstring>
+#include <map>
+#include <mutex>
 #include <new>
+#include <utility>
 
 #include "dpb_internal.h"
 
 namespace dpb {
 const char *last_error_message();
+
+cudaError_t allow_smem(const void *func, size_t bytes) {
+    static std::mutex mu;
+    static std::map<std::pair<const void *, int>, size_t> granted;  // (kernel, device) -> bytes set
+    if (bytes <= 48 * 1024) return cudaSuccess;                      // within the default limit
+    int dev = -1;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    std::lock_guard<std::mutex> lock(mu);
+    size_t &have = granted[{func, dev}];
+    if (have >= bytes) return cudaSuccess;
+    e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    if (e == cudaSuccess) have = bytes;
+    return e;
 }
+}  // namespace dpb
 
 namespace {
 
@@ -89,9 +107,10 @@ dpb_status dpb_plan_create(const dpb_config *cfg, const uint32_t *generators, dp
         *out = p;
         return DPB_OK;
     }
-    if (cudaGetDevice(&p->device) != cudaSuccess) {
+    if (cudaGetDevice(&p->device) != cudaSuccess ||
+        cudaDeviceGetAttribute(&p->sms, cudaDevAttrMultiProcessorCount, p->device) != cudaSuccess) {
         delete p;
-        return dpb::fail(DPB_ERR_CUDA, "cudaGetDevice failed");
+        return dpb::fail(DPB_ERR_CUDA, "cudaGetDevice or its multiprocessor count failed");
     }
     const size_t mb = sizeof(uint32_t) * p->M.size(), gb = sizeof(uint32_t) * p->G.size();
     struct Up {

@@ -129,9 +129,7 @@ __global__ void __launch_bounds__(256) decode_lut_kernel(DecodeArgs a, int t) {
 }
 
 int grid_for(const dpb_plan *p, int64_t T, int warps) {
-    int sms = 0;
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, p->device);
-    return (int)std::min<int64_t>((T + warps - 1) / warps, (int64_t)sms * 16);
+    return (int)std::min<int64_t>((T + warps - 1) / warps, (int64_t)std::max(p->sms, 1) * 16);
 }
 
 }  // namespace
@@ -143,8 +141,7 @@ cudaError_t run_decode_lut(const dpb_plan *p, const DecodeArgs &a, int64_t T, cu
     const int warps = 8;
     const size_t smem = 128 /* alignment */ +
                         sizeof(uint32_t) * ((size_t)pad32(p->cfg.d) + (size_t)warps * decode_warp_words(p->cfg.d, p->code_len));
-    const cudaError_t e = cudaFuncSetAttribute(decode_lut_kernel<Tio, NKC, VEC>,
-                                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    const cudaError_t e = allow_smem((const void *)decode_lut_kernel<Tio, NKC, VEC>, smem);
     if (e != cudaSuccess) return e;
     decode_lut_kernel<Tio, NKC, VEC><<<grid_for(p, T, warps), warps * 32, smem, stream>>>(a, p->t);
     return cudaGetLastError();
@@ -182,12 +179,12 @@ cudaError_t launch_decode(const dpb_plan *p, const int32_t *idx, const float *va
     const size_t smem = sizeof(uint32_t) * ((size_t)c.d + (size_t)warps * 2 * c.d);
     const int grid = grid_for(p, T, warps);
     if (c.dtype == DPB_BF16) {
-        cudaFuncSetAttribute(decode_warp_kernel<__nv_bfloat16>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        const cudaError_t e = allow_smem((const void *)decode_warp_kernel<__nv_bfloat16>, smem);
+        if (e != cudaSuccess) return e;
         decode_warp_kernel<__nv_bfloat16><<<grid, warps * 32, smem, stream>>>(a);
     } else {
-        cudaFuncSetAttribute(decode_warp_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)smem);
+        const cudaError_t e = allow_smem((const void *)decode_warp_kernel<float>, smem);
+        if (e != cudaSuccess) return e;
         decode_warp_kernel<float><<<grid, warps * 32, smem, stream>>>(a);
     }
     return cudaGetLastError();

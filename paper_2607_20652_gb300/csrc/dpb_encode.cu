@@ -224,9 +224,7 @@ cudaError_t launch_encode(const dpb_plan *p, const void *x, int64_t T, const flo
     const float2 *tab = nullptr;
     if (mu && tab_scratch) {
         const int64_t m = (int64_t)p->m_mask + 1;
-        int sms = 0;
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, p->device);
-        const int64_t want = (m + 255) / 256, cap = (int64_t)sms * 8;
+        const int64_t want = (m + 255) / 256, cap = (int64_t)std::max(p->sms, 1) * 8;
         pack_tables_kernel<<<(unsigned)(want < cap ? want : cap), 256, 0, stream>>>(mu, sigma, tab_scratch, m);
         const cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
@@ -262,17 +260,15 @@ cudaError_t launch_encode(const dpb_plan *p, const void *x, int64_t T, const flo
     int warps = 4;
     while (warps > 1 && head + warps * per_warp > 200 * 1024) --warps;
     const size_t smem = head + warps * per_warp;
-    int sms = 0;
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, p->device);
     const int64_t want = (T + warps - 1) / warps;
-    const int grid = (int)std::min<int64_t>(want, (int64_t)sms * 16);
+    const int grid = (int)std::min<int64_t>(want, (int64_t)std::max(p->sms, 1) * 16);
     if (c.dtype == DPB_BF16) {
-        cudaFuncSetAttribute(encode_warp_kernel<__nv_bfloat16>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        const cudaError_t e = allow_smem((const void *)encode_warp_kernel<__nv_bfloat16>, smem);
+        if (e != cudaSuccess) return e;
         encode_warp_kernel<__nv_bfloat16><<<grid, warps * 32, smem, stream>>>(a);
     } else {
-        cudaFuncSetAttribute(encode_warp_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)smem);
+        const cudaError_t e = allow_smem((const void *)encode_warp_kernel<float>, smem);
+        if (e != cudaSuccess) return e;
         encode_warp_kernel<float><<<grid, warps * 32, smem, stream>>>(a);
     }
     return cudaGetLastError();

@@ -965,14 +965,10 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
 template <int NKC, int KPL, bool COSET, bool WIDE = false>
 cudaError_t launch_kpl(const dpb_plan *p, const Args &a, int warps, cudaStream_t stream) {
     const size_t smem = encode_mma_smem(p, warps);
-    const cudaError_t e =
-        cudaFuncSetAttribute(encode_kernel<NKC, KPL, COSET, WIDE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)smem);
+    const cudaError_t e = allow_smem((const void *)encode_kernel<NKC, KPL, COSET, WIDE>, smem);
     if (e != cudaSuccess) return e;
-    int sms = 0;
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, p->device);
     const int64_t pairs = WIDE ? a.T : (a.T + 1) / 2;
-    const int grid = (int)std::min<int64_t>((pairs + warps - 1) / warps, (int64_t)std::max(sms, 1));
+    const int grid = (int)std::min<int64_t>((pairs + warps - 1) / warps, (int64_t)std::max(p->sms, 1));
     encode_kernel<NKC, KPL, COSET, WIDE><<<grid, warps * 32, smem, stream>>>(a);
     return cudaGetLastError();
 }

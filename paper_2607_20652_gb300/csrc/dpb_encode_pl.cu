@@ -772,12 +772,10 @@ cudaError_t launch_encode_pl(const dpb_plan *p, const void *x, int64_t T, const 
     a.inv_sqrt_d = p->inv_sqrt_d;
     a.nbs = pl_stages(c, a.kvh, a.dmax);
     const size_t smem = encode_pl_smem(p);
-    const cudaError_t e = cudaFuncSetAttribute(encode_pl_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    const cudaError_t e = allow_smem((const void *)encode_pl_kernel, smem);
     if (e != cudaSuccess) return e;
-    int sms = 0;
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, p->device);
     const int64_t groups = (T + kTokens - 1) / kTokens;
-    const int grid = (int)std::min<int64_t>(groups, (int64_t)std::max(sms, 1));
+    const int grid = (int)std::min<int64_t>(groups, (int64_t)std::max(p->sms, 1));
     encode_pl_kernel<<<grid, kTokens * 32, smem, stream>>>(a);
     return cudaGetLastError();
 }

@@ -12,6 +12,7 @@
 struct dpb_plan {
     dpb_config cfg;             // resolved: every derived field filled in
     int device = 0;             // device current at creation; tables live there
+    int sms = 0;                // its multiprocessor count (0 for a host-only plan)
     int t = 0;                  // field GF(2^t)
     uint32_t poly = 0;          // p(z), bit t set
     int code_len = 0;           // k (global) or sum of k_per_level
@@ -88,6 +89,12 @@ cudaError_t launch_encode_pl(const dpb_plan *p, const void *x, int64_t T, const 
 int encode_mma_warps(const dpb_plan *p);
 size_t encode_mma_smem(const dpb_plan *p, int warps);
 constexpr size_t kMaxSmemPerBlock = 227 * 1024;
+
+// Lets kernel `func` use `bytes` of dynamic shared memory on the current
+// device. The attribute is set the first time a kernel needs more than its
+// default (and again only when a later launch needs more), so repeated
+// launches make no driver call; returns the error of a failed set.
+cudaError_t allow_smem(const void *func, size_t bytes);
 
 // Records a message for dpb_last_error() and returns `s`.
 dpb_status fail(dpb_status s, const char *fmt, ...);

@@ -10,9 +10,15 @@
 // device status word) lives here in a file-scope device array instead.
 //
 // The array is a fixed kNoAllocScratchBytes per device; every GPU that loads
-// the library holds it until the process exits. Host code cannot use the
-// array's name as a device address, so the address is looked up once per
-// device with cudaGetSymbolAddress and cached.
+// the library holds it until the process exits. What the encoder needs of it
+// is the status word alone (kStatusBytes), whatever the plan and T: the
+// optional packed (mu, 1/sigma) copy of the standardisation tables, which
+// dpb_encode keeps in a large enough workspace, is left out here, so a
+// standardised call reads mu and sigma from the caller's two tables (the same
+// arithmetic, one more load per candidate). No plan or batch size can need
+// more than the array holds; a static_assert ties the two sizes together.
+// Host code cannot use the array's name as a device address, so the address
+// is looked up once per device with cudaGetSymbolAddress and cached.
 #include <cstdint>
 #include <mutex>
 
@@ -22,6 +28,8 @@ namespace {
 
 constexpr size_t kNoAllocScratchBytes = 4096;
 constexpr int kMaxDevices = 64;
+static_assert(dpb::kStatusBytes <= kNoAllocScratchBytes,
+              "the built-in scratch must hold the device status word");
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
@@ -70,13 +78,9 @@ extern "C" dpb_status dpb_encode_noalloc(const dpb_plan *plan, const void *x, in
         return dpb::fail(DPB_ERR_INVALID_ARG, "idx, val, xnorm, mu and sigma must be 4-byte aligned");
     if ((mu == nullptr) != (sigma == nullptr))
         return dpb::fail(DPB_ERR_INVALID_ARG, "mu and sigma must both be given or both be NULL");
-    // the built-in scratch holds the status word; the optional packed tables
-    // of a workspace are left out (the encoder then reads mu and sigma apart)
-    const size_t need = dpb::kStatusBytes;
-    if (need > kNoAllocScratchBytes)
-        return dpb::fail(DPB_ERR_UNSUPPORTED,
-                         "this plan needs %zu bytes of scratch for T=%lld; the built-in scratch holds %zu",
-                         need, (long long)T, kNoAllocScratchBytes);
+    // the built-in scratch holds the status word only (see the static_assert);
+    // the optional packed tables of a workspace are left out, and the encoder
+    // then reads mu and sigma apart
     if (plan->device < 0) return dpb::fail(DPB_ERR_CUDA, "plan was created without a CUDA device");
     int dev = -1;
     if (cudaGetDevice(&dev) != cudaSuccess) return dpb::fail(DPB_ERR_CUDA, "cudaGetDevice failed");

@@ -377,8 +377,7 @@ __global__ void stats_update_kernel(double *acc, int64_t m, double alpha, float 
 
 template <typename Tio, int NKC>
 cudaError_t run_search(const StatsArgs &a, int32_t n_sample, size_t smem, cudaStream_t stream) {
-    const cudaError_t e =
-        cudaFuncSetAttribute(stats_search_kernel<Tio, NKC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    const cudaError_t e = allow_smem((const void *)stats_search_kernel<Tio, NKC>, smem);
     if (e != cudaSuccess) return e;
     stats_search_kernel<Tio, NKC><<<n_sample, kSearchThreads, smem, stream>>>(a);
     return cudaGetLastError();

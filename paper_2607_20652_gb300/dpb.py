@@ -226,7 +226,10 @@ class Plan:
         cache = self.__dict__.setdefault("_ws_cache", {})
         ws = cache.get(key)
         if ws is None or ws.numel() < self.workspace_size(T):
-            ws = cache[key] = self.workspace(T, dev)
+            # allocated and zeroed on the stream the calls use, so the first
+            # kernel cannot start before the fill ends
+            with torch.cuda.stream(s):
+                ws = cache[key] = self.workspace(T, dev)
         return ws
 
     def status(self, device=None, stream=None, clear: bool = True) -> int:

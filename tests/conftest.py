@@ -1,4 +1,5 @@
-"""Shared pytest set-up: the ``gpu`` marker and repo-root import path."""
+"""Shared pytest set-up: the ``gpu`` marker, the repo-root import path and
+the parity report printed at the end of the session."""
 import os
 import sys
 
@@ -9,3 +10,15 @@ if ROOT not in sys.path:
 
 def pytest_configure(config):
     config.addinivalue_line("markers", "gpu: needs a CUDA GPU (sm_103a) and the built library")
+
+
+def pytest_terminal_summary(terminalreporter, exitstatus, config):
+    """Near-tie counts and worst element-wise errors of every GPU-oracle
+    comparison (relative to max(|ref_i|, row rms); val relative to |x|)."""
+    from tests import parity
+    lines = parity.summary_lines()
+    if not lines:
+        return
+    terminalreporter.write_sep("=", "parity report: near-ties (counted, exempt) and worst errors")
+    for line in lines:
+        terminalreporter.write_line(line)

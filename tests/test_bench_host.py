@@ -55,18 +55,26 @@ def test_roofline_arithmetic():
     assert work["encode"]["bytes"] == 65536 * 2052
     assert work["encode"]["tensor_flops"] == 65536 * 4 * 2 * 8 * 16 * 768
     assert work["backward"]["bytes"] == 65536 * 5376
-    assert work["encode"]["int_ops"] == 65536 * 4 * 8 * 768
+    # 24,576 sign applications per token; a LOP3 flips a packed bf16 pair
+    assert work["encode"]["int_ops"] == 65536 * 4 * 8 * 768 / 2
+    assert bench.algorithmic_work(cfg, 1, 0.0, 4)["encode"]["int_ops"] == 4 * 8 * 768  # fp32: one each
     assert work["decode"]["fp_ops"] == 65536 * (40 * 768 + 3 * 768)
     peaks = {"hbm_gbs": 6781.4, "bf16_tflops_sustained": 1714.8, "sm_max_mhz": 2070.0}
-    # encode: 24,576 sign applications per token at 152 x 64 logic ops per clock
-    # bind before its 786,432 tensor flops at 1714.8 TFLOP/s
+    # encode: 12,288 LOP3 per token at 152 x 64 logic ops per clock (40 us at
+    # T = 65536) bind before its 786,432 tensor flops at 1714.8 TFLOP/s (30 us)
     r = bench.roofline_for("encode", work["encode"], 200e-6, peaks, "measured")
     assert r["bound"] == "alu" and r["pipe"] == "integer logic" and abs(r["peak"] - 152 * 64 * 2070e6 / 1e12) < 1e-3
     assert abs(r["frac"] - work["encode"]["int_ops"] / 200e-6 / (152 * 64 * 2070e6)) < 1e-3
-    assert abs(r["t_roofline_us"] - 1e6 * work["encode"]["int_ops"] / (152 * 64 * 2070e6)) < 0.01
+    assert abs(r["t_roofline_us"] - 40.0) < 0.1
+    assert "maximum SM clock" in r["peak_source"]
+    # with clock samples the ALU peak follows the median clock: a kernel run at
+    # 1035 MHz is held to half the issue rate
+    half = bench.roofline_for("encode", work["encode"], 200e-6, peaks, "measured", clocks={"sm_mhz": 1035.0})
+    assert abs(half["peak"] - r["peak"] / 2) < 1e-3 and abs(half["frac"] - 2 * r["frac"]) < 1e-3
+    assert "1035 MHz" in half["peak_source"]
     r = bench.roofline_for("decode", work["decode"], 100e-6, peaks, "measured")
     assert r["bound"] == "alu" and r["pipe"] == "fp32" and abs(r["peak"] - 152 * 128 * 2070e6 / 1e12) < 1e-3
-    # a pure-HBM call picks the copy bandwidth
-    r = bench.roofline_for("copy", {"bytes": 6781.4e9 * 1e-3}, 2e-3, peaks, "measured")
+    # a pure-HBM call picks the copy bandwidth, whatever the clock
+    r = bench.roofline_for("copy", {"bytes": 6781.4e9 * 1e-3}, 2e-3, peaks, "measured", clocks={"sm_mhz": 900.0})
     assert r["bound"] == "hbm" and abs(r["frac"] - 0.5) < 1e-6 and r["unit"] == "GB/s"
     assert abs(r["frac_nominal"] - 6781.4 / 2 / 7900.0) < 1e-4  # and the nominal 7.9 TB/s beside it

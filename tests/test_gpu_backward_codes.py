@@ -7,8 +7,8 @@ multiple of 32 hashed entries and four lanes each to the rest. These codes
 cover every such split (0, 1, 31, 32, 33, 63, 64, 65, 100 and all hashed
 entries, of 128, or of 96 where d < 128), rows whose width leaves a partial 32-coordinate block and a
 partial chunk of blocks (d = 100, 102, 200; 102 also takes the scalar row path), with and without the decode's r and
-with and without standardisation tables. fp32 rows: within 1e-5 relative per
-row, as for every fp32 gradient.
+with and without standardisation tables. fp32 rows, element by element:
+within 1e-5 of max(|ref_i|, row rms), as for every fp32 output.
 """
 import numpy as np
 import pytest
@@ -71,6 +71,9 @@ def test_backward_on_crafted_codes(d, kept_r, tables):
                                  sigma=None if sigma is None else sigma.astype(np.float64))
     assert parity.rel_rows(gx.cpu().numpy(), gx_o).max() <= 1e-5
     assert parity.rel_rows(gv.cpu().numpy(), gv_o).max() <= 1e-5
+    parity.record(tokens=T, near_ties=0,
+                  gx=parity.check_elementwise(gx.cpu().numpy(), gx_o, 1e-5, False, "grad_x"),
+                  gv=parity.check_elementwise(gv.cpu().numpy(), gv_o, 1e-5, False, "grad_val"))
 
 
 @pytest.mark.parametrize("d", [100, 102, 200, 768])
@@ -93,3 +96,6 @@ def test_decode_on_crafted_codes(d):
     r_o = oracle.decode(ref, idx, val.astype(np.float64), norm_match=0)
     assert parity.rel_rows(y.cpu().numpy(), y_o).max() <= 1e-5
     assert parity.rel_rows(r.cpu().numpy(), r_o).max() <= 1e-5
+    parity.record(tokens=T, near_ties=0,
+                  y=parity.check_elementwise(y.cpu().numpy(), y_o, 1e-5, False, "decode y"),
+                  r=parity.check_elementwise(r.cpu().numpy(), r_o, 1e-5, False, "kept r"))

@@ -89,9 +89,12 @@ def _gpu(plan, x_np, mu=None, sigma=None, gy_np=None):
 
 
 def _check_all(plan, ref, x, g, gy=None, mu=None, sigma=None, rows=None):
-    """Compare the GPU outputs g (for rows `rows` of the batch) with the oracle."""
+    """Compare the GPU outputs g (for rows `rows` of the batch) with the oracle:
+    codes as sets (near-ties counted), then decode and backward element by
+    element on the GPU's own code."""
     rows = np.arange(len(x)) if rows is None else rows
-    tol = parity.TOL[plan.config["dtype"] == dpb.BF16 and "bf16" or "f32"]
+    bf16 = plan.config["dtype"] == dpb.BF16
+    tol = parity.TOL["bf16" if bf16 else "f32"]
     xr = x.astype(np.float64)
     idx_o, val_o, xn_o, gap = oracle.encode(ref, xr, mu=mu, sigma=sigma)
     gi, gvl, gxn = g["idx"][rows], g["val"][rows], g["xnorm"][rows]
@@ -102,7 +105,8 @@ def _check_all(plan, ref, x, g, gy=None, mu=None, sigma=None, rows=None):
     y_o = oracle.decode(ref, gi, gvl.astype(np.float64), gxn.astype(np.float64))
     e = parity.rel_rows(g["y"][rows], y_o)
     assert e.max() <= tol, f"decode error {e.max():.3e} > {tol}"
-    report = dict(near_ties=near, tokens=len(rows), val_err=worst_val, dec_err=float(e.max()))
+    ey = parity.check_elementwise(g["y"][rows], y_o, tol, bf16, "decode y")
+    report = dict(near_ties=near, tokens=len(rows), val=worst_val, y=ey)
     if gy is not None:
         gx_o, gv_o = oracle.backward(ref, xr, gi, gvl.astype(np.float64), gy.astype(np.float64),
                                      sigma=sigma)
@@ -110,8 +114,10 @@ def _check_all(plan, ref, x, g, gy=None, mu=None, sigma=None, rows=None):
         ev = parity.rel_rows(g["gv"][rows], gv_o)
         assert ex.max() <= tol, f"grad_x error {ex.max():.3e} > {tol}"
         assert ev.max() <= 1e-5, f"grad_val error {ev.max():.3e} > 1e-5"
-        report.update(gx_err=float(ex.max()), gv_err=float(ev.max()))
+        report.update(gx=parity.check_elementwise(g["gx"][rows], gx_o, tol, bf16, "grad_x"),
+                      gv=parity.check_elementwise(g["gv"][rows], gv_o, 1e-5, False, "grad_val"))
     assert g["status"] == 0, f"device status 0x{g['status']:x}"
+    parity.record(**report)
     print(report)
     return report
 
@@ -183,7 +189,7 @@ def test_wide_planted_parity():
     # (cross-talk of 56 hashed features lifts many basis coordinates to |x| ~ 1,
     # and they take code slots); parity with the oracle is what is asserted.
     assert recovered > 0.4
-    assert rep["near_ties"] <= T // 20
+    assert rep["near_ties"] <= T // 20, rep
 
 
 def test_wide_full_size_sampled():
@@ -336,13 +342,18 @@ def test_kept_r_matches_the_oracle_and_the_rebuilt_backward(d, dtype):
     assert torch.equal(y, y_kept)
     r_o = oracle.decode(ref, idx.cpu().numpy(), val.cpu().numpy().astype(np.float64), norm_match=0)
     assert parity.rel_rows(r.cpu().numpy(), r_o).max() <= 1e-5
+    er = parity.check_elementwise(r.cpu().numpy(), r_o, 1e-5, False, "kept r")
     tol = parity.TOL[dtype]
+    bf16 = dtype == "bf16"
     assert parity.rel_rows(gx1.float().cpu().numpy(), gx0.float().cpu().numpy()).max() <= max(tol, 1e-5)
     assert parity.rel_rows(gv1.cpu().numpy(), gv0.cpu().numpy()).max() <= 1e-5
     gx_o, gv_o = oracle.backward(ref, x_np.astype(np.float64), idx.cpu().numpy(),
                                  val.cpu().numpy().astype(np.float64), gy_np.astype(np.float64))
     assert parity.rel_rows(gx1.float().cpu().numpy(), gx_o).max() <= tol
     assert parity.rel_rows(gv1.cpu().numpy(), gv_o).max() <= 1e-5
+    parity.record(tokens=300, near_ties=0, r=er,
+                  gx=parity.check_elementwise(gx1.float().cpu().numpy(), gx_o, tol, bf16, "grad_x (kept r)"),
+                  gv=parity.check_elementwise(gv1.cpu().numpy(), gv_o, 1e-5, False, "grad_val (kept r)"))
 
 
 @pytest.mark.parametrize("T", [300, 4099])
@@ -367,7 +378,8 @@ def test_coset_scoring_matches_the_oracle(T):
         assert g["status"] == 0
         parity.check_code_order(g["idx"][rows], g["val"][rows])
         near, worst = parity.compare_codes(g["idx"][rows], g["val"][rows], idx_o, val_o, gap, xn_o)
-        assert near <= max(2, len(rows) // 10)
+        assert near <= max(2, len(rows) // 10), f"{near} near-ties of {len(rows)} tokens"
+        parity.record(tokens=len(rows), near_ties=near, val=worst)
         reports.append((near, worst))
     print(reports)
 

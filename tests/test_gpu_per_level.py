@@ -66,17 +66,21 @@ def _check(plan, ref, kls, x, g, mu=None, sigma=None, gy=None):
         near, worst, off = max(near, n), max(worst, w), off + K
     y_o = oracle.decode(ref, g["idx"], g["val"].astype(np.float64), g["xnorm"].astype(np.float64))
     e = parity.rel_rows(g["y"], y_o)
-    assert e.max() <= parity.TOL["bf16"], f"decode error {e.max():.3e}"
-    report = dict(tokens=len(x), near_ties=near, val_err=worst, dec_err=float(e.max()))
+    tol = parity.TOL["bf16"]
+    assert e.max() <= tol, f"decode error {e.max():.3e}"
+    report = dict(tokens=len(x), near_ties=near, val=worst,
+                  y=parity.check_elementwise(g["y"], y_o, tol, True, "decode y"))
     if gy is not None:
         gx_o, gv_o = oracle.backward(ref, xr, g["idx"], g["val"].astype(np.float64), gy.astype(np.float64),
                                      sigma=sigma)
         ex, ev = parity.rel_rows(g["gx"], gx_o), parity.rel_rows(g["gv"], gv_o)
-        assert ex.max() <= parity.TOL["bf16"], f"grad_x error {ex.max():.3e}"
+        assert ex.max() <= tol, f"grad_x error {ex.max():.3e}"
         assert ev.max() <= 1e-5, f"grad_val error {ev.max():.3e}"
-        report.update(gx_err=float(ex.max()), gv_err=float(ev.max()))
+        report.update(gx=parity.check_elementwise(g["gx"], gx_o, tol, True, "grad_x"),
+                      gv=parity.check_elementwise(g["gv"], gv_o, 1e-5, False, "grad_val"))
     assert g["status"] == 0, f"device status 0x{g['status']:x}"
     assert near <= max(2, len(x) // 10), report
+    parity.record(**report)
     print(report)
     return report
 

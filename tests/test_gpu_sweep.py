@@ -62,7 +62,7 @@ def test_sweep_point_full_size_sampled(w):
     idx_o, val_o, xn_o, gap = oracle.encode(ref, xr)
     parity.check_code_order(gi, gvl)
     near, worst = parity.compare_codes(gi, gvl, idx_o, val_o, gap, xn_o)
-    assert near <= max(2, len(rows) // 10)
+    assert near <= max(2, len(rows) // 10), f"{near} near-ties of {len(rows)} tokens"
     assert np.all(np.abs(gxn - xn_o) <= 1e-5 * xn_o)
     tol = parity.TOL["bf16"]
     y_o = oracle.decode(ref, gi, gvl.astype(np.float64), gxn.astype(np.float64))
@@ -70,3 +70,10 @@ def test_sweep_point_full_size_sampled(w):
     gx_o, gv_o = oracle.backward(ref, xr, gi, gvl.astype(np.float64), gy[rows].astype(np.float64))
     assert parity.rel_rows(gx.float().cpu().numpy()[rows], gx_o).max() <= tol
     assert parity.rel_rows(gv.cpu().numpy()[rows], gv_o).max() <= 1e-5
+    parity.record(tokens=len(rows), near_ties=near, val=worst,
+                  y=parity.check_elementwise(y.float().cpu().numpy()[rows], y_o, tol, True, "decode y"),
+                  r=parity.check_elementwise(r.cpu().numpy()[rows],
+                                             oracle.decode(ref, gi, gvl.astype(np.float64), norm_match=0),
+                                             1e-5, False, "kept r"),
+                  gx=parity.check_elementwise(gx.float().cpu().numpy()[rows], gx_o, tol, True, "grad_x"),
+                  gv=parity.check_elementwise(gv.cpu().numpy()[rows], gv_o, 1e-5, False, "grad_val"))

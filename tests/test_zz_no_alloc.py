@@ -4,8 +4,9 @@ It exists for callers that cannot allocate device memory (plug-ins inside a
 runtime that owns every allocation and hands them only input and output
 buffers). Its scratch lives in a fixed device array inside the library. This
 test calls it through the C ABI twice in a row and checks each call against
-dpb_encode on the same inputs, within the tolerances of the parity tests;
-the second call also shows that the shared scratch starts clean.
+dpb_encode on the same inputs, within the tolerances of the parity tests, for
+the global (mma.sync) and the per-level (tcgen05) encoders; the second call
+also shows that the shared scratch starts clean.
 """
 import ctypes
 
@@ -62,6 +63,21 @@ def test_noalloc_matches_encode_twice(lib, dtype, d, m_bits, levels, beam, k):
         parity.check_code_order(idx, val)
         near, _ = parity.compare_codes(idx, val, ri, rv.astype(np.float64), np.full(T, np.inf), rxn)
         assert near == 0
+        assert np.array_equal(idx, ri) and np.array_equal(val, rv)
+        assert np.allclose(xn, rxn, rtol=1e-6, atol=0)
+
+
+def test_noalloc_per_level_plan_matches_encode_twice(lib):
+    # the paper's per-level selection (tcgen05 scoring): 3L layout of App. G
+    plan = dpb.Plan(d=1024, levels=3, bits=[10, 15, 17], children=[0, 256, 256], dtype="bf16",
+                    select_mode=dpb.SELECT_PER_LEVEL, k_per_level=[16, 32, 64])
+    T = 203                                        # 25 blocks of 8 tokens and a ragged tail
+    x = torch.from_numpy(inputs.to_bf16(inputs.gaussian_rows(T, 1024, 44))).cuda().to(torch.bfloat16)
+    ri, rv, rxn = (t.cpu().numpy() for t in dpb.encode(plan, x, workspace=plan.workspace(T)))
+    torch.cuda.synchronize()
+    for _ in range(2):
+        idx, val, xn, st = _noalloc(lib, plan, x)
+        assert st == 0
         assert np.array_equal(idx, ri) and np.array_equal(val, rv)
         assert np.allclose(xn, rxn, rtol=1e-6, atol=0)
 
