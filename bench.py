@@ -477,7 +477,7 @@ def run_ours(args, world, rank, local):
     seed = shard_seed(w["seed"], rank)
     x, gy, idx_true, host = make_inputs_gpu(w, plan, seed, device)
     # oracle leg: seeded rows of the batch rebuilt by the oracle alone, checked after timing
-    check = rank == 0 and world == 1 and not args.no_parity and not std and not args.coset
+    check = rank == 0 and world == 1 and not args.no_parity and not args.standardise and not args.coset
     if check:
         pref, prows, px = parity_rows(w, host, T, seed)
         x[torch.from_numpy(prows).to(device)] = torch.from_numpy(px).to(device).to(torch.bfloat16)
