@@ -321,16 +321,21 @@ __device__ __forceinline__ void sweep_accumulate(const Sweep &s, float *out, con
 
 // Code shape of a sweep. kSweepWide rounds the runs up to one of five
 // unrolled widths (the extra runs read all-zero tables) and does two blocks
-// per trip: the fewest instructions. kSweepCompact always does all 13 runs,
-// one block per trip: the least code, for kernels whose other phases already
-// fill the instruction caches.
+// per trip: the fewest instructions. kSweepCompact does one block per trip
+// and rounds the runs up to 8, 10 or 13 only: less code, for kernels whose
+// other phases already fill the instruction caches.
 enum SweepShape { kSweepWide, kSweepCompact };
 
 template <int NKC, SweepShape SHAPE>
 __device__ __forceinline__ void sweep_accumulate_runs(const Sweep &s, float *out, const uint32_t *koff,
                                                       int d, float scale) {
     if constexpr (SHAPE == kSweepCompact) {
-        sweep_accumulate<NKC, kMaxRuns, 1>(s, out, koff, d, scale);
+        if (s.runs <= 8)
+            sweep_accumulate<NKC, 8, 1>(s, out, koff, d, scale);
+        else if (s.runs <= 10)
+            sweep_accumulate<NKC, 10, 1>(s, out, koff, d, scale);
+        else
+            sweep_accumulate<NKC, kMaxRuns, 1>(s, out, koff, d, scale);
     } else if (s.runs <= 4) {
         sweep_accumulate<NKC, 4, 2>(s, out, koff, d, scale);
     } else if (s.runs <= 6) {
