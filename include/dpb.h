@@ -314,6 +314,21 @@ dpb_status dpb_encode_noalloc(const dpb_plan *plan, const void *x, int64_t T, co
                               const float *sigma, int32_t *idx, float *val, float *xnorm,
                               int32_t *status_out, void *stream);
 
+/*
+ * dpb_debug_set_wait_limit -- test hook for the bounded waits of the
+ * per-level (tcgen05) encoder; the paper has no counterpart. Every
+ * mbarrier wait of that kernel's main loop (a generator-tile copy landing,
+ * the MMAs of a chunk or level finishing) gives up after `tries` polls for
+ * the launches that follow, from any thread; -1 restores the default
+ * (2^20 polls). A wait that gives up stops the block: the kernel sets
+ * DPB_DEV_TIMEOUT in the workspace status, waits (with the default bound)
+ * for its copies and MMAs still in flight, frees its tensor memory and
+ * returns; that call's codes are incomplete. With tries = 0 every such wait
+ * gives up at once, which lets a test exercise that path without a fault.
+ * Returns DPB_ERR_INVALID_ARG for tries < -1.
+ */
+dpb_status dpb_debug_set_wait_limit(int32_t tries);
+
 /* Static description of a status code. */
 const char *dpb_status_string(dpb_status s);
 

@@ -24,7 +24,8 @@
 //  - one thread issues the 4 MMAs of the chunk and commits them to an
 //    mbarrier that frees the chunk's buffers; scores accumulate in TMEM.
 // Every mbarrier wait is bounded; a wait that gives up sets
-// DPB_DEV_TIMEOUT, and the block drains its MMAs and frees its TMEM.
+// DPB_DEV_TIMEOUT and stops the block, which then waits (again bounded) for
+// its bulk copies and MMAs still in flight and frees its TMEM.
 //
 // Selection of a level (one warp per token, lane = parent slot): each lane
 // keeps the 4 largest of its row's group maxima (the largest key |z| of each
@@ -36,6 +37,7 @@
 // child) are dropped. When K distinct candidates reach tau they are exactly
 // the level's top K.
 #include <algorithm>
+#include <atomic>
 
 #include "dpb_encode_mma.cuh"
 #include "dpb_internal.h"
@@ -51,7 +53,7 @@ constexpr int kATile = 128 * kChunk * 2;  // one M = 128 tile of a chunk
 constexpr int kSelCap = 256;    // gathered candidates per token and level (up to 8 per lane)
 constexpr int kMaxK = 64;       // K_l per level
 constexpr int kMaxStages = 4;   // generator-tile stages in flight
-constexpr uint32_t kSpin = 1u << 20;  // bound of every mbarrier wait
+constexpr uint32_t kSpin = 1u << 20;  // default bound of the main loop's mbarrier waits, and of the drain
 // at least this much shared memory per block, so that one block (holding all
 // 512 TMEM columns) runs per SM
 constexpr int kMinSmem = 120 * 1024;
@@ -69,6 +71,7 @@ struct Args {
     int kl[DPB_MAX_LEVELS], delta[DPB_MAX_LEVELS], off[DPB_MAX_LEVELS];
     int64_t gt_off[DPB_MAX_LEVELS];
     float inv_sqrt_d;
+    uint32_t spin;  // bound (tries) of the main loop's mbarrier waits
 };
 
 // ---- layout --------------------------------------------------------------------
@@ -102,8 +105,8 @@ __host__ __device__ inline Layout layout(int d, int levels, int kvh, int dmax, i
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
 
-__device__ __forceinline__ bool mbar_wait(uint32_t mbar, uint32_t parity) {
-    for (uint32_t i = 0; i < kSpin; ++i) {
+__device__ __forceinline__ bool mbar_wait(uint32_t mbar, uint32_t parity, uint32_t spin) {
+    for (uint32_t i = 0; i < spin; ++i) {
         uint32_t done;
         asm volatile(
             "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
@@ -427,6 +430,14 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
     auto stage_b = [&](uint32_t g) { return sB + (g % (uint32_t)nbs) * a.dmax * 128; };
     uint32_t G = 0;  // chunks whose MMAs were committed
     bool failed = false;
+    // thread 0: generator tiles are copied and consumed in chunk order; the
+    // copies of chunks [consumed, issued) are in flight
+    uint32_t issued = 0, consumed = 0;
+    bool tfail = false;  // thread 0: a wait of its own gave up
+    auto issue_b = [&](uint32_t g, const uint32_t *src, int D) {
+        copy_b(stage_b(g), src, D, full_b(g));
+        issued = g + 1;
+    };
     const uint32_t lo_mask = (1u << a.t) - 1u;
     const int64_t ngroups = (a.T + kTokens - 1) / kTokens;
     uint16_t *xh = reinterpret_cast<uint16_t *>(xw + warp * nblk * 16);
@@ -501,15 +512,14 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
             // one ahead of the first chunk with two
             const int ahead = nbs >= 3 ? nbs : nbs - 1;
             if (tid == 0)
-                for (int c = 0; c < min(ahead, nch); ++c)
-                    copy_b(stage_b(G0 + c), gt + (int64_t)c * D * 32, D, full_b(G0 + c));
+                for (int c = 0; c < min(ahead, nch); ++c) issue_b(G0 + c, gt + (int64_t)c * D * 32, D);
             for (int c = 0; c < nch; ++c) {
                 const uint32_t g = G0 + c;
                 {
                     // A stage g & 1 is free once the MMAs of chunk g - 2 are done
                     bool ok = true;
-                    if (c >= 2) ok = mbar_wait(mma_done(g - 2), phase(g - 2));
-                    if (__syncthreads_or(!ok)) {  // every thread leaves together
+                    if (c >= 2) ok = mbar_wait(mma_done(g - 2), phase(g - 2), a.spin);
+                    if (__syncthreads_or(!ok || tfail)) {  // every thread leaves together
                         failed = true;
                         break;
                     }
@@ -543,9 +553,13 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
                 asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                 __syncthreads();
                 if (tid == 0) {
-                    if (!mbar_wait(full_b(g), phase(g))) {
-                        set_status(a.status, DPB_DEV_TIMEOUT);  // the commit below still arrives
+                    if (!mbar_wait(full_b(g), phase(g), a.spin)) {
+                        // no MMA for this chunk (the commit below still arrives);
+                        // the block stops at its next barrier
+                        set_status(a.status, DPB_DEV_TIMEOUT);
+                        tfail = true;
                     } else {
+                        consumed = g + 1;
                         asm volatile("tcgen05.fence::after_thread_sync;");
                         const uint32_t bb = smem_u32(stage_b(g));
                         for (int tt = 0; tt < ntiles; ++tt) {
@@ -566,17 +580,18 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
                         // the tile nbs - 2 chunks ahead goes to the stage chunk g - 2
                         // read; its MMAs were waited for at the top of this chunk,
                         // so thread 0 goes on to the next chunk without waiting
-                        if (c >= 2 && c + nbs - 2 < nch)
-                            copy_b(stage_b(g + nbs - 2), gt + (int64_t)(c + nbs - 2) * D * 32, D,
-                                   full_b(g + nbs - 2));
+                        if (!tfail && c >= 2 && c + nbs - 2 < nch)
+                            issue_b(g + nbs - 2, gt + (int64_t)(c + nbs - 2) * D * 32, D);
                     } else if (c + 1 < nch) {
                         // two stages: the next tile goes to the stage chunk g - 1
                         // read, once its MMAs are done
-                        const bool ok = c == 0 || mbar_wait(mma_done(g - 1), phase(g - 1));
-                        if (ok)
-                            copy_b(stage_b(g + 1), gt + (int64_t)(c + 1) * D * 32, D, full_b(g + 1));
-                        else
+                        const bool ok = !tfail && (c == 0 || mbar_wait(mma_done(g - 1), phase(g - 1), a.spin));
+                        if (ok) {
+                            issue_b(g + 1, gt + (int64_t)(c + 1) * D * 32, D);
+                        } else {
                             set_status(a.status, DPB_DEV_TIMEOUT);
+                            tfail = true;
+                        }
                     }
                 }
                 G = g + 1;
@@ -584,8 +599,8 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
             if (failed) break;
             {
                 // the last commit covers every MMA of the level
-                const bool ok = mbar_wait(mma_done(G - 1), phase(G - 1));
-                if (__syncthreads_or(!ok)) {
+                const bool ok = mbar_wait(mma_done(G - 1), phase(G - 1), a.spin);
+                if (__syncthreads_or(!ok || tfail)) {
                     failed = true;
                     break;
                 }
@@ -650,8 +665,13 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
         }
     }
     if (failed) set_status(a.status, DPB_DEV_TIMEOUT);
-    // drain: the last commit is waited for (bounded) before TMEM is freed
-    if (failed && G > 0) mbar_wait(mma_done(G - 1), phase(G - 1));
+    // drain (bounded, with the default bound): every generator-tile copy still
+    // in flight lands, and the last commit (which covers every MMA issued)
+    // arrives, before the block frees its TMEM and its shared memory
+    if (failed && tid == 0) {
+        for (uint32_t g = consumed; g < issued; ++g) mbar_wait(full_b(g), phase(g), kSpin);
+        if (G > 0) mbar_wait(mma_done(G - 1), phase(G - 1), kSpin);
+    }
     asm volatile("tcgen05.fence::before_thread_sync;");
     __syncthreads();
     if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" ::"r"(tmem));
@@ -715,6 +735,10 @@ void build_per_level_tables(dpb_plan *p) {
 
 namespace {
 
+// Bound of the main loop's mbarrier waits for the launches that follow (-1:
+// the default kSpin); set by dpb_debug_set_wait_limit.
+std::atomic<int32_t> g_wait_limit{-1};
+
 // Generator-tile stages: as many as fit (at least 2).
 int pl_stages(const dpb_config &c, int kvh, int dmax) {
     for (int nbs = kMaxStages; nbs > 2; --nbs)
@@ -771,6 +795,8 @@ cudaError_t launch_encode_pl(const dpb_plan *p, const void *x, int64_t T, const 
     }
     a.inv_sqrt_d = p->inv_sqrt_d;
     a.nbs = pl_stages(c, a.kvh, a.dmax);
+    const int32_t lim = g_wait_limit.load(std::memory_order_relaxed);
+    a.spin = lim < 0 ? kSpin : (uint32_t)lim;
     const size_t smem = encode_pl_smem(p);
     const cudaError_t e = allow_smem((const void *)encode_pl_kernel, smem);
     if (e != cudaSuccess) return e;
@@ -781,3 +807,9 @@ cudaError_t launch_encode_pl(const dpb_plan *p, const void *x, int64_t T, const 
 }
 
 }  // namespace dpb
+
+extern "C" dpb_status dpb_debug_set_wait_limit(int32_t tries) {
+    if (tries < -1) return dpb::fail(DPB_ERR_INVALID_ARG, "tries must be -1 (default) or >= 0");
+    dpb::g_wait_limit.store(tries, std::memory_order_relaxed);
+    return DPB_OK;
+}

@@ -21,7 +21,7 @@ MAX_CHILDREN = 256
 F32, BF16 = 0, 1
 SELECT_GLOBAL, SELECT_PER_LEVEL = 0, 1
 SCORING_CONTRACTION, SCORING_COSET_WHT = 0, 1
-DEV_BAD_INDEX, DEV_BAD_SIGMA, DEV_SHORT_CODE = 0x1, 0x2, 0x4
+DEV_BAD_INDEX, DEV_BAD_SIGMA, DEV_SHORT_CODE, DEV_TIMEOUT = 0x1, 0x2, 0x4, 0x8
 
 _STATUS = {0: "ok", 1: "invalid argument", 2: "unsupported configuration", 3: "CUDA error",
            4: "device wait timed out", 5: "out of memory", 6: "device-side error flagged"}
@@ -66,7 +66,7 @@ _lib = None
 EXPORTS = ("dpb_plan_create", "dpb_plan_destroy", "dpb_plan_config", "dpb_plan_tables",
            "dpb_code_length", "dpb_workspace_size", "dpb_encode", "dpb_decode", "dpb_backward",
            "dpb_workspace_status", "dpb_status_string", "dpb_last_error", "dpb_encode_noalloc",
-           "dpb_stats_accumulate", "dpb_stats_update", "dpb_forward")
+           "dpb_stats_accumulate", "dpb_stats_update", "dpb_forward", "dpb_debug_set_wait_limit")
 
 
 def library_path() -> str:
@@ -96,6 +96,7 @@ def load(path: Optional[str] = None):
     lib.dpb_backward.argtypes = [vp, vp, vp, vp, i64, vp, vp, vp, vp, vp, vp, sz, vp]
     lib.dpb_workspace_status.argtypes = [vp, ctypes.c_int, ctypes.POINTER(ctypes.c_int32), vp]
     lib.dpb_encode_noalloc.argtypes = [vp, vp, i64, vp, vp, vp, vp, vp, vp, vp]
+    lib.dpb_debug_set_wait_limit.argtypes = [ctypes.c_int32]
     lib.dpb_stats_accumulate.argtypes = [vp, vp, i64, vp, vp, vp, ctypes.c_int32, vp, vp, sz, vp]
     lib.dpb_stats_update.argtypes = [vp, vp, ctypes.c_float, vp, vp, vp]
     lib.dpb_forward.argtypes = [vp, vp, i64, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
@@ -390,6 +391,12 @@ def stats_step(plan: Plan, x: torch.Tensor, mu: torch.Tensor, sigma: torch.Tenso
                                         stream=stream),
              lambda a: stats_update(plan, a, alpha, mu, sigma, stream=stream), acc, group)
     return mu, sigma
+
+
+def set_wait_limit(tries: int = -1):
+    """dpb_debug_set_wait_limit: bound of the per-level encoder's main-loop
+    mbarrier waits for the launches that follow (-1 restores the default)."""
+    _check(load().dpb_debug_set_wait_limit(int(tries)))
 
 
 def workspace_status(workspace: torch.Tensor, clear: bool = False, stream=None) -> int:

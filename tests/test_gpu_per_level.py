@@ -149,3 +149,24 @@ def test_paper_3l_layout_at_scale_sampled():
     rows = np.random.default_rng(5).choice(T, 48, replace=False)
     sub = {k: (v[rows] if isinstance(v, np.ndarray) and v.shape[:1] == (T,) else v) for k, v in g.items()}
     _check(plan, ref, kls, x[rows], sub)
+
+
+def test_wait_that_gives_up_is_flagged_and_leaves_the_context_usable():
+    # With the main loop's mbarrier waits bounded at 0 polls, the first wait of
+    # the tcgen05 encoder gives up at once: the kernel flags DPB_DEV_TIMEOUT,
+    # lets its generator-tile copies and MMAs in flight land, frees its tensor
+    # memory and returns. A normal call right after must run (its tensor-memory
+    # allocation succeeds) and match the oracle.
+    kls = [16, 32, 64]
+    plan, ref = _plan_ref(1024, [10, 15, 17], [0, 256, 256], kls)
+    x = inputs.to_bf16(inputs.gaussian_rows(40, 1024, 12))
+    xt = torch.from_numpy(x).cuda().to(torch.bfloat16)
+    ws = plan.workspace(40)
+    try:
+        dpb.set_wait_limit(0)
+        dpb.encode(plan, xt, workspace=ws)
+        torch.cuda.synchronize()
+    finally:
+        dpb.set_wait_limit(-1)
+    assert dpb.workspace_status(ws) & dpb.DEV_TIMEOUT
+    _check(plan, ref, kls, x, _gpu(plan, x))
