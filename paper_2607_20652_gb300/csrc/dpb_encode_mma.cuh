@@ -386,10 +386,11 @@ __device__ __forceinline__ int merge_entrants(uint64_t *L, int k, uint64_t *E, c
 
 // Fast path (no standardisation, k <= 16 R): see the header comment. `row`
 // is the token's row as 16-byte chunks (8 coordinates each); this lane reads
-// chunks lane + 32 j (again from L1 in the later passes). The union's first k
-// go to the list; coordinates that reach its k-th word without being among
-// their lane's R kept words are merged in afterwards. Returns false, with
-// nothing written, when more of them arrive than the scratch holds.
+// chunks lane + 32 j. The union's first k go to the list; coordinates that
+// reach its k-th word without being among their lane's R kept words (the
+// extras; only lanes whose R kept words all reach it can have them, and the
+// warp rescans just those, from L1) are merged in afterwards. Returns false,
+// with nothing written, when more of them arrive than the scratch holds.
 template <int R, int KPL>
 __device__ __forceinline__ bool level0_union(const uint4 *row, int nch, int k, uint64_t *E, int ecap, uint64_t *L,
                                              uint32_t *beam) {
@@ -418,40 +419,42 @@ __device__ __forceinline__ bool level0_union(const uint4 *row, int nch, int k, u
     for (int r = 0; r < R; ++r)
         if (r == (k - 1) % R) mine = top[r];
     const uint32_t tau = __shfl_sync(kFull, mine, (k - 1) / R);
-    int nx = 0;
+    // Extras are unkept words in [tau, kept_min): only lanes whose R kept
+    // words all reach tau can have them. The warp rescans just those lanes'
+    // coordinates together (a few per lane), gathering the extras into E.
+    const bool flag = kept_min >= tau && kept_min != 0u;
+    const unsigned fm = __ballot_sync(kFull, flag);
+    const int nf = __popc(fm), ne = 8 * ((nch + 31) / 32);  // flagged lanes; coordinate slots per lane
+    const int cap = ecap - 16;                               // E's last 16 entries hold the flagged lanes
+    int total = 0;
+    if (nf) {
+        uint32_t *fl = reinterpret_cast<uint32_t *>(E + cap);
+        if (flag) fl[__popc(fm & lanes_below())] = (uint32_t)lane;
+        __syncwarp();
+        const uint16_t *xs = reinterpret_cast<const uint16_t *>(row);
 #pragma unroll 1
-    for (int ch = lane; ch < nch; ch += 32) {
-        const uint4 v = row[ch];
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-            const uint32_t w = cword0(elem16(v, e), (uint32_t)(8 * ch + e));
-            nx += (w >= tau) & (w < kept_min);
+        for (int q0 = 0; q0 < nf * ne; q0 += 32) {
+            const int q = q0 + lane, f = q / ne, j = q - f * ne;
+            const int owner = q < nf * ne ? (int)fl[f] : 0;
+            const int ch = owner + 32 * (j >> 3), i = 8 * ch + (j & 7);
+            const uint32_t km = __shfl_sync(kFull, kept_min, owner);
+            uint32_t w = 0u;
+            if (q < nf * ne && ch < nch) w = cword0(xs[i], (uint32_t)i);
+            const bool take = w >= tau && w < km && w != 0u;
+            const unsigned mb = __ballot_sync(kFull, take);
+            const int pos = total + __popc(mb & lanes_below());
+            if (take && pos < cap) E[pos] = widen0(w);
+            total += __popc(mb);
         }
+        __syncwarp();
     }
-    const int total = __reduce_add_sync(kFull, nx);
-    if (total > ecap) return false;
+    if (total > cap) return false;
 #pragma unroll
     for (int r = 0; r < R; ++r) {
         const int e = lane * R + r;
         if (e < k) L[e] = widen0(top[r]);
     }
     if (total > 0) {
-        int off = nx;  // exclusive prefix of the extras over the lanes
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int v = __shfl_up_sync(kFull, off, o);
-            if (lane >= o) off += v;
-        }
-        off -= nx;
-#pragma unroll 1
-        for (int ch = lane; ch < nch; ch += 32) {
-            const uint4 v = row[ch];
-#pragma unroll
-            for (int e = 0; e < 8; ++e) {
-                const uint32_t w = cword0(elem16(v, e), (uint32_t)(8 * ch + e));
-                if (w >= tau && w < kept_min) E[off++] = widen0(w);
-            }
-        }
         __syncwarp();
         merge_sorted<KPL>(L, k, E, total, nullptr);
         if (lane < kBeam) beam[lane] = cword_idx(L[lane]);
