@@ -13,7 +13,7 @@ size_t encode_mma_smem(const dpb_plan *p, int warps) {
 }
 
 int encode_mma_warps(const dpb_plan *p) {
-    for (int w : {16, 12, 8, 4})
+    for (int w : {20, 16, 12, 8, 4})
         if (encode_mma_smem(p, w) <= kMaxSmemPerBlock) return w;
     return 0;
 }

@@ -13,7 +13,7 @@
 // a pair sit 16 apart in the parent's sign word over the block, and one shift
 // moves both to the bf16 sign positions 15 and 31. The sign word of parent p
 // over block m is
-//     W5[p & 31] ^ PQ[m][(p_lo >> 5) & 31] ^ XOR_k VH_k[m][chunk_k(p_hi)],
+//     W5[p & 31] ^ (bit m of W5[(p_lo >> 5) & 31] ? ~0 : 0) ^ XOR_k VH_k[m][chunk_k(p_hi)],
 // the Walsh, block-parity and inverse-coordinate parts of parity(M[iota] & p)
 // (App. A.4 Eq. 26). Gamma_l lives in shared memory in B-fragment order.
 //
@@ -43,7 +43,7 @@
 namespace dpb {
 namespace mmaenc {
 
-constexpr int kMaxWarps = 16;
+constexpr int kMaxWarps = 20;
 constexpr int kBeam = 8;
 
 struct Args {
@@ -64,9 +64,8 @@ struct Args {
 // ---- shared-memory layout (32-bit words) ------------------------------------------
 
 __host__ __device__ inline int block_words(int levels, int nblk, int nkc) {
-    // frag [(L-1)][nblk][32][8], W5 [32], PQ [32][32], VH [nkc][32][32],
-    // DD [(L-1)][kDedupSlots][2], G [L][16]
-    return (levels - 1) * nblk * 256 + 32 + 1024 + nkc * 1024 + (levels - 1) * kDedupSlots * 2 + 8 * 16;
+    // frag [(L-1)][nblk][32][8], W5 [32], VH [nkc][32][32], DD [(L-1)][kDedupSlots], G [L][16]
+    return (levels - 1) * nblk * 256 + 32 + nkc * 1024 + (levels - 1) * kDedupSlots + 8 * 16;
 }
 
 // 64-bit entries of the per-warp scratch buffer: the entrants of a merge, the
@@ -115,21 +114,24 @@ __device__ __forceinline__ void mma_bf16(float (&c)[4], uint32_t a0, uint32_t a1
         : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-// Byte offsets of parent p into PQ[m] and VH_k[m], packed four to a word.
+// Parts of parent p's sign words: its Walsh word, the block-parity word
+// (bit m = parity(m AND u), u = bits 5..9 of p_lo: the Walsh word of u) and
+// the byte offsets into VH_k[m], packed to a word.
 struct ParentOff {
     uint32_t w5;  // the Walsh word (the same for every block)
-    uint32_t o;   // PQ, VH_0, VH_1, VH_2 byte offsets
+    uint32_t pq;  // the block-parity word
+    uint32_t o;   // VH_0, VH_1, VH_2 byte offsets (bytes 1..3)
     uint32_t o3;  // VH_3 byte offset
 };
 
 __device__ __forceinline__ ParentOff parent_offsets(uint32_t p, int t, const uint32_t *w5) {
     ParentOff po;
     po.w5 = w5[p & 31u];  // t >= 5: bits 0..4 belong to p_lo
-    const uint32_t b1 = (((p & ((1u << t) - 1u)) >> 5) & 31u) * 4u;
+    po.pq = w5[((p & ((1u << t) - 1u)) >> 5) & 31u];
     const uint32_t h0 = ((p >> t) & 31u) * 4u, h1 = ((p >> (t + 5)) & 31u) * 4u;
     const uint32_t h2 = ((p >> min(t + 10, 31)) & 31u) * 4u;
     const uint32_t h3 = ((p >> min(t + 15, 31)) & 31u) * 4u;
-    po.o = b1 | (h0 << 8) | (h1 << 16) | (h2 << 24);
+    po.o = (h0 << 8) | (h1 << 16) | (h2 << 24);
     po.o3 = h3;
     return po;
 }
@@ -137,10 +139,9 @@ __device__ __forceinline__ ParentOff parent_offsets(uint32_t p, int t, const uin
 // Sign word of a parent over 32-coordinate block m (bit l = 1: coordinate
 // 32 m + l of phi~_p is negative).
 template <int NKC>
-__device__ __forceinline__ uint32_t parent_signs(const ParentOff &po, const uint32_t *pq, const uint32_t *vh, int m) {
-    const char *P = reinterpret_cast<const char *>(pq + m * 32);
+__device__ __forceinline__ uint32_t parent_signs(const ParentOff &po, const uint32_t *vh, int m) {
     const char *V = reinterpret_cast<const char *>(vh + m * 32);
-    uint32_t s = po.w5 ^ *reinterpret_cast<const uint32_t *>(P + __byte_perm(po.o, 0, 0x4440)) ^
+    uint32_t s = po.w5 ^ (0u - ((po.pq >> m) & 1u)) ^
                  *reinterpret_cast<const uint32_t *>(V + __byte_perm(po.o, 0, 0x4441));
     s ^= *reinterpret_cast<const uint32_t *>(V + 4096 + __byte_perm(po.o, 0, 0x4442));
     if (NKC > 2) s ^= *reinterpret_cast<const uint32_t *>(V + 8192 + __byte_perm(po.o, 0, 0x4443));
@@ -653,10 +654,9 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
 
     uint32_t *s_frag = smem;
     uint32_t *s_w5 = s_frag + (L - 1) * nblk * 256;
-    uint32_t *s_pq = s_w5 + 32;
-    uint32_t *s_vh = s_pq + 1024;
+    uint32_t *s_vh = s_w5 + 32;
     uint32_t *s_dd = s_vh + NKC * 1024;
-    uint32_t *s_g = s_dd + (L - 1) * kDedupSlots * 2;
+    uint32_t *s_g = s_dd + (L - 1) * kDedupSlots;
     {
         if (COSET) {
             for (int i = threadIdx.x; i < (L - 1) * (nblk + 16); i += blockDim.x) s_frag[i] = a.coset[i];
@@ -670,9 +670,8 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
             for (int l = 0; l < 32; ++l) word |= (uint32_t)(__popc(l & v) & 1) << l;
             s_w5[v] = word;
         }
-        for (int i = threadIdx.x; i < 1024; i += blockDim.x) s_pq[i] = (__popc((i >> 5) & i & 31) & 1) ? ~0u : 0u;
         for (int i = threadIdx.x; i < NKC * 1024; i += blockDim.x) s_vh[i] = a.VH[i];
-        for (int i = threadIdx.x; i < (L - 1) * kDedupSlots * 2; i += blockDim.x) s_dd[i] = a.DD[i];
+        for (int i = threadIdx.x; i < (L - 1) * kDedupSlots; i += blockDim.x) s_dd[i] = a.DD[i];
         for (int i = threadIdx.x; i < L * 16; i += blockDim.x) s_g[i] = a.G[(i >> 4) * DPB_MAX_CHILDREN + (i & 15)];
     }
     __syncthreads();
@@ -742,7 +741,7 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
                 const uint32_t pr = (row & 1) && nhalf < 2 ? 0u : beams[(row & 1) * kBeam + (row >> 1)];
                 const ParentOff po = parent_offsets(pr, t, s_w5);
                 uint32_t *sw = reinterpret_cast<uint32_t *>(E);
-                for (int m = lane >> 4; m < nblk; m += 2) sw[m * 16 + row] = parent_signs<NKC>(po, s_pq, s_vh, m);
+                for (int m = lane >> 4; m < nblk; m += 2) sw[m * 16 + row] = parent_signs<NKC>(po, s_vh, m);
             }
             __syncwarp();
             float sc[2][4];  // [token][2 h + (r & 1)]: this lane's children 8 h + 2 q4 + (r & 1)
@@ -838,7 +837,7 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
                             sc[tk][e] = standardise(sc[tk][e], (tk ? p1 : p0) ^ gl[8 * (e >> 1) + 2 * q4 + (e & 1)],
                                                     a, a.status);
             }
-            const uint32_t *ddl = s_dd + (l - 1) * kDedupSlots * 2;
+            const uint32_t *ddl = s_dd + (l - 1) * kDedupSlots;
             uint32_t pcur = p0;
             if constexpr (WIDE) {
                 // repeats over all pairs S' < S < beam of the 16 slots: pair q = lane + 32 r
@@ -854,10 +853,10 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
                     const uint32_t delta = beams[S] ^ beams[Sp];
                     uint32_t h = dedup_hash(delta);
                     for (int probe = 0; probe < kDedupSlots; ++probe) {
-                        const uint32_t key = ddl[2 * h];
-                        if (key == 0u) break;
-                        if (key == delta + 1u) {
-                            const uint32_t bit = (uint32_t)S * 16u + (ddl[2 * h + 1] & 0xffu);
+                        const uint32_t ent = ddl[h];
+                        if (ent == 0u) break;
+                        if ((ent >> 4) == delta + 1u) {
+                            const uint32_t bit = (uint32_t)S * 16u + (ent & 15u);
                             atomicOr(&dup[bit >> 5], 1u << (bit & 31u));
                         }
                         h = (h + 1u) & (kDedupSlots - 1);
@@ -886,9 +885,9 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
                         delta = bt[ps] ^ bt[psp];
                         uint32_t h = dedup_hash(delta);
                         for (int probe = 0; probe < kDedupSlots; ++probe) {
-                            const uint32_t key = ddl[2 * h];
-                            if (key == 0u) break;
-                            if (key == delta + 1u) {
+                            const uint32_t ent = ddl[h];
+                            if (ent == 0u) break;
+                            if ((ent >> 4) == delta + 1u) {
                                 hit = true;
                                 break;
                             }
@@ -901,10 +900,10 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
                         if (hit) {
                             uint32_t h = dedup_hash(delta);
                             for (int probe = 0; probe < kDedupSlots; ++probe) {
-                                const uint32_t key = ddl[2 * h];
-                                if (key == 0u) break;
-                                if (key == delta + 1u) {
-                                    const uint32_t bit = (uint32_t)ps * 16u + (ddl[2 * h + 1] & 0xffu);
+                                const uint32_t ent = ddl[h];
+                                if (ent == 0u) break;
+                                if ((ent >> 4) == delta + 1u) {
+                                    const uint32_t bit = (uint32_t)ps * 16u + (ent & 15u);
                                     atomicOr(&dup[bit >> 5], 1u << (bit & 31u));
                                 }
                                 h = (h + 1u) & (kDedupSlots - 1);

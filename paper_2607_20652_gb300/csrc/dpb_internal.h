@@ -28,8 +28,9 @@ struct dpb_plan {
     // Tensor-core encoder tables (built when mma_encode is set):
     //  FRAG[l-1][m][lane][8]: the generator signs gamma_j of level l over
     //    32-coordinate block m, as bf16 +-1 pairs in mma.sync B-fragment order;
-    //  DD[l-1][kDedupSlots][2]: open-addressing table of the differences
-    //    g_j ^ g_j' (j != j') of level l, value (j | j' << 8), key + 1 (0 = empty).
+    //  DD[l-1][kDedupSlots]: open-addressing table of the differences
+    //    g_j ^ g_j' (j != j') of level l below 2^bits[l-1], one word per
+    //    entry: (difference + 1) << 4 | j (0 = empty).
     bool mma_encode = false;
     std::vector<uint32_t> FRAG;
     std::vector<uint32_t> DD;

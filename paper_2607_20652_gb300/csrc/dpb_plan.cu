@@ -154,6 +154,8 @@ void build_mma_tables(dpb_plan *p) {
     bool ok = c.dtype == DPB_BF16 && c.d % 32 == 0 && c.d >= 32 && c.d <= 1024 && c.levels >= 2 &&
               c.select_mode == DPB_SELECT_GLOBAL && c.beam >= 1 && c.beam <= 16 && c.k >= c.beam && c.k <= 256;
     for (int l = 1; l < c.levels && ok; ++l) ok = c.children[l] == 16;
+    // a difference + 1 below 2^bits[L-2] must fit the 28 key bits of a DD entry
+    ok = ok && c.bits[c.levels - 2] <= 27;
     const int nblk = c.d / 32;
     // every level's fragments, the tables and the warps' lists share one block
     p->mma_encode = ok;
@@ -173,9 +175,9 @@ void build_mma_tables(dpb_plan *p) {
                     const int ia = 32 * m + frag_coord(q4, pair, 0), ib = 32 * m + frag_coord(q4, pair, 1);
                     p->FRAG[(((size_t)(l - 1) * nblk + m) * 32 + lane) * 8 + w] = sign_bf16(g, ia) | (sign_bf16(g, ib) << 16);
                 }
-    p->DD.assign((size_t)(c.levels - 1) * kDedupSlots * 2, 0u);
+    p->DD.assign((size_t)(c.levels - 1) * kDedupSlots, 0u);
     for (int l = 1; l < c.levels; ++l) {
-        uint32_t *tab = &p->DD[(size_t)(l - 1) * kDedupSlots * 2];
+        uint32_t *tab = &p->DD[(size_t)(l - 1) * kDedupSlots];
         const uint32_t *g = &p->G[(size_t)l * DPB_MAX_CHILDREN];
         // parents of level l lie below 2^bits[l-1], so only differences below
         // that bound can make two parents share a child
@@ -186,9 +188,8 @@ void build_mma_tables(dpb_plan *p) {
                 const uint32_t delta = g[j] ^ g[jj];
                 if (delta >= bound) continue;
                 uint32_t h = dedup_hash(delta);
-                while (tab[2 * h] != 0) h = (h + 1) & (kDedupSlots - 1);
-                tab[2 * h] = delta + 1;
-                tab[2 * h + 1] = (uint32_t)j | ((uint32_t)jj << 8);
+                while (tab[h] != 0) h = (h + 1) & (kDedupSlots - 1);
+                tab[h] = ((delta + 1) << 4) | (uint32_t)j;
             }
     }
 }
