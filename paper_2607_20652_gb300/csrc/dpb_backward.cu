@@ -156,7 +156,7 @@ constexpr int kChunkBlocks = 4;                       // 32-coordinate blocks pe
 constexpr int kTabStride = 17;                        // 16 entries + 1 pad (bank spread)
 constexpr int kChunkTables = kChunkBlocks * 8 * kTabStride;  // nibble tables of a chunk (words)
 constexpr int kScratchWords = pad64(kSweepWords > kChunkTables ? kSweepWords : kChunkTables);
-constexpr int kBwdWarps = 8;
+constexpr int kBwdWarps = 14;  // two blocks of 14 warps fill an SM's shared memory at d = 768
 static_assert(kChunkBlocks == 4, "the analysis gives a code 4 lanes, one per block of a chunk");
 
 // Per-warp words: the scratch (a sweep's tables, or a chunk's nibble tables;
@@ -300,7 +300,7 @@ __device__ __forceinline__ void analyse(const BwdWarp &w, int nh, int d, const u
 }
 
 template <typename Tio, int NKC, bool VEC>
-__global__ void __launch_bounds__(kBwdWarps * 32, 3) backward_lut_kernel(BackwardArgs a, int t) {
+__global__ void __launch_bounds__(kBwdWarps * 32, 2) backward_lut_kernel(BackwardArgs a, int t) {
     extern __shared__ __align__(16) uint32_t smem_raw[];
     uint32_t *smem = aligned_smem<256>(smem_raw);
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
@@ -480,10 +480,15 @@ int grid_for(const dpb_plan *p, int64_t T, int warps) {
 
 template <typename Tio, int NKC, bool VEC>
 cudaError_t run_backward_lut(const dpb_plan *p, const BackwardArgs &a, int64_t T, cudaStream_t stream) {
-    const int warps = kBwdWarps;
-    const size_t smem = 256 /* alignment */ +
-                        sizeof(uint32_t) * ((size_t)bwd_block_words(p->cfg.d, NKC) +
-                                            (size_t)warps * bwd_warp_words(p->cfg.d, p->code_len));
+    // kBwdWarps per block (two blocks per SM at d = 768, k = 64), fewer when
+    // long rows or codes would not fit
+    auto smem_for = [&](int w) {
+        return 256 /* alignment */ + sizeof(uint32_t) * ((size_t)bwd_block_words(p->cfg.d, NKC) +
+                                                         (size_t)w * bwd_warp_words(p->cfg.d, p->code_len));
+    };
+    int warps = kBwdWarps;
+    while (warps > 1 && smem_for(warps) > kMaxSmemPerBlock) warps /= 2;
+    const size_t smem = smem_for(warps);
     const cudaError_t e = allow_smem((const void *)backward_lut_kernel<Tio, NKC, VEC>, smem);
     if (e != cudaSuccess) return e;
     backward_lut_kernel<Tio, NKC, VEC><<<grid_for(p, T, warps), warps * 32, smem, stream>>>(a, p->t);
