@@ -707,6 +707,196 @@ def run_e2e(plan, x, gy, args, device, stream, world):
 
 
 # ---------------------------------------------------------------------------
+# the small global-mode workloads (supplementary lines; they fit in L2)
+# ---------------------------------------------------------------------------
+
+L2_FLUSH_BYTES = 512 << 20  # written between steps: more than the 129 MB L2
+
+
+def run_global_small(args, world, rank, local):
+    """The tiny (fp32, encode + decode + backward) and GPT-2-width (bf16 with 5%
+    outlier rows, encode + decode) workloads. Their working sets fit in L2, so
+    every step is timed on its own (CUDA events around its calls) after a
+    512 MB write that flushes L2; the line's time is the mean of those steps.
+    A seeded sample of rows (every row of tiny) is checked against the oracle
+    on the last step's outputs."""
+    import torch
+    from paper_2607_20652_gb300 import configs, dpb, inputs
+    device = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(device)
+    w = dict(configs.WORKLOADS[args.workload])
+    T, d = w["T"], w["d"]
+    bwd = w["passes"] == "fwd+bwd"
+    plan = dpb.Plan(d=d, levels=w["levels"], m_bits=w["m_bits"], children=w["children"], beam=w["beam"],
+                    k=w["k"], dtype=w["dtype"], norm_match=1)
+    seed = shard_seed(w["seed"], rank)
+    xh = inputs.gaussian_rows(T, d, seed, w.get("outlier_frac", 0.0), w.get("outlier_scale", 10.0))
+    gyh = inputs.normal((T, d), seed + w.get("grad_seed", 1))
+    if w["dtype"] == "bf16":
+        xh, gyh = inputs.to_bf16(xh), inputs.to_bf16(gyh)
+    x = torch.from_numpy(xh).to(device).to(plan.torch_dtype)
+    gy = torch.from_numpy(gyh).to(device).to(plan.torch_dtype)
+    k = plan.code_len
+    idx = torch.empty((T, k), dtype=torch.int32, device=device)
+    val = torch.empty((T, k), dtype=torch.float32, device=device)
+    xn = torch.empty((T,), dtype=torch.float32, device=device)
+    y, gx = torch.empty_like(x), torch.empty_like(x)
+    gv = torch.empty((T, k), dtype=torch.float32, device=device)
+    rk = torch.empty((T, d), dtype=torch.float32, device=device) if bwd else None
+    ws = plan.workspace(T, device)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=device)
+    stream = torch.cuda.current_stream(device)
+    stages = ["encode", "decode"] + (["backward"] if bwd else [])
+
+    def step(ev=None):
+        flush.fill_(1.0)
+        if ev:
+            ev[0].record(stream)
+        dpb.encode(plan, x, idx=idx, val=val, xnorm=xn, workspace=ws, stream=stream)
+        if ev:
+            ev[1].record(stream)
+        dpb.decode(plan, idx, val, xn, y=y, workspace=ws, stream=stream, r_out=rk)
+        if ev:
+            ev[2].record(stream)
+        if bwd:
+            dpb.backward(plan, x, idx, val, gy, grad_x=gx, grad_val=gv, workspace=ws, stream=stream, r=rk)
+            if ev:
+                ev[3].record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize(device)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(len(stages) + 1)] for _ in range(args.steps)]
+    clocks = ClockSampler(None)
+    clocks.start()
+    time.sleep(0.3)
+    barrier(world)
+    for e in evs:
+        step(e)
+    torch.cuda.synchronize(device)
+    barrier(world)
+    clk = clocks.stop()
+    ms = statistics.mean(e[0].elapsed_time(e[-1]) for e in evs)
+    ms_max = max_over_ranks(ms, world, device)
+    kern_ms = {n: statistics.mean(e[j].elapsed_time(e[j + 1]) for e in evs) for j, n in enumerate(stages)}
+    idx_np = idx.cpu().numpy()
+    k_hash = float(np.mean(np.sum(idx_np >= d, axis=1)))
+    peaks, src = load_peaks()
+    s_el = 4 if w["dtype"] == "f32" else 2
+    work = algorithmic_work(plan.config, T, k_hash, s_el)
+    kernels = {n: {"ms": round(v, 4), **{kk: vv for kk, vv in
+                                         roofline_for(n, work[n], v / 1e3, peaks, src, clocks=clk).items()
+                                         if kk in ("bound", "pipe", "frac", "t_roofline_us")}}
+               for n, v in kern_ms.items()}
+    step_roof_us = sum(kernels[n]["t_roofline_us"] for n in kernels)
+    dom = max(kern_ms, key=kern_ms.get)
+    line = {
+        "metric": f"DPB tokens/sec ({'+'.join(stages)}), {args.workload} config, 1 GB300",
+        "value": round(whole_job_rate(T, world, 1, ms_max / 1e3), 1), "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_max, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": w["dtype"], "data": "synthetic",
+        "config": {"workload": args.workload, "T_per_gpu": T, "d": d, "features": 2 ** w["m_bits"],
+                   "levels": w["levels"], "children": w["children"], "beam": w["beam"], "k": w["k"],
+                   "inputs": "x ~ N(0,1)" + (f", {int(100 * w['outlier_frac'])}% of rows x{w['outlier_scale']:g}"
+                                             if w.get("outlier_frac") else "") + f", {w['dtype']}",
+                   "l2": "512 MB written before every step (flush); each step timed on its own"},
+        "roofline": roofline_for(dom, work[dom], kern_ms[dom] / 1e3, peaks, src, clocks=clk),
+        "step_roofline": {"t_roofline_us": round(step_roof_us, 2), "t_measured_us": round(1e3 * ms_max, 2),
+                          "frac": round(step_roof_us / (1e3 * ms_max), 4)},
+        "kernels": kernels, "k_hash": round(k_hash, 2), "gpu_launches": len(stages) * args.steps, "clocks": clk,
+        "device_status": dpb.workspace_status(ws),
+    }
+    if rank == 0 and world == 1 and not args.no_parity:
+        line["parity"] = small_parity(w, plan, xh, gyh if bwd else None,
+                                      {"idx": idx, "val": val, "xnorm": xn, "y": y, "gx": gx if bwd else None,
+                                       "gv": gv if bwd else None, "r": rk})
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = small_cpu_baseline(w, xh, gyh if bwd else None, plan)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    return 0
+
+
+def _small_ref(w, plan):
+    import oracle
+    c = plan.config
+    return oracle.resolve(d=c["d"], m_bits=w["m_bits"], levels=c["levels"], children=c["children"],
+                          beam=c["beam"], k=c["k"], seed=c["generator_seed"], norm_match=c["norm_match"],
+                          t=c["field_t"], poly=c["field_poly"], bits=c["bits"])
+
+
+def small_parity(w, plan, xh, gyh, out):
+    """Oracle leg: every row of tiny, 256 seeded rows of GPT-2 width, checked
+    by the rules of the -m gpu parity tests."""
+    import oracle
+    from paper_2607_20652_gb300 import inputs
+    from tests import parity
+    T = len(xh)
+    rows = np.arange(T) if T <= 256 else np.unique(np.concatenate([inputs.sample_rows(T, 256, 77), [0, T - 1]]))
+    ref = _small_ref(w, plan)
+    bf16 = w["dtype"] == "bf16"
+    tol = parity.TOL["bf16" if bf16 else "f32"]
+    import torch
+
+    def host(v):
+        if v is None:
+            return None
+        return (v.cpu().numpy() if v.dtype == torch.int32 else v.float().cpu().numpy())[rows]
+
+    get = {kk: host(v) for kk, v in out.items()}
+    xr = xh[rows].astype(np.float64)
+    res = {"tokens": int(len(rows)), "sample": "every row" if T <= 256 else f"{len(rows)} seeded rows"}
+    try:
+        idx_o, val_o, xn_o, gap = oracle.encode(ref, xr)
+        parity.check_code_order(get["idx"], get["val"])
+        near, worst = parity.compare_codes(get["idx"], get["val"], idx_o, val_o, gap, xn_o)
+        res.update(near_ties=near, val_err=worst)
+        y_o = oracle.decode(ref, get["idx"], get["val"].astype(np.float64), get["xnorm"].astype(np.float64))
+        res["y_err"] = parity.check_elementwise(get["y"], y_o, tol, bf16, "decode y")
+        if gyh is not None:
+            r_o = oracle.decode(ref, get["idx"], get["val"].astype(np.float64), norm_match=0)
+            res["r_err"] = parity.check_elementwise(get["r"], r_o, 1e-5, False, "kept r")
+            gx_o, gv_o = oracle.backward(ref, xr, get["idx"], get["val"].astype(np.float64),
+                                         gyh[rows].astype(np.float64))
+            res["gx_err"] = parity.check_elementwise(get["gx"], gx_o, tol, bf16, "grad_x")
+            res["gv_err"] = parity.check_elementwise(get["gv"], gv_o, 1e-5, False, "grad_val")
+        res["ok"] = True
+    except AssertionError as e:
+        res.update(ok=False, failure=str(e)[:300])
+    for kk in ("val_err", "y_err", "r_err", "gx_err", "gv_err"):
+        if kk in res:
+            res[kk] = float(f"{res[kk]:.3e}")
+    return res
+
+
+def small_cpu_baseline(w, xh, gyh, plan):
+    """The oracle on the host cores over the same rows (all of tiny; the first
+    2048 of GPT-2 width), as for the wide workload."""
+    import oracle
+    ref = _small_ref(w, plan)
+    n = min(len(xh), 2048)
+    x = xh[:n].astype(np.float64)
+    cores = host_cores()
+    cuts = np.linspace(0, n, cores + 1).astype(int)
+
+    def part(i):
+        xs = x[cuts[i]:cuts[i + 1]]
+        idx, val, xn, _ = oracle.encode(ref, xs)
+        oracle.decode(ref, idx, val, xn)
+        if gyh is not None:
+            oracle.backward(ref, xs, idx, val, gyh[cuts[i]:cuts[i + 1]].astype(np.float64))
+
+    import concurrent.futures
+    t0 = time.perf_counter()
+    with concurrent.futures.ThreadPoolExecutor(max_workers=cores) as ex:
+        list(ex.map(part, range(cores)))
+    secs = time.perf_counter() - t0
+    return {"value": round(n / secs, 2), "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "sample": f"first {n} tokens of the {'tiny' if len(xh) <= 256 else 'gpt2'} workload, "
+                      f"C oracle (fp64) in {cores} threads over token ranges; {secs:.2f} s"}
+
+
+# ---------------------------------------------------------------------------
 # the paper's per-level layouts (supplementary lines; the headline is "wide")
 # ---------------------------------------------------------------------------
 
@@ -1026,11 +1216,12 @@ def main(argv=None):
     ap.add_argument("--standardise", action="store_true",
                     help="live standardisation tables and the per-step EMA update in the timed step")
     ap.add_argument("--no-dense", action="store_true", help="gpt2small: skip the dense model of the same shape")
-    ap.add_argument("--workload", default=WORKLOAD, choices=[WORKLOAD, "paper3l", "paper2l", "gpt2small", "sweep"],
+    ap.add_argument("--workload", default=WORKLOAD,
+                    choices=[WORKLOAD, "tiny", "gpt2", "paper3l", "paper2l", "gpt2small", "sweep"],
                     help="wide (the headline, global selection) or one of the paper's per-level layouts")
     args = ap.parse_args(argv)
     if args.steps is None:
-        args.steps = {WORKLOAD: 1500, "paper3l": 200, "paper2l": 200}.get(args.workload, 20)
+        args.steps = {WORKLOAD: 1500, "paper3l": 200, "paper2l": 200, "tiny": 200, "gpt2": 200}.get(args.workload, 20)
     world, rank, local = dist_env()
     if args.warmup < 3 and args.impl == "ours":
         print("note: at least 3 warm-up steps are used", file=sys.stderr)
@@ -1041,6 +1232,8 @@ def main(argv=None):
         return run_transformer(args, world, rank, local)
     if args.workload == "sweep":
         return run_sweep(args, world, rank, local)
+    if args.workload in ("tiny", "gpt2"):
+        return run_global_small(args, world, rank, local)
     if args.workload != WORKLOAD:
         return run_per_level(args, world, rank, local)
     return run_ours(args, world, rank, local)
