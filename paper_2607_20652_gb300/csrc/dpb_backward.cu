@@ -156,7 +156,8 @@ constexpr int kChunkBlocks = 4;                       // 32-coordinate blocks pe
 constexpr int kTabStride = 17;                        // 16 entries + 1 pad (bank spread)
 constexpr int kChunkTables = kChunkBlocks * 8 * kTabStride;  // nibble tables of a chunk (words)
 constexpr int kScratchWords = pad64(kSweepWords > kChunkTables ? kSweepWords : kChunkTables);
-constexpr int kBwdWarps = 14;  // two blocks of 14 warps fill an SM's shared memory at d = 768
+constexpr int kBwdWarps = 14;  // at most; two blocks of 14 fill an SM's shared memory at d = 768
+constexpr size_t kSmemPerSm = 228 * 1024;
 static_assert(kChunkBlocks == 4, "the analysis gives a code 4 lanes, one per block of a chunk");
 
 // Per-warp words: the scratch (a sweep's tables, or a chunk's nibble tables;
@@ -480,14 +481,23 @@ int grid_for(const dpb_plan *p, int64_t T, int warps) {
 
 template <typename Tio, int NKC, bool VEC>
 cudaError_t run_backward_lut(const dpb_plan *p, const BackwardArgs &a, int64_t T, cudaStream_t stream) {
-    // kBwdWarps per block (two blocks per SM at d = 768, k = 64), fewer when
-    // long rows or codes would not fit
+    // The warps per block that put the most warps on an SM: shared memory
+    // (228 KB per SM, 1 KB of it reserved per block) and the 2 x kBwdWarps
+    // warps that the registers allow (kBwdWarps = 14: two blocks at d = 768,
+    // k = 64; two of 10 at d = 1024, k = 112)
     auto smem_for = [&](int w) {
         return 256 /* alignment */ + sizeof(uint32_t) * ((size_t)bwd_block_words(p->cfg.d, NKC) +
                                                          (size_t)w * bwd_warp_words(p->cfg.d, p->code_len));
     };
-    int warps = kBwdWarps;
-    while (warps > 1 && smem_for(warps) > kMaxSmemPerBlock) warps /= 2;
+    int warps = 1, best = 0;
+    for (int w = kBwdWarps; w >= 1; --w) {
+        if (smem_for(w) > kMaxSmemPerBlock) continue;
+        const int blocks = std::min((int)(kSmemPerSm / (smem_for(w) + 1024)), 2 * kBwdWarps / w);
+        if (blocks * w > best) {
+            best = blocks * w;
+            warps = w;
+        }
+    }
     const size_t smem = smem_for(warps);
     const cudaError_t e = allow_smem((const void *)backward_lut_kernel<Tio, NKC, VEC>, smem);
     if (e != cudaSuccess) return e;
