@@ -334,13 +334,15 @@ def parity_check(ref, rows, x_rows, gy_rows, out):
     xr = x_rows.astype(np.float64)
     gi, gvl, gxn = out["idx"], out["val"], out["xnorm"]
     res = {"tokens": int(len(rows)), "sample": f"{len(rows)} seeded rows of the timed batch (oracle-built x)",
-           "rule": "indices as sets except near-ties (gap < 1e-5 relative, counted); val within 1e-5 |x|; "
+           "rule": "indices as sets except near-ties (gap < 1e-5 relative, counted; their values checked against "
+                   "their features' scores); val within 1e-5 |x|; "
                    "y, grad_x within 2e-2 max(|ref_i|, row rms) + 1 bf16 spacing, r and grad_val within 1e-5, "
                    "element by element, decode and backward on the GPU's own code"}
     try:
         idx_o, val_o, xn_o, gap = oracle.encode(ref, xr)
         parity.check_code_order(gi, gvl)
         near, worst_val = parity.compare_codes(gi, gvl, idx_o, val_o, gap, xn_o)
+        parity.check_near_tie_values(ref, xr, gi, gvl, gap < parity.NEAR_TIE)
         res.update(near_ties=near, near_tie_tokens=[int(r) for r in np.asarray(rows)[gap < parity.NEAR_TIE]][:16],
                    val_err=worst_val)
         assert np.all(np.abs(gxn - xn_o) <= 1e-5 * np.maximum(xn_o, 1e-30)), "|x| differs"
@@ -850,6 +852,7 @@ def small_parity(w, plan, xh, gyh, out):
         idx_o, val_o, xn_o, gap = oracle.encode(ref, xr)
         parity.check_code_order(get["idx"], get["val"])
         near, worst = parity.compare_codes(get["idx"], get["val"], idx_o, val_o, gap, xn_o)
+        parity.check_near_tie_values(ref, xr, get["idx"], get["val"], gap < parity.NEAR_TIE)
         res.update(near_ties=near, val_err=worst)
         y_o = oracle.decode(ref, get["idx"], get["val"].astype(np.float64), get["xnorm"].astype(np.float64))
         res["y_err"] = parity.check_elementwise(get["y"], y_o, tol, bf16, "decode y")

@@ -100,6 +100,7 @@ def _check_all(plan, ref, x, g, gy=None, mu=None, sigma=None, rows=None):
     gi, gvl, gxn = g["idx"][rows], g["val"][rows], g["xnorm"][rows]
     parity.check_code_order(gi, gvl)
     near, worst_val = parity.compare_codes(gi, gvl, idx_o, val_o, gap, xn_o)
+    parity.check_near_tie_values(ref, xr, gi, gvl, gap < parity.NEAR_TIE, mu, sigma)
     assert np.all(np.abs(gxn - xn_o) <= 1e-5 * np.maximum(xn_o, 1e-30))
     # decode, checked on the GPU's own code
     y_o = oracle.decode(ref, gi, gvl.astype(np.float64), gxn.astype(np.float64))
@@ -378,6 +379,7 @@ def test_coset_scoring_matches_the_oracle(T):
         assert g["status"] == 0
         parity.check_code_order(g["idx"][rows], g["val"][rows])
         near, worst = parity.compare_codes(g["idx"][rows], g["val"][rows], idx_o, val_o, gap, xn_o)
+        parity.check_near_tie_values(ref, x[rows], g["idx"][rows], g["val"][rows], gap < parity.NEAR_TIE)
         assert near <= max(2, len(rows) // 10), f"{near} near-ties of {len(rows)} tokens"
         parity.record(tokens=len(rows), near_ties=near, val=worst)
         reports.append((near, worst))

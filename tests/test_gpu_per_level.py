@@ -64,6 +64,7 @@ def _check(plan, ref, kls, x, g, mu=None, sigma=None, gy=None):
         parity.check_code_order(g["idx"][:, seg], g["val"][:, seg])
         n, w = parity.compare_codes(g["idx"][:, seg], g["val"][:, seg], idx_o[:, seg], val_o[:, seg], gap, xn_o)
         near, worst, off = max(near, n), max(worst, w), off + K
+    parity.check_near_tie_values(ref, xr, g["idx"], g["val"], gap < parity.NEAR_TIE, mu, sigma)
     y_o = oracle.decode(ref, g["idx"], g["val"].astype(np.float64), g["xnorm"].astype(np.float64))
     e = parity.rel_rows(g["y"], y_o)
     tol = parity.TOL["bf16"]

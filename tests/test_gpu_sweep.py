@@ -62,6 +62,7 @@ def test_sweep_point_full_size_sampled(w):
     idx_o, val_o, xn_o, gap = oracle.encode(ref, xr)
     parity.check_code_order(gi, gvl)
     near, worst = parity.compare_codes(gi, gvl, idx_o, val_o, gap, xn_o)
+    parity.check_near_tie_values(ref, xr, gi, gvl, gap < parity.NEAR_TIE)
     assert near <= max(2, len(rows) // 10), f"{near} near-ties of {len(rows)} tokens"
     assert np.all(np.abs(gxn - xn_o) <= 1e-5 * xn_o)
     tol = parity.TOL["bf16"]

@@ -53,3 +53,19 @@ def test_summary_counts_tokens_and_near_ties():
     lines = parity.summary_lines(rep)
     assert lines[0].startswith("a: 100 tokens, 2 near-ties")
     assert "150 tokens, 2 near-ties (1.33%)" in lines[-1] and "y 3.0e-03" in lines[-1]
+
+
+def test_near_tie_values_are_checked_against_each_features_score():
+    # a near-tie token's code need not be the oracle's, but each entry's value
+    # must be its feature's score <phi_i, x>; a wrong value is caught
+    import oracle
+    from paper_2607_20652_gb300 import inputs
+    ref = oracle.resolve(d=64, m_bits=12, levels=3, children=16, beam=4, k=8)
+    x = inputs.gaussian_rows(3, 64, 5).astype(np.float64)
+    idx, val, _, _ = oracle.encode(ref, x)
+    near = np.array([True, False, True])
+    assert parity.check_near_tie_values(ref, x, idx, val, near) == 16
+    bad = val.copy()
+    bad[2, 5] *= 1.001
+    with pytest.raises(AssertionError, match="near-tie token 2"):
+        parity.check_near_tie_values(ref, x, idx, bad, near)
