@@ -21,8 +21,11 @@
 //    shift moves to the bf16 sign positions;
 //  - B (Delta_l x 64 bf16, the generators' +-1 signs in the same order) is
 //    one bulk copy of the plan's precomputed tile;
-//  - one thread issues the 4 MMAs of the chunk and commits them to an
-//    mbarrier that frees the chunk's buffers; scores accumulate in TMEM.
+//  - a ninth warp's lane 0 issues the MMAs of a chunk once the 8 token
+//    warps have arrived on the A stage's mbarrier and the generator tile has
+//    landed, and commits them to an mbarrier that frees the chunk's buffers;
+//    scores accumulate in TMEM. The token warps build the next A stage
+//    meanwhile (two stages), so no warp both builds A and waits to issue.
 // Every mbarrier wait is bounded; a wait that gives up sets
 // DPB_DEV_TIMEOUT and stops the block, which then waits (again bounded) for
 // its bulk copies and MMAs still in flight and frees its TMEM.
@@ -47,6 +50,8 @@ namespace dpb {
 namespace {
 
 constexpr int kTokens = 8;      // tokens per block, one per warp
+constexpr int kThreads = (kTokens + 1) * 32;  // and a ninth warp, whose lane 0 issues the MMAs
+constexpr int kIssuer = kTokens * 32;         // that thread
 constexpr int kRows = 32;       // tensor-core rows per token (parent slots)
 constexpr int kChunk = 64;      // coordinates per K chunk
 constexpr int kATile = 128 * kChunk * 2;  // one M = 128 tile of a chunk
@@ -97,7 +102,7 @@ __host__ __device__ inline Layout layout(int d, int levels, int kvh, int dmax, i
     l.w5 = l.g + levels * 256 * 4;
     l.par = l.w5 + 32 * 4;
     l.mbar = l.par + kTokens * kRows * 4;
-    l.total = l.mbar + 2 * kMaxStages * 8 + 16;
+    l.total = l.mbar + (2 * kMaxStages + 2) * 8 + 16;
     return l;
 }
 
@@ -381,7 +386,7 @@ __device__ __forceinline__ float standardise(float s, uint32_t c, const Args &a,
 
 // ---- the kernel ----------------------------------------------------------------------
 
-__global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
+__global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
     extern __shared__ __align__(1024) uint8_t smem[];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int d = a.d, nblk = a.nblk, L = a.levels;
@@ -392,8 +397,9 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
     uint32_t *vh = reinterpret_cast<uint32_t *>(smem + lay.vh);
     uint32_t *gs = reinterpret_cast<uint32_t *>(smem + lay.g);
     uint32_t *w5 = reinterpret_cast<uint32_t *>(smem + lay.w5);
-    uint64_t *mbar = reinterpret_cast<uint64_t *>(smem + lay.mbar);  // full_b[stages], mma_done[stages]
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(mbar + 2 * kMaxStages);
+    // full_b[stages], mma_done[stages], a_full[2]
+    uint64_t *mbar = reinterpret_cast<uint64_t *>(smem + lay.mbar);
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(mbar + 2 * kMaxStages + 2);
     WarpBufs wb;
     wb.par = reinterpret_cast<uint32_t *>(smem + lay.par) + warp * kRows;
     wb.z = reinterpret_cast<float *>(sB + warp * kSelBytes);
@@ -408,6 +414,9 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
     if (tid == 0) {
         for (int i = 0; i < 2 * kMaxStages; ++i)
             asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(mbar + i)));
+        for (int i = 0; i < 2; ++i)  // an A stage is built once each of the token warps arrives
+            asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(mbar + 2 * kMaxStages + i)),
+                         "r"(kTokens));
         asm volatile("fence.mbarrier_init.release.cluster;");
     }
     if (warp == 0) {
@@ -428,12 +437,14 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
     auto mma_done = [&](uint32_t g) { return mbar0 + 8u * (kMaxStages + g % (uint32_t)nbs); };
     auto phase = [&](uint32_t g) { return (g / (uint32_t)nbs) & 1u; };
     auto stage_b = [&](uint32_t g) { return sB + (g % (uint32_t)nbs) * a.dmax * 128; };
-    uint32_t G = 0;  // chunks whose MMAs were committed
+    // A stage g & 1 is built for chunk g the (g / 2)-th time
+    auto a_full = [&](uint32_t g) { return mbar0 + 8u * (2 * kMaxStages + (g & 1u)); };
+    uint32_t G = 0;  // chunks of the levels done so far (every thread)
     bool failed = false;
-    // thread 0: generator tiles are copied and consumed in chunk order; the
-    // copies of chunks [consumed, issued) are in flight
-    uint32_t issued = 0, consumed = 0;
-    bool tfail = false;  // thread 0: a wait of its own gave up
+    // the issuer: generator tiles are copied and consumed in chunk order (the
+    // copies of chunks [consumed, issued) are in flight); Gc chunks committed
+    uint32_t issued = 0, consumed = 0, Gc = 0;
+    bool tfail = false;  // a wait of this thread gave up
     auto issue_b = [&](uint32_t g, const uint32_t *src, int D) {
         copy_b(stage_b(g), src, D, full_b(g));
         issued = g + 1;
@@ -444,7 +455,7 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
 
     for (int64_t grp = blockIdx.x; grp < ngroups && !failed; grp += gridDim.x) {
         const int64_t tok = grp * kTokens + warp;
-        const bool live = tok < a.T;
+        const bool live = warp < kTokens && tok < a.T;
         // ---- the row in the pair layout: word m*16 + i = (x[32m+i], x[32m+i+16]); |x|; level 0 ----
         if (live) {
             const uint4 *row = reinterpret_cast<const uint4 *>(a.x + tok * d);
@@ -473,7 +484,7 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
             if (a.mu)
                 for (int i = lane; i < d; i += 32) standardise(0.f, (uint32_t)i, a, a.status);
             select_level(scan0, min(32, d / 32 * 32), a.kl[0], wb, a, tok, a.off[0], L > 1);
-        } else {
+        } else if (warp < kTokens) {
             wb.par[lane] = 0u;
             __syncwarp();
         }
@@ -506,105 +517,107 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
             const uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(D >> 3) << 17) | (8u << 24);
             const uint32_t *gt = a.GT + a.gt_off[l];
             const uint32_t G0 = G;
-            // the level's first nbs - 1 tiles (every earlier MMA is done, so
-            // every stage is free)
-            // the first tiles: every stage with three or more (all free here),
-            // one ahead of the first chunk with two
+            // the level's first tiles (every earlier MMA is done, so every stage
+            // is free): every stage with three or more, one with two
             const int ahead = nbs >= 3 ? nbs : nbs - 1;
-            if (tid == 0)
+            bool bfail = false;  // a builder's wait gave up
+            if (tid == kIssuer) {
+                // ---- the issuer: for each chunk, once its A stage is built and
+                // its generator tile has landed, the MMAs and their commit; it
+                // refills a generator stage once the MMAs that read it are done
                 for (int c = 0; c < min(ahead, nch); ++c) issue_b(G0 + c, gt + (int64_t)c * D * 32, D);
-            for (int c = 0; c < nch; ++c) {
-                const uint32_t g = G0 + c;
-                {
-                    // A stage g & 1 is free once the MMAs of chunk g - 2 are done
-                    bool ok = true;
-                    if (c >= 2) ok = mbar_wait(mma_done(g - 2), phase(g - 2), a.spin);
-                    if (__syncthreads_or(!ok || tfail)) {  // every thread leaves together
-                        failed = true;
-                        break;
-                    }
-                }
-                uint8_t *As = sA + (g & 1u) * 2 * kATile;
-#pragma unroll
-                for (int tt = 0; tt < 2; ++tt) {
-                    if (tt < ntiles) {
-                        const int m = 2 * c + hb;
-                        const bool rv = irv[tt];
-                        uint32_t sw = iw5[tt] ^ (0u - (uint32_t)(__popc((uint32_t)m & iu[tt]) & 1));
-#pragma unroll
-                        for (int k = 0; k < 4; ++k)
-                            if (k < a.kvh) sw ^= vh[(k * nblk + m) * 32 + ihv[tt][k]];
-                        const uint4 *xs = reinterpret_cast<const uint4 *>(ixt[tt] + m * 16);
-                        uint8_t *At = As + tt * kATile;
-#pragma unroll
-                        for (int q = 0; q < 4; ++q) {
-                            const uint4 xv = xs[q];
-                            const int sh = 15 - 4 * q;
-                            uint4 av;
-                            av.x = rv ? xv.x ^ ((sw << sh) & 0x80008000u) : 0u;
-                            av.y = rv ? xv.y ^ ((sw << (sh - 1)) & 0x80008000u) : 0u;
-                            av.z = rv ? xv.z ^ ((sw << (sh - 2)) & 0x80008000u) : 0u;
-                            av.w = rv ? xv.w ^ ((sw << (sh - 3)) & 0x80008000u) : 0u;
-                            *reinterpret_cast<uint4 *>(At + (rr >> 3) * 1024 + (4 * hb + q) * 128 + (rr & 7) * 16) =
-                                av;
-                        }
-                    }
-                }
-                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-                __syncthreads();
-                if (tid == 0) {
-                    if (!mbar_wait(full_b(g), phase(g), a.spin)) {
-                        // no MMA for this chunk (the commit below still arrives);
-                        // the block stops at its next barrier
+                for (int c = 0; c < nch; ++c) {
+                    const uint32_t g = G0 + c;
+                    if (!mbar_wait(a_full(g), (g >> 1) & 1u, a.spin) || !mbar_wait(full_b(g), phase(g), a.spin)) {
                         set_status(a.status, DPB_DEV_TIMEOUT);
                         tfail = true;
-                    } else {
-                        consumed = g + 1;
-                        asm volatile("tcgen05.fence::after_thread_sync;");
-                        const uint32_t bb = smem_u32(stage_b(g));
-                        for (int tt = 0; tt < ntiles; ++tt) {
-                            const uint32_t ab = smem_u32(As + tt * kATile);
+                        break;
+                    }
+                    consumed = g + 1;
+                    asm volatile("tcgen05.fence::after_thread_sync;");
+                    const uint32_t bb = smem_u32(stage_b(g));
+                    const uint8_t *As = sA + (g & 1u) * 2 * kATile;
+                    for (int tt = 0; tt < ntiles; ++tt) {
+                        const uint32_t ab = smem_u32(As + tt * kATile);
 #pragma unroll
-                            for (int k = 0; k < kChunk / 16; ++k) {
-                                const uint32_t acc = (c > 0 || k > 0) ? 1u : 0u;
-                                asm volatile(
-                                    "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-                                    "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem + 256 * tt),
-                                    "l"(tile_desc(ab + 256 * k)), "l"(tile_desc(bb + 256 * k)), "r"(idesc), "r"(acc));
-                            }
+                        for (int k = 0; k < kChunk / 16; ++k) {
+                            const uint32_t acc = (c > 0 || k > 0) ? 1u : 0u;
+                            asm volatile(
+                                "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+                                "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem + 256 * tt),
+                                "l"(tile_desc(ab + 256 * k)), "l"(tile_desc(bb + 256 * k)), "r"(idesc), "r"(acc));
                         }
                     }
                     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
                         mma_done(g)));
-                    if (nbs >= 3) {
-                        // the tile nbs - 2 chunks ahead goes to the stage chunk g - 2
-                        // read; its MMAs were waited for at the top of this chunk,
-                        // so thread 0 goes on to the next chunk without waiting
-                        if (!tfail && c >= 2 && c + nbs - 2 < nch)
-                            issue_b(g + nbs - 2, gt + (int64_t)(c + nbs - 2) * D * 32, D);
-                    } else if (c + 1 < nch) {
-                        // two stages: the next tile goes to the stage chunk g - 1
-                        // read, once its MMAs are done
-                        const bool ok = !tfail && (c == 0 || mbar_wait(mma_done(g - 1), phase(g - 1), a.spin));
-                        if (ok) {
-                            issue_b(g + 1, gt + (int64_t)(c + 1) * D * 32, D);
-                        } else {
+                    Gc = g + 1;
+                    // the tile nbs - 2 chunks ahead (nbs >= 3) or the next one (two
+                    // stages), past the first `ahead`, goes to the stage that chunk
+                    // next - nbs read, once that chunk's MMAs are done (a chunk of
+                    // an earlier level is done already)
+                    const int next = c + (nbs >= 3 ? nbs - 2 : 1);
+                    if (next >= ahead && next < nch) {
+                        const uint32_t prev = G0 + (uint32_t)next - (uint32_t)nbs;
+                        if (next >= nbs && !mbar_wait(mma_done(prev), phase(prev), a.spin)) {
                             set_status(a.status, DPB_DEV_TIMEOUT);
                             tfail = true;
+                            break;
                         }
+                        issue_b(G0 + next, gt + (int64_t)next * D * 32, D);
                     }
                 }
-                G = g + 1;
+            } else if (tid < kIssuer) {
+                // ---- the token warps build A: chunk g's stage is free once the
+                // MMAs of chunk g - 2 are done
+                for (int c = 0; c < nch; ++c) {
+                    const uint32_t g = G0 + c;
+                    if (c >= 2 && !mbar_wait(mma_done(g - 2), phase(g - 2), a.spin)) {
+                        bfail = true;
+                        break;
+                    }
+                    uint8_t *As = sA + (g & 1u) * 2 * kATile;
+#pragma unroll
+                    for (int tt = 0; tt < 2; ++tt) {
+                        if (tt < ntiles) {
+                            const int m = 2 * c + hb;
+                            const bool rv = irv[tt];
+                            uint32_t sw = iw5[tt] ^ (0u - (uint32_t)(__popc((uint32_t)m & iu[tt]) & 1));
+#pragma unroll
+                            for (int k = 0; k < 4; ++k)
+                                if (k < a.kvh) sw ^= vh[(k * nblk + m) * 32 + ihv[tt][k]];
+                            const uint4 *xs = reinterpret_cast<const uint4 *>(ixt[tt] + m * 16);
+                            uint8_t *At = As + tt * kATile;
+#pragma unroll
+                            for (int q = 0; q < 4; ++q) {
+                                const uint4 xv = xs[q];
+                                const int sh = 15 - 4 * q;
+                                uint4 av;
+                                av.x = rv ? xv.x ^ ((sw << sh) & 0x80008000u) : 0u;
+                                av.y = rv ? xv.y ^ ((sw << (sh - 1)) & 0x80008000u) : 0u;
+                                av.z = rv ? xv.z ^ ((sw << (sh - 2)) & 0x80008000u) : 0u;
+                                av.w = rv ? xv.w ^ ((sw << (sh - 3)) & 0x80008000u) : 0u;
+                                *reinterpret_cast<uint4 *>(At + (rr >> 3) * 1024 + (4 * hb + q) * 128 + (rr & 7) * 16) =
+                                    av;
+                            }
+                        }
+                    }
+                    // this thread's stores, then the warp's, are seen by the tensor
+                    // cores once the issuer has seen the warp's arrival
+                    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                    __syncwarp();
+                    if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(a_full(g)) : "memory");
+                }
             }
-            if (failed) break;
             {
                 // the last commit covers every MMA of the level
-                const bool ok = mbar_wait(mma_done(G - 1), phase(G - 1), a.spin);
-                if (__syncthreads_or(!ok || tfail)) {
+                const uint32_t gl1 = G0 + nch - 1;
+                const bool ok = !bfail && !tfail && mbar_wait(mma_done(gl1), phase(gl1), a.spin);
+                if (__syncthreads_or(!ok)) {
                     failed = true;
                     break;
                 }
             }
+            G = G0 + nch;
             asm volatile("tcgen05.fence::after_thread_sync;");
             const uint32_t *gl = gs + l * 256;
             // ---- standardised scores, once per candidate (§2.2): z replaces s in
@@ -613,7 +626,7 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
             // tokens q and q + 4) of tile w / 4, or with one tile half w / 4 of
             // the columns: all eight warps keep table loads in flight.
             if (a.mu) {
-                {
+                if (warp < kTokens) {
                     const int q = warp & 3, tile = ntiles == 2 ? warp >> 2 : 0;
                     const int half = ((D + 31) / 32 + 1) / 2 * 32;  // whole 32-column loads
                     const int cb = ntiles == 2 ? 0 : (warp >> 2) * half, ce = ntiles == 2 ? D : min(D, cb + half);
@@ -668,9 +681,9 @@ __global__ void __launch_bounds__(kTokens * 32, 1) encode_pl_kernel(Args a) {
     // drain (bounded, with the default bound): every generator-tile copy still
     // in flight lands, and the last commit (which covers every MMA issued)
     // arrives, before the block frees its TMEM and its shared memory
-    if (failed && tid == 0) {
+    if (failed && tid == kIssuer) {
         for (uint32_t g = consumed; g < issued; ++g) mbar_wait(full_b(g), phase(g), kSpin);
-        if (G > 0) mbar_wait(mma_done(G - 1), phase(G - 1), kSpin);
+        if (Gc > 0) mbar_wait(mma_done(Gc - 1), phase(Gc - 1), kSpin);
     }
     asm volatile("tcgen05.fence::before_thread_sync;");
     __syncthreads();
@@ -802,7 +815,7 @@ cudaError_t launch_encode_pl(const dpb_plan *p, const void *x, int64_t T, const 
     if (e != cudaSuccess) return e;
     const int64_t groups = (T + kTokens - 1) / kTokens;
     const int grid = (int)std::min<int64_t>(groups, (int64_t)std::max(p->sms, 1));
-    encode_pl_kernel<<<grid, kTokens * 32, smem, stream>>>(a);
+    encode_pl_kernel<<<grid, kThreads, smem, stream>>>(a);
     return cudaGetLastError();
 }
 
