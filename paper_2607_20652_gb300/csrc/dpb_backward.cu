@@ -155,16 +155,17 @@ __global__ void __launch_bounds__(128) backward_warp_kernel(BackwardArgs a) {
 constexpr int kChunkBlocks = 4;                       // 32-coordinate blocks per analysis chunk
 constexpr int kTabStride = 17;                        // 16 entries + 1 pad (bank spread)
 constexpr int kChunkTables = kChunkBlocks * 8 * kTabStride;  // nibble tables of a chunk (words)
-constexpr int kScratchWords = pad64(kSweepWords > kChunkTables ? kSweepWords : kChunkTables);
-constexpr int kBwdWarps = 14;  // at most; two blocks of 14 fill an SM's shared memory at d = 768
-constexpr size_t kSmemPerSm = 228 * 1024;
+__host__ __device__ constexpr int bwd_scratch_words(int qn, int nkc) {
+    return pad64(sweep_words(qn, nkc) > kChunkTables ? sweep_words(qn, nkc) : kChunkTables);
+}
+constexpr int kBwdWarps = 15;  // at most per block; two blocks of 15 per SM at d = 768
 static_assert(kChunkBlocks == 4, "the analysis gives a code 4 lanes, one per block of a chunk");
 
 // Per-warp words: the scratch (a sweep's tables, or a chunk's nibble tables;
 // first, so that it keeps the region's 256-byte alignment), then r / dL/dr /
 // grad_x (d) and the code's lists (list, map, sums, offsets).
-__host__ __device__ constexpr int bwd_warp_words(int d, int k) {
-    return pad64(kScratchWords + pad4(d) + 6 * pad4(k));
+__host__ __device__ constexpr int bwd_warp_words(int d, int k, int nkc) {
+    return pad64(bwd_scratch_words((d + 31) / 32, nkc) + pad4(d) + 6 * pad4(k));
 }
 
 __host__ __device__ constexpr int bwd_block_words(int d, int nkc) {
@@ -318,10 +319,10 @@ __global__ void __launch_bounds__(kBwdWarps * 32, 2) backward_lut_kernel(Backwar
     for (int i = threadIdx.x; i < NKC * ((d + 31) / 32) * 32; i += blockDim.x) vh2[i] = a.VH[i];
     load_koff(a.M, d, t, koff);  // ends with __syncthreads()
 
-    uint32_t *base = smem + bwd_block_words(d, NKC) + (size_t)warp * bwd_warp_words(d, k);
+    uint32_t *base = smem + bwd_block_words(d, NKC) + (size_t)warp * bwd_warp_words(d, k, NKC);
     BwdWarp w;
     w.scratch = base;
-    w.buf = reinterpret_cast<float *>(base + kScratchWords);
+    w.buf = reinterpret_cast<float *>(base + bwd_scratch_words((d + 31) / 32, NKC));
     w.hc = reinterpret_cast<uint32_t *>(w.buf + dp);
     w.ha = reinterpret_cast<float *>(w.hc + kp);
     w.cmap = reinterpret_cast<int *>(w.ha + kp);
@@ -329,7 +330,7 @@ __global__ void __launch_bounds__(kBwdWarps * 32, 2) backward_lut_kernel(Backwar
     w.o1 = reinterpret_cast<uint32_t *>(w.gv + kp);
     w.o2 = w.o1 + kp;
     float *bterm = reinterpret_cast<float *>(w.o2);  // basis grad_x terms, after the analysis
-    Sweep sw = sweep_at(w.scratch);
+    Sweep sw = sweep_at(w.scratch, (d + 31) / 32, NKC);
 
     const Tio *X = static_cast<const Tio *>(a.x);
     const Tio *GY = static_cast<const Tio *>(a.gy);
@@ -481,24 +482,12 @@ int grid_for(const dpb_plan *p, int64_t T, int warps) {
 
 template <typename Tio, int NKC, bool VEC>
 cudaError_t run_backward_lut(const dpb_plan *p, const BackwardArgs &a, int64_t T, cudaStream_t stream) {
-    // The warps per block that put the most warps on an SM: shared memory
-    // (228 KB per SM, 1 KB of it reserved per block) and the 2 x kBwdWarps
-    // warps that the registers allow (kBwdWarps = 14: two blocks at d = 768,
-    // k = 64; two of 10 at d = 1024, k = 112)
-    auto smem_for = [&](int w) {
-        return 256 /* alignment */ + sizeof(uint32_t) * ((size_t)bwd_block_words(p->cfg.d, NKC) +
-                                                         (size_t)w * bwd_warp_words(p->cfg.d, p->code_len));
-    };
-    int warps = 1, best = 0;
-    for (int w = kBwdWarps; w >= 1; --w) {
-        if (smem_for(w) > kMaxSmemPerBlock) continue;
-        const int blocks = std::min((int)(kSmemPerSm / (smem_for(w) + 1024)), 2 * kBwdWarps / w);
-        if (blocks * w > best) {
-            best = blocks * w;
-            warps = w;
-        }
-    }
-    const size_t smem = smem_for(warps);
+    const size_t per_block = 256 /* alignment */ + sizeof(uint32_t) * (size_t)bwd_block_words(p->cfg.d, NKC);
+    const size_t per_warp = sizeof(uint32_t) * (size_t)bwd_warp_words(p->cfg.d, p->code_len, NKC);
+    const void *fn = (const void *)backward_lut_kernel<Tio, NKC, VEC>;
+    const int warps = best_warps(fn, kBwdWarps, per_block, per_warp);
+    if (warps <= 0) return cudaErrorInvalidConfiguration;
+    const size_t smem = per_block + (size_t)warps * per_warp;
     const cudaError_t e = allow_smem((const void *)backward_lut_kernel<Tio, NKC, VEC>, smem);
     if (e != cudaSuccess) return e;
     backward_lut_kernel<Tio, NKC, VEC><<<grid_for(p, T, warps), warps * 32, smem, stream>>>(a, p->t);

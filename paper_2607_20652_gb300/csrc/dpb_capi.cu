@@ -6,6 +6,7 @@
 #include <map>
 #include <mutex>
 #include <new>
+#include <tuple>
 #include <utility>
 
 #include "dpb_internal.h"
@@ -26,6 +27,36 @@ cudaError_t allow_smem(const void *func, size_t bytes) {
     e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
     if (e == cudaSuccess) have = bytes;
     return e;
+}
+
+int best_warps(const void *func, int max_warps, size_t per_block, size_t per_warp) {
+    static std::mutex mu;
+    static std::map<std::tuple<const void *, int, size_t, size_t>, int> chosen;
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+    const auto key = std::make_tuple(func, dev, per_block, per_warp);
+    {
+        std::lock_guard<std::mutex> lock(mu);
+        const auto it = chosen.find(key);
+        if (it != chosen.end()) return it->second;
+    }
+    int best = 0, best_resident = 0;
+    for (int w = max_warps; w >= 1; --w) {
+        const size_t smem = per_block + (size_t)w * per_warp;
+        if (smem > kMaxSmemPerBlock || allow_smem(func, smem) != cudaSuccess) continue;
+        int blocks = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&blocks, func, 32 * w, smem) != cudaSuccess) {
+            cudaGetLastError();
+            continue;
+        }
+        if (blocks * w > best_resident) {
+            best_resident = blocks * w;
+            best = w;
+        }
+    }
+    std::lock_guard<std::mutex> lock(mu);
+    chosen[key] = best;
+    return best;
 }
 }  // namespace dpb
 

@@ -92,12 +92,14 @@ __global__ void __launch_bounds__(128) decode_warp_kernel(DecodeArgs a) {
 // Per-warp shared memory of the decoder, in 4-byte words: one sweep's tables
 // (first, so that they keep the region's 128-byte alignment), r (d) and the
 // hashed list (indices, coefficients).
-__host__ __device__ constexpr int decode_warp_words(int d, int k) {
-    return pad32(kSweepWords + pad4(d) + 2 * pad4(k));
+__host__ __device__ constexpr int decode_warp_words(int d, int k, int nkc) {
+    return pad32(sweep_words((d + 31) / 32, nkc) + pad4(d) + 2 * pad4(k));
 }
 
+constexpr int kDecWarps = 9;  // at most per block; four such blocks per SM at 56 registers
+
 template <typename Tio, int NKC, bool VEC>
-__global__ void __launch_bounds__(256) decode_lut_kernel(DecodeArgs a, int t) {
+__global__ void __launch_bounds__(kDecWarps * 32, 4) decode_lut_kernel(DecodeArgs a, int t) {
     extern __shared__ __align__(16) uint32_t smem_raw[];
     uint32_t *smem = aligned_smem<128>(smem_raw);
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
@@ -105,10 +107,11 @@ __global__ void __launch_bounds__(256) decode_lut_kernel(DecodeArgs a, int t) {
     uint32_t *koff = smem;
     load_koff(a.M, d, t, koff);
     const int dp = pad4(d), kp = pad4(a.k);
-    uint32_t *base = smem + pad32(d) + (size_t)warp * decode_warp_words(d, a.k);
-    Sweep sw = sweep_at(base);
-    float *r = reinterpret_cast<float *>(base + kSweepWords);
-    HashedList hl{base + kSweepWords + dp, reinterpret_cast<float *>(base + kSweepWords + dp + kp), nullptr};
+    const int sww = sweep_words((d + 31) / 32, NKC);
+    uint32_t *base = smem + pad32(d) + (size_t)warp * decode_warp_words(d, a.k, NKC);
+    Sweep sw = sweep_at(base, (d + 31) / 32, NKC);
+    float *r = reinterpret_cast<float *>(base + sww);
+    HashedList hl{base + sww + dp, reinterpret_cast<float *>(base + sww + dp + kp), nullptr};
     Tio *Y = static_cast<Tio *>(a.y);
     for (int64_t tk = (int64_t)blockIdx.x * nwarps + warp; tk < a.T; tk += (int64_t)gridDim.x * nwarps) {
         RowOps<VEC>::fill(r, d, 0.f);
@@ -138,10 +141,13 @@ namespace {
 
 template <typename Tio, int NKC, bool VEC>
 cudaError_t run_decode_lut(const dpb_plan *p, const DecodeArgs &a, int64_t T, cudaStream_t stream) {
-    const int warps = 8;
-    const size_t smem = 128 /* alignment */ +
-                        sizeof(uint32_t) * ((size_t)pad32(p->cfg.d) + (size_t)warps * decode_warp_words(p->cfg.d, p->code_len));
-    const cudaError_t e = allow_smem((const void *)decode_lut_kernel<Tio, NKC, VEC>, smem);
+    const size_t per_block = 128 /* alignment */ + sizeof(uint32_t) * (size_t)pad32(p->cfg.d);
+    const size_t per_warp = sizeof(uint32_t) * (size_t)decode_warp_words(p->cfg.d, p->code_len, NKC);
+    const void *fn = (const void *)decode_lut_kernel<Tio, NKC, VEC>;
+    const int warps = best_warps(fn, kDecWarps, per_block, per_warp);
+    if (warps <= 0) return cudaErrorInvalidConfiguration;
+    const size_t smem = per_block + (size_t)warps * per_warp;
+    const cudaError_t e = allow_smem(fn, smem);
     if (e != cudaSuccess) return e;
     decode_lut_kernel<Tio, NKC, VEC><<<grid_for(p, T, warps), warps * 32, smem, stream>>>(a, p->t);
     return cudaGetLastError();

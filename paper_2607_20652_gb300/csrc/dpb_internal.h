@@ -97,6 +97,13 @@ constexpr size_t kMaxSmemPerBlock = 227 * 1024;
 // launches make no driver call; returns the error of a failed set.
 cudaError_t allow_smem(const void *func, size_t bytes);
 
+// The warps per block (1..max_warps) that put the most warps of kernel
+// `func` on an SM of the current device, by the occupancy calculator, when a
+// block of w warps takes per_block + w per_warp bytes of dynamic shared
+// memory (ties go to more warps per block); 0 if none fits. Cached per
+// (kernel, device, sizes).
+int best_warps(const void *func, int max_warps, size_t per_block, size_t per_warp);
+
 // Records a message for dpb_last_error() and returns `s`.
 dpb_status fail(dpb_status s, const char *fmt, ...);
 

@@ -32,21 +32,26 @@ constexpr int kMaxKChunks = 4;   // ceil(16 / 5) chunks of inv(iota) for t <= 16
 constexpr int kMaxRuns = 13;     // ceil(64 / 5) runs of 5 codes per sweep
 constexpr int kShflRuns = 7;     // even runs 0, 2, ..., 12
 
-// Shared-memory words of one sweep's tables.
 constexpr int kMaxBlocks = 64;   // 32-coordinate blocks of d <= 2048
-constexpr int kSweepWords = 2 * kMaxBlocks /* ZQ (uint2 per block) */ +
-                            2 * 32 * kMaxKChunks /* ZH (uint2 entries) */ +
-                            32 * kShflRuns /* odd runs' value tables */ + 64 /* coefficients */;
+
+// Shared-memory words of one sweep's tables for qn 32-coordinate blocks and
+// nkc chunk tables of inv(iota): ZQ (a uint2 per block, padded to 128
+// bytes), ZH (nkc tables of 2 x 32 words), the odd runs' value tables (6 x 32
+// words, 128-byte aligned) and the coefficients (64). A multiple of 32 words.
+__host__ __device__ constexpr int sweep_words(int qn, int nkc) {
+    return ((2 * qn + 31) & ~31) + 64 * nkc + 32 * (kMaxRuns - kShflRuns) + 64;
+}
 
 struct Sweep {
     uint2 zl;                 // ZL(lane) for codes 0..31 (x) and 32..63 (y)
     float vt[kShflRuns];      // lane v holds the table of run 2i at v
-    uint2 *zq;                // [kMaxBlocks] (shared)
-    uint32_t *zh;             // [kMaxKChunks][2][32]: codes 0..31, then 32..63 (shared)
+    uint2 *zq;                // [qn] (shared)
+    uint32_t *zh;             // [nkc][2][32]: codes 0..31, then 32..63 (shared)
     float *vto;               // [6][32] odd runs (shared)
     float *coef;              // [64] (shared)
     uint32_t vto_s;           // shared-window address of vto (128-byte aligned)
     int runs;                 // ceil(codes / 5)
+    int nkc;                  // chunk tables of inv(iota) held
 };
 
 // Shared-window (32-bit) address of a pointer into this block's shared memory.
@@ -73,15 +78,16 @@ __device__ __forceinline__ uint32_t *aligned_smem(uint32_t *raw) {
     return raw + ((A - (smem_u32(raw) & (A - 1))) & (A - 1)) / 4;
 }
 
-// A sweep's tables at base, which must be 128-byte aligned (the odd value
-// tables are addressed by OR).
-__device__ __forceinline__ Sweep sweep_at(uint32_t *base) {
+// A sweep's tables at base (sweep_words(qn, nkc) words), which must be
+// 128-byte aligned (the odd value tables are addressed by OR).
+__device__ __forceinline__ Sweep sweep_at(uint32_t *base, int qn, int nkc) {
     Sweep s;
     s.zq = reinterpret_cast<uint2 *>(base);
-    s.zh = reinterpret_cast<uint32_t *>(s.zq + kMaxBlocks);
-    s.vto = reinterpret_cast<float *>(s.zh + 64 * kMaxKChunks);
+    s.zh = base + ((2 * qn + 31) & ~31);
+    s.vto = reinterpret_cast<float *>(s.zh + 64 * nkc);
     s.coef = s.vto + 32 * (kMaxRuns - kShflRuns);
     s.vto_s = smem_u32(s.vto);
+    s.nkc = nkc;
     return s;
 }
 
@@ -126,6 +132,7 @@ __device__ __forceinline__ void sweep_build_signs(uint32_t ca, uint32_t cb, int 
     }
 #pragma unroll
     for (int k = 0; k < kMaxKChunks; ++k) {
+        if (k >= s.nkc) break;  // chunks past the held ones are zero (t <= 5 nkc)
         uint2 acc = make_uint2(0u, 0u);
 #pragma unroll
         for (int bb = 0; bb < 5; ++bb) {
@@ -256,7 +263,8 @@ __host__ __device__ constexpr int pad4(int v) { return (v + 3) & ~3; }
 // Sizes rounded up to 32 words (128 bytes) and 64 words (256 bytes).
 __host__ __device__ constexpr int pad32(int v) { return (v + 31) & ~31; }
 __host__ __device__ constexpr int pad64(int v) { return (v + 63) & ~63; }
-static_assert(kSweepWords % 32 == 0, "a sweep's tables keep the 128-byte alignment of what follows");
+static_assert(sweep_words(24, 2) % 32 == 0 && sweep_words(64, 4) % 32 == 0,
+              "a sweep's tables keep the 128-byte alignment of what follows");
 
 // ---- a token's code -----------------------------------------------------------
 
