@@ -531,7 +531,9 @@ cudaError_t launch_backward(const dpb_plan *p, const void *x, const int32_t *idx
         return c.dtype == DPB_BF16 ? dispatch_backward_lut<__nv_bfloat16>(p, a, T, stream)
                                    : dispatch_backward_lut<float>(p, a, T, stream);
     }
-    const int warps = 4;
+    // 4 warps, fewer when the four d-length buffers per warp would not fit (d = 4096: 3)
+    int warps = 4;
+    while (warps > 1 && sizeof(uint32_t) * ((size_t)c.d + (size_t)warps * 4 * c.d) > kMaxSmemPerBlock) --warps;
     const size_t smem = sizeof(uint32_t) * ((size_t)c.d + (size_t)warps * 4 * c.d);
     const int grid = grid_for(p, T, warps);
     if (c.dtype == DPB_BF16) {

@@ -25,7 +25,10 @@ cudaError_t allow_smem(const void *func, size_t bytes) {
     size_t &have = granted[{func, dev}];
     if (have >= bytes) return cudaSuccess;
     e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
-    if (e == cudaSuccess) have = bytes;
+    if (e == cudaSuccess)
+        have = bytes;
+    else
+        cudaGetLastError();  // returned to the caller: not left for its next CUDA check
     return e;
 }
 
@@ -88,8 +91,14 @@ dpb_status check_vec(const void *ptr, const char *name, bool required) {
     return DPB_OK;
 }
 
+// A failed launch is reported through the returned status; the runtime's
+// last-error slot is cleared so that the caller's next CUDA check (PyTorch's,
+// for instance) does not see it again.
 dpb_status launched(cudaError_t e, const char *what) {
-    if (e != cudaSuccess) return dpb::fail(DPB_ERR_CUDA, "%s launch failed: %s", what, cudaGetErrorString(e));
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return dpb::fail(DPB_ERR_CUDA, "%s launch failed: %s", what, cudaGetErrorString(e));
+    }
     return DPB_OK;
 }
 
@@ -153,11 +162,13 @@ dpb_status dpb_plan_create(const dpb_config *cfg, const uint32_t *generators, dp
         if (u.src->empty()) continue;
         const size_t bytes = sizeof(uint32_t) * u.src->size();
         if (cudaMalloc(u.dst, bytes) != cudaSuccess) {
+            cudaGetLastError();
             for (const Up &v : ups) cudaFree(*v.dst);
             delete p;
             return dpb::fail(DPB_ERR_NO_MEMORY, "device table allocation failed");
         }
         if (cudaMemcpy(*u.dst, u.src->data(), bytes, cudaMemcpyHostToDevice) != cudaSuccess) {
+            cudaGetLastError();
             for (const Up &v : ups) cudaFree(*v.dst);
             delete p;
             return dpb::fail(DPB_ERR_CUDA, "device table upload failed");

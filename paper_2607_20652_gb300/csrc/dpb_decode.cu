@@ -181,7 +181,8 @@ cudaError_t launch_decode(const dpb_plan *p, const int32_t *idx, const float *va
         return c.dtype == DPB_BF16 ? dispatch_decode_lut<__nv_bfloat16>(p, a, T, stream)
                                    : dispatch_decode_lut<float>(p, a, T, stream);
     }
-    const int warps = 4;
+    int warps = 4;  // fewer when the two d-length buffers per warp would not fit
+    while (warps > 1 && sizeof(uint32_t) * ((size_t)c.d + (size_t)warps * 2 * c.d) > kMaxSmemPerBlock) --warps;
     const size_t smem = sizeof(uint32_t) * ((size_t)c.d + (size_t)warps * 2 * c.d);
     const int grid = grid_for(p, T, warps);
     if (c.dtype == DPB_BF16) {

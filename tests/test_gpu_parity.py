@@ -294,6 +294,26 @@ def test_limits_config():
     _check_all(plan, ref, x, g, gy=gy)
 
 
+@pytest.mark.parametrize("kw", [
+    # d = 4096 with 2^31 features (t = 16: four chunks of the inverse half), beam 32,
+    # 256 children, k = 256: the warp-per-token encoder, the plain decode/backward loops
+    dict(d=4096, levels=3, m_bits=31, children=256, beam=32, k=256, dtype="f32"),
+    # eight levels up to 2^31, beam 16 (the tensor-core encoder's two halves of 8
+    # slots), k = 256 (8 list words per lane)
+    dict(d=1024, levels=8, m_bits=31, children=16, beam=16, k=256, dtype="bf16"),
+], ids=["d4096-2^31-b32-c256-k256", "L8-2^31-b16-k256"])
+def test_maximum_sizes(kw):
+    plan = dpb.Plan(**kw)
+    ref = _ref(plan)
+    T = 6
+    x = inputs.gaussian_rows(T, kw["d"], 61)
+    gy = inputs.normal((T, kw["d"]), 62)
+    if kw["dtype"] == "bf16":
+        x, gy = inputs.to_bf16(x), inputs.to_bf16(gy)
+    g = _gpu(plan, x, gy_np=gy)
+    _check_all(plan, ref, x, g, gy=gy)
+
+
 def test_bad_index_is_flagged_not_faulted():
     plan = dpb.Plan(d=64, levels=3, m_bits=12, children=16, beam=4, k=4, dtype="f32", norm_match=0)
     idx = torch.tensor([[1, 70, 5000, -3], [2, 3, 4, 4095]], dtype=torch.int32, device="cuda")
