@@ -314,6 +314,44 @@ def test_maximum_sizes(kw):
     _check_all(plan, ref, x, g, gy=gy)
 
 
+def test_batch_past_two_gigabytes_of_rows():
+    # T = 2^20 + 37 tokens at d = 768 bf16: the rows span 1.6 GB, so element and
+    # byte offsets pass 2^31. The rows are 4096 seeded rows tiled on the GPU:
+    # every copy of a row must give bit-identical outputs (a property at any
+    # size), and sampled rows match the oracle.
+    w = configs.WORKLOADS["wide"]
+    plan = _plan(w)
+    ref = _ref(plan)
+    n, T, d = 4096, (1 << 20) + 37, w["d"]
+    xs = inputs.to_bf16(inputs.gaussian_rows(n, d, 123))
+    gys = inputs.to_bf16(inputs.normal((n, d), 124))
+    dev = torch.device("cuda")
+    reps = (T + n - 1) // n
+    x = torch.from_numpy(xs).to(dev).to(torch.bfloat16).repeat(reps, 1)[:T].contiguous()
+    gy = torch.from_numpy(gys).to(dev).to(torch.bfloat16).repeat(reps, 1)[:T].contiguous()
+    ws = plan.workspace(T, dev)
+    idx, val, xn = dpb.encode(plan, x, workspace=ws)
+    del x
+    y = dpb.decode(plan, idx, val, xn, workspace=ws)
+    xb = torch.from_numpy(xs).to(dev).to(torch.bfloat16).repeat(reps, 1)[:T].contiguous()
+    gx, gv = dpb.backward(plan, xb, idx, val, gy, workspace=ws)
+    torch.cuda.synchronize()
+    assert dpb.workspace_status(ws) == 0
+    late = np.array([T - 1, T - 2, T - 37, (1 << 20) - 1, 3 * (1 << 18) + 5, (1 << 19) + 11])
+    for name, t_ in (("idx", idx), ("val", val), ("y", y), ("gx", gx), ("gv", gv)):
+        a = t_[torch.from_numpy(late).to(dev)].cpu()
+        b = t_[torch.from_numpy(late % n).to(dev)].cpu()
+        assert torch.equal(a, b), f"{name}: a late copy of a row differs from its first copy"
+    rows = np.unique(np.concatenate([late % n, inputs.sample_rows(n, 10, 125)]))
+    g = {"idx": idx[torch.from_numpy(rows).to(dev)].cpu().numpy(),
+         "val": val[torch.from_numpy(rows).to(dev)].cpu().numpy(),
+         "xnorm": xn[torch.from_numpy(rows).to(dev)].cpu().numpy(),
+         "y": y[torch.from_numpy(rows).to(dev)].float().cpu().numpy(),
+         "gx": gx[torch.from_numpy(rows).to(dev)].float().cpu().numpy(),
+         "gv": gv[torch.from_numpy(rows).to(dev)].cpu().numpy(), "status": 0}
+    _check_all(plan, ref, xs[rows], g, gy=gys[rows])
+
+
 def test_bad_index_is_flagged_not_faulted():
     plan = dpb.Plan(d=64, levels=3, m_bits=12, children=16, beam=4, k=4, dtype="f32", norm_match=0)
     idx = torch.tensor([[1, 70, 5000, -3], [2, 3, 4, 4095]], dtype=torch.int32, device="cuda")
