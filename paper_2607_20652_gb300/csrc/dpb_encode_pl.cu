@@ -33,12 +33,11 @@
 // Selection of a level (one warp per token, lane = parent slot): each lane
 // keeps the 4 largest of its row's group maxima (the largest key |z| of each
 // 8 consecutive children; every key at level 0), the warp sorts the union and
-// takes a threshold tau at rank K + K/2 of its distinct keys. Each of those
-// keys is a candidate's, so at least K + K/2 distinct candidates reach tau.
-// Every candidate at or above tau is gathered (one pass with running ballot
-// positions), sorted, and its repeated indices (two parents can share a
-// child) are dropped. When K distinct candidates reach tau they are exactly
-// the level's top K.
+// takes a threshold tau at rank K of its distinct keys. Each of those keys is
+// a candidate's, so at least K distinct candidates reach tau, and with them
+// the level's top K. Every candidate at or above tau is gathered (one pass
+// with running ballot positions), sorted, and its repeated indices (two
+// parents can share a child) are dropped; the first K remain.
 #include <algorithm>
 #include <atomic>
 
@@ -263,14 +262,16 @@ __device__ __forceinline__ int sort_keep(int n, int K, const WarpBufs &w, const 
 }
 
 // The top K distinct candidates of one token, as explained in the header.
-// `scan(f)` calls f(z, index, live, gend) for every candidate of this lane, in
-// the same order each time and in step across the warp; gend marks the last
-// candidate of a group. Writes code columns
-// [col, col + K) of row `tok` and, when `par_out`, the kept indices as the
-// next level's parents. Returns the number of distinct candidates kept
-// (< K only with the status bit set).
+// `scan(f)` calls f(v, live, gend, index) for every candidate of this lane, in
+// the same order each time and in step across the warp: v is its score before
+// the factor `scale` (> 0; the score is z = v scale), gend marks the last
+// candidate of a group (a group is live or not as a whole), and index() gives
+// its feature index. Scaling is monotone, so a group's largest |z| is its
+// largest |v| scaled once. Writes code columns [col, col + K) of row `tok`
+// and, when `par_out`, the kept indices as the next level's parents. Returns
+// the number of distinct candidates kept (< K only with the status bit set).
 template <class Scan>
-__device__ __forceinline__ int select_level(Scan scan, int nlive, int K, const WarpBufs &w, const Args &a,
+__device__ __forceinline__ int select_level(Scan scan, float scale, int K, const WarpBufs &w, const Args &a,
                                             int64_t tok, int col, bool par_out) {
     const int lane = threadIdx.x & 31;
     uint32_t top[4];
@@ -283,12 +284,12 @@ __device__ __forceinline__ int select_level(Scan scan, int nlive, int K, const W
         const bool group = pass == 0;
 #pragma unroll
         for (int r = 0; r < 4; ++r) top[r] = 0u;
-        uint32_t gm = 0u;  // the largest key of the current group
-        scan([&](float z, uint32_t, bool live, bool gend) {
-            gm = max(gm, live ? akey(z) + 1u : 0u);
+        float gm = -1.f;  // the largest |v| of the current group (-1: none live)
+        scan([&](float v, bool live, bool gend, auto) {
+            if (live) gm = fmaxf(gm, fabsf(v));
             if (gend || !group) {
-                uint32_t c = gm;
-                gm = 0u;
+                uint32_t c = gm >= 0.f ? akey(gm * scale) + 1u : 0u;
+                gm = -1.f;
 #pragma unroll
                 for (int r = 0; r < 4; ++r) {
                     const uint32_t hi = max(top[r], c);
@@ -297,7 +298,7 @@ __device__ __forceinline__ int select_level(Scan scan, int nlive, int K, const W
                 }
             }
         });
-        mmaenc::warp_sort_desc<4>(top);
+        mmaenc::warp_sort_desc_runs<4>(top);  // each lane's 4 are in order already
         // distinct keys of the sorted union (copies of one child share a key):
         // drank[r] = rank among them, 0 for a repeat or an empty slot
         {
@@ -329,46 +330,41 @@ __device__ __forceinline__ int select_level(Scan scan, int nlive, int K, const W
         nd = (int)__reduce_max_sync(kFull, (uint32_t)nd);
         if (nd >= K) break;
     }
-    (void)nlive;
-    int distinct = 0;
-    // tau = the union's distinct key of rank K + K/2 (so that at least that many
-    // distinct candidates reach it), rank K when too many candidates do
-    int target = min(K + K / 2, nd);
-    for (int attempt = 0; attempt < 2; ++attempt) {
-        uint32_t mine = 0u;
+    // tau = the union's distinct key of rank K: every key of the union is some
+    // candidate's, so K distinct candidates reach it and the level's top K
+    // distinct all do (the union's last distinct key when it holds fewer)
+    const int target = min(K, nd);
+    uint32_t mine = 0u;
 #pragma unroll
-        for (int r = 0; r < 4; ++r)
-            if (drank[r] == target) mine = top[r];
-        uint32_t tau = __reduce_max_sync(kFull, mine);
-        if (tau == 0u) tau = 1u;
-        // gather every candidate at or above tau, warp-interleaved in scan
-        // order (one pass: positions come from the running ballot counts)
-        int n = 0;
-        scan([&](float z, uint32_t ci, bool live, bool) {
-            const bool take = live && akey(z) + 1u >= tau;
-            const unsigned mb = __ballot_sync(kFull, take);
-            if (mb) {  // rare: most candidates fall short of tau
-                const int pos = n + __popc(mb & ((1u << lane) - 1u));
-                if (take && pos < kSelCap) {
-                    w.z[pos] = z;
-                    w.id[pos] = ci;
-                }
-                n += __popc(mb);
+    for (int r = 0; r < 4; ++r)
+        if (drank[r] == target) mine = top[r];
+    uint32_t tau = __reduce_max_sync(kFull, mine);
+    if (tau == 0u) tau = 1u;
+    // key(z) + 1 >= tau exactly when |z| >= the float with bits tau - 1
+    const float tf = __uint_as_float(tau - 1u);
+    // gather every candidate at or above tau, warp-interleaved in scan order
+    // (one pass: positions come from the running ballot counts)
+    int n = 0;
+    scan([&](float v, bool live, bool, auto index) {
+        const float z = v * scale;
+        const bool take = live && fabsf(z) >= tf;
+        const unsigned mb = __ballot_sync(kFull, take);
+        if (mb) {  // rare: most candidates fall short of tau
+            const int pos = n + __popc(mb & ((1u << lane) - 1u));
+            if (take && pos < kSelCap) {
+                w.z[pos] = z;
+                w.id[pos] = index();
             }
-        });
-        if (n > kSelCap) {
-            if (attempt == 0 && target > K) {
-                target = min(K, nd);
-                continue;
-            }
-            set_status(a.status, DPB_DEV_SHORT_CODE);
-            n = kSelCap;
+            n += __popc(mb);
         }
-        __syncwarp();
-        distinct = n <= 128 ? sort_keep<4>(n, K, w, a, tok, col, par_out, true)
-                            : sort_keep<8>(n, K, w, a, tok, col, par_out, true);
-        break;
+    });
+    if (n > kSelCap) {
+        set_status(a.status, DPB_DEV_SHORT_CODE);
+        n = kSelCap;
     }
+    __syncwarp();
+    const int distinct = n <= 128 ? sort_keep<4>(n, K, w, a, tok, col, par_out, true)
+                                  : sort_keep<8>(n, K, w, a, tok, col, par_out, true);
     if (distinct < K) {
         set_status(a.status, DPB_DEV_SHORT_CODE);
         for (int e = distinct + lane; e < K; e += 32) {
@@ -478,12 +474,12 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
                 for (int i = lane; i < d; i += 32) {
                     const int m = i >> 5, wl = i & 31;
                     const float xv = __uint_as_float((uint32_t)xh[(m * 16 + (wl & 15)) * 2 + (wl >> 4)] << 16);
-                    f(standardise(xv, (uint32_t)i, a, nullptr), (uint32_t)i, true, true);
+                    f(standardise(xv, (uint32_t)i, a, nullptr), true, true, [&] { return (uint32_t)i; });
                 }
             };
             if (a.mu)
                 for (int i = lane; i < d; i += 32) standardise(0.f, (uint32_t)i, a, a.status);
-            select_level(scan0, min(32, d / 32 * 32), a.kl[0], wb, a, tok, a.off[0], L > 1);
+            select_level(scan0, 1.f, a.kl[0], wb, a, tok, a.off[0], L > 1);
         } else if (warp < kTokens) {
             wb.par[lane] = 0u;
             __syncwarp();
@@ -664,14 +660,14 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
                     for (int c0 = 0; c0 < D; c0 += 32) {
                         uint32_t v[32];
                         tmem_ld32(taddr + c0, v);
+                        // D is a multiple of 16: a group of 8 columns is live as a whole
 #pragma unroll
-                        for (int j = 0; j < 32; ++j) {
-                            const uint32_t ci = p ^ gl[c0 + j];
-                            f(__uint_as_float(v[j]) * scale, ci, rv && c0 + j < D, (j & 7) == 7);
-                        }
+                        for (int j = 0; j < 32; ++j)
+                            f(__uint_as_float(v[j]), rv && c0 + j < D, (j & 7) == 7,
+                              [&] { return p ^ gl[c0 + j]; });
                     }
                 };
-                select_level(scanl, P, a.kl[l], wb, a, tok, a.off[l], l + 1 < L);
+                select_level(scanl, scale, a.kl[l], wb, a, tok, a.off[l], l + 1 < L);
             }
             asm volatile("tcgen05.fence::before_thread_sync;");
             __syncthreads();
