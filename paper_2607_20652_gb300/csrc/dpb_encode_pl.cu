@@ -32,7 +32,8 @@
 //
 // Selection of a level (one warp per token, lane = parent slot): each lane
 // keeps the 4 largest of its row's group maxima (the largest key |z| of each
-// 8 consecutive children; every key at level 0), the warp sorts the union and
+// 8 consecutive children; at level 0, of each 8 of the lane's coordinates
+// lane + 32 j with consecutive j), the warp sorts the union and
 // takes a threshold tau at rank K of its distinct keys. Each of those keys is
 // a candidate's, so at least K distinct candidates reach tau, and with them
 // the level's top K. Every candidate at or above tau is gathered (one pass
@@ -363,8 +364,11 @@ __device__ __forceinline__ int select_level(Scan scan, float scale, int K, const
         n = kSelCap;
     }
     __syncwarp();
-    const int distinct = n <= 128 ? sort_keep<4>(n, K, w, a, tok, col, par_out, true)
-                                  : sort_keep<8>(n, K, w, a, tok, col, par_out, true);
+    // the narrowest sort that holds them: 32, 64, 128 or 256 words
+    const int distinct = n <= 32    ? sort_keep<1>(n, K, w, a, tok, col, par_out, true)
+                         : n <= 64  ? sort_keep<2>(n, K, w, a, tok, col, par_out, true)
+                         : n <= 128 ? sort_keep<4>(n, K, w, a, tok, col, par_out, true)
+                                    : sort_keep<8>(n, K, w, a, tok, col, par_out, true);
     if (distinct < K) {
         set_status(a.status, DPB_DEV_SHORT_CODE);
         for (int e = distinct + lane; e < K; e += 32) {
@@ -470,11 +474,14 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
             ss = warp_sum(ss);
             if (lane == 0 && a.xnorm) a.xnorm[tok] = sqrtf(ss);
             __syncwarp();
+            // a lane's coordinates lane + 32 j in groups of 8 consecutive j (d is
+            // a multiple of 64, so every lane has the same count)
             auto scan0 = [&](auto f) {
                 for (int i = lane; i < d; i += 32) {
                     const int m = i >> 5, wl = i & 31;
                     const float xv = __uint_as_float((uint32_t)xh[(m * 16 + (wl & 15)) * 2 + (wl >> 4)] << 16);
-                    f(standardise(xv, (uint32_t)i, a, nullptr), true, true, [&] { return (uint32_t)i; });
+                    f(standardise(xv, (uint32_t)i, a, nullptr), true, (m & 7) == 7 || i + 32 >= d,
+                      [&] { return (uint32_t)i; });
                 }
             };
             if (a.mu)
