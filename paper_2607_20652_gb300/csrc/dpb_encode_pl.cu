@@ -41,6 +41,7 @@
 // parents can share a child) are dropped; the first K remain.
 #include <algorithm>
 #include <atomic>
+#include <type_traits>
 
 #include "dpb_encode_mma.cuh"
 #include "dpb_internal.h"
@@ -280,15 +281,15 @@ __device__ __forceinline__ int select_level(Scan scan, float scale, int K, const
     int nd = 0;  // distinct keys in the union
     // Group maxima first; when they hold fewer than K distinct keys (rows of
     // few children, or copies), every candidate's key instead.
-#pragma unroll 1
-    for (int pass = 0; pass < 2; ++pass) {
-        const bool group = pass == 0;
+    // each lane's 4 largest keys: of its group maxima, or (EVERY) of all its
+    // candidates; the choice is made at compile time, out of the candidate loop
+    auto lane_keys = [&](auto every) {
 #pragma unroll
         for (int r = 0; r < 4; ++r) top[r] = 0u;
         float gm = -1.f;  // the largest |v| of the current group (-1: none live)
         scan([&](float v, bool live, bool gend, auto) {
             if (live) gm = fmaxf(gm, fabsf(v));
-            if (gend || !group) {
+            if (gend || decltype(every)::value) {
                 uint32_t c = gm >= 0.f ? akey(gm * scale) + 1u : 0u;
                 gm = -1.f;
 #pragma unroll
@@ -299,6 +300,13 @@ __device__ __forceinline__ int select_level(Scan scan, float scale, int K, const
                 }
             }
         });
+    };
+#pragma unroll 1
+    for (int pass = 0; pass < 2; ++pass) {
+        if (pass == 0)
+            lane_keys(std::false_type{});
+        else
+            lane_keys(std::true_type{});
         mmaenc::warp_sort_desc_runs<4>(top);  // each lane's 4 are in order already
         // distinct keys of the sorted union (copies of one child share a key):
         // drank[r] = rank among them, 0 for a repeat or an empty slot
@@ -667,11 +675,12 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
                     for (int c0 = 0; c0 < D; c0 += 32) {
                         uint32_t v[32];
                         tmem_ld32(taddr + c0, v);
-                        // D is a multiple of 16: a group of 8 columns is live as a whole
+                        // D is a multiple of 16: columns c0 + 16 .. c0 + 31 exist as a
+                        // whole or not at all, and a group of 8 is live as a whole
+                        const bool hi = rv && c0 + 32 <= D;
 #pragma unroll
                         for (int j = 0; j < 32; ++j)
-                            f(__uint_as_float(v[j]), rv && c0 + j < D, (j & 7) == 7,
-                              [&] { return p ^ gl[c0 + j]; });
+                            f(__uint_as_float(v[j]), j < 16 ? rv : hi, (j & 7) == 7, [&] { return p ^ gl[c0 + j]; });
                     }
                 };
                 select_level(scanl, scale, a.kl[l], wb, a, tok, a.off[l], l + 1 < L);
