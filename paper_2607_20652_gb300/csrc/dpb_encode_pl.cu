@@ -142,7 +142,10 @@ __device__ __forceinline__ void copy_b(void *dst, const uint32_t *src, int D, ui
                  : "memory");
 }
 
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
+// Issues the load of 32 consecutive 32-bit columns of this warp's 32 TMEM
+// lanes (one lane per thread). The registers hold the data only after
+// tmem_ld_wait on them.
+__device__ __forceinline__ void tmem_ld32_issue(uint32_t taddr, uint32_t (&v)[32]) {
     asm volatile(
         "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,"
         "%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
@@ -151,7 +154,24 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
           "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]),
           "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
         : "r"(taddr));
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Waits for this thread's TMEM loads. The registers of the load are tied in
+// as read-write operands, so that no use of them is scheduled before the wait.
+__device__ __forceinline__ void tmem_ld_wait(uint32_t (&v)[32]) {
+    asm volatile("tcgen05.wait::ld.sync.aligned;"
+                 : "+r"(v[0]), "+r"(v[1]), "+r"(v[2]), "+r"(v[3]), "+r"(v[4]), "+r"(v[5]), "+r"(v[6]), "+r"(v[7]),
+                   "+r"(v[8]), "+r"(v[9]), "+r"(v[10]), "+r"(v[11]), "+r"(v[12]), "+r"(v[13]), "+r"(v[14]),
+                   "+r"(v[15]), "+r"(v[16]), "+r"(v[17]), "+r"(v[18]), "+r"(v[19]), "+r"(v[20]), "+r"(v[21]),
+                   "+r"(v[22]), "+r"(v[23]), "+r"(v[24]), "+r"(v[25]), "+r"(v[26]), "+r"(v[27]), "+r"(v[28]),
+                   "+r"(v[29]), "+r"(v[30]), "+r"(v[31])
+                 :
+                 : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
+    tmem_ld32_issue(taddr, v);
+    tmem_ld_wait(v);
 }
 
 // Stores 32 consecutive 32-bit columns of this warp's 32 TMEM lanes (one
@@ -506,8 +526,10 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
             const int pp = P <= 16 ? 16 : 32, ntiles = pp / 16;  // slots per token, M = 128 tiles
             // this thread builds block half hb of row rr of each tile
             const int rr = tid & 127, hb = tid >> 7;
-            uint32_t ip[2], iw5[2], iu[2], ihv[2][4];
-            bool irv[2];
+            // A row that is no live parent (a slot past K_{l-1}, a token past T)
+            // takes parent 0 and whatever x its buffer holds: the selection
+            // reads only live rows, and an MMA row depends on its own A row only
+            uint32_t iw5[2], iu[2], ihv[2][4];
             const uint32_t *ixt[2];
 #pragma unroll
             for (int tt = 0; tt < 2; ++tt) {
@@ -517,8 +539,6 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
                 const bool ok = tt < ntiles && grp * kTokens + tokw < a.T && slot < P;
                 const uint32_t *par = reinterpret_cast<const uint32_t *>(smem + lay.par) + tokw * kRows;
                 const uint32_t pv = ok ? par[slot] : 0u;
-                irv[tt] = ok;
-                ip[tt] = pv;
                 iw5[tt] = w5[pv & 31u];
                 iu[tt] = (pv & lo_mask) >> 5;
 #pragma unroll
@@ -591,7 +611,6 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
                     for (int tt = 0; tt < 2; ++tt) {
                         if (tt < ntiles) {
                             const int m = 2 * c + hb;
-                            const bool rv = irv[tt];
                             uint32_t sw = iw5[tt] ^ (0u - (uint32_t)(__popc((uint32_t)m & iu[tt]) & 1));
 #pragma unroll
                             for (int k = 0; k < 4; ++k)
@@ -603,10 +622,10 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
                                 const uint4 xv = xs[q];
                                 const int sh = 15 - 4 * q;
                                 uint4 av;
-                                av.x = rv ? xv.x ^ ((sw << sh) & 0x80008000u) : 0u;
-                                av.y = rv ? xv.y ^ ((sw << (sh - 1)) & 0x80008000u) : 0u;
-                                av.z = rv ? xv.z ^ ((sw << (sh - 2)) & 0x80008000u) : 0u;
-                                av.w = rv ? xv.w ^ ((sw << (sh - 3)) & 0x80008000u) : 0u;
+                                av.x = xv.x ^ ((sw << sh) & 0x80008000u);
+                                av.y = xv.y ^ ((sw << (sh - 1)) & 0x80008000u);
+                                av.z = xv.z ^ ((sw << (sh - 2)) & 0x80008000u);
+                                av.w = xv.w ^ ((sw << (sh - 3)) & 0x80008000u);
                                 *reinterpret_cast<uint4 *>(At + (rr >> 3) * 1024 + (4 * hb + q) * 128 + (rr & 7) * 16) =
                                     av;
                             }
@@ -731,7 +750,7 @@ dpb_status check_per_level(const dpb_config &c) {
 
 void build_per_level_tables(dpb_plan *p) {
     const dpb_config &c = p->cfg;
-    const int nblk = c.d / 32, nch = c.d / kChunk;
+    const int nch = c.d / kChunk;
     auto sign = [&](uint32_t g, int iota) -> uint32_t {
         return (__builtin_popcount(p->M[iota] & g) & 1) ? 0xBF80u : 0x3F80u;
     };
