@@ -283,8 +283,53 @@ __device__ __forceinline__ int sort_keep(int n, int K, const WarpBufs &w, const 
     return distinct;
 }
 
+// Sorts the union of the lanes' R keys (each lane's already descending; 0 =
+// empty) and ranks its distinct keys (copies of one child share a key):
+// drank[r] = rank of key r among them, 0 for a repeat or an empty slot.
+// Returns the number of distinct keys.
+template <int R>
+__device__ __forceinline__ int union_distinct(uint32_t (&v)[R], int (&drank)[R]) {
+    const int lane = threadIdx.x & 31;
+    mmaenc::warp_sort_desc_runs<R>(v);
+    uint32_t prev = __shfl_up_sync(kFull, v[R - 1], 1);
+    int cnt = 0;
+    bool first[R];
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+        first[r] = v[r] != 0u && ((r == 0 && lane == 0) || v[r] != prev);
+        prev = v[r];
+        cnt += first[r];
+    }
+    int base = cnt;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int t = __shfl_up_sync(kFull, base, o);
+        if (lane >= o) base += t;
+    }
+    base -= cnt;
+    int nd = 0;
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+        drank[r] = first[r] ? base + 1 : 0;
+        base += first[r];
+        nd = max(nd, drank[r]);
+    }
+    return (int)__reduce_max_sync(kFull, (uint32_t)nd);
+}
+
+// The union's distinct key of rank `target` (0 if none).
+template <int R>
+__device__ __forceinline__ uint32_t key_of_rank(const uint32_t (&v)[R], const int (&drank)[R], int target) {
+    uint32_t mine = 0u;
+#pragma unroll
+    for (int r = 0; r < R; ++r)
+        if (drank[r] == target) mine = v[r];
+    return __reduce_max_sync(kFull, mine);
+}
+
 // The top K distinct candidates of one token, as explained in the header.
-// `scan(f)` calls f(v, live, gend, index) for every candidate of this lane, in
+// `scan(f)` calls f(v, live, gend, index) for every candidate of this lane (the
+// first nlive lanes hold candidates), in
 // the same order each time and in step across the warp: v is its score before
 // the factor `scale` (> 0; the score is z = v scale), gend marks the last
 // candidate of a group (a group is live or not as a whole), and index() gives
@@ -293,11 +338,10 @@ __device__ __forceinline__ int sort_keep(int n, int K, const WarpBufs &w, const 
 // and, when `par_out`, the kept indices as the next level's parents. Returns
 // the number of distinct candidates kept (< K only with the status bit set).
 template <class Scan>
-__device__ __forceinline__ int select_level(Scan scan, float scale, int K, const WarpBufs &w, const Args &a,
-                                            int64_t tok, int col, bool par_out) {
+__device__ __forceinline__ int select_level(Scan scan, int nlive, float scale, int K, const WarpBufs &w,
+                                            const Args &a, int64_t tok, int col, bool par_out) {
     const int lane = threadIdx.x & 31;
     uint32_t top[4];
-    int drank[4];
     int nd = 0;  // distinct keys in the union
     // Group maxima first; when they hold fewer than K distinct keys (rows of
     // few children, or copies), every candidate's key instead.
@@ -321,53 +365,34 @@ __device__ __forceinline__ int select_level(Scan scan, float scale, int K, const
             }
         });
     };
+    // the union of each lane's first R keys, sorted, and the distinct key of a
+    // given rank in it: R = 2 when the nlive lanes that hold candidates give
+    // at least 2 K keys that way, else R = 4
+    uint32_t u2[2], u4[4];
+    int dr2[2], dr4[4];
+    const bool narrow = nlive >= K;
 #pragma unroll 1
     for (int pass = 0; pass < 2; ++pass) {
         if (pass == 0)
             lane_keys(std::false_type{});
         else
             lane_keys(std::true_type{});
-        mmaenc::warp_sort_desc_runs<4>(top);  // each lane's 4 are in order already
-        // distinct keys of the sorted union (copies of one child share a key):
-        // drank[r] = rank among them, 0 for a repeat or an empty slot
-        {
-            uint32_t prev = __shfl_up_sync(kFull, top[3], 1);
-            int cnt = 0;
-            bool first[4];
+        if (narrow) {
+            u2[0] = top[0];
+            u2[1] = top[1];
+            nd = union_distinct<2>(u2, dr2);
+        } else {
 #pragma unroll
-            for (int r = 0; r < 4; ++r) {
-                first[r] = top[r] != 0u && ((r == 0 && lane == 0) || top[r] != prev);
-                prev = top[r];
-                cnt += first[r];
-            }
-            int base = cnt;
-#pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-                const int t = __shfl_up_sync(kFull, base, o);
-                if (lane >= o) base += t;
-            }
-            base -= cnt;
-#pragma unroll
-            for (int r = 0; r < 4; ++r) {
-                drank[r] = first[r] ? base + 1 : 0;
-                base += first[r];
-            }
+            for (int r = 0; r < 4; ++r) u4[r] = top[r];
+            nd = union_distinct<4>(u4, dr4);
         }
-        nd = 0;
-#pragma unroll
-        for (int r = 0; r < 4; ++r) nd = max(nd, drank[r]);
-        nd = (int)__reduce_max_sync(kFull, (uint32_t)nd);
         if (nd >= K) break;
     }
     // tau = the union's distinct key of rank K: every key of the union is some
     // candidate's, so K distinct candidates reach it and the level's top K
     // distinct all do (the union's last distinct key when it holds fewer)
     const int target = min(K, nd);
-    uint32_t mine = 0u;
-#pragma unroll
-    for (int r = 0; r < 4; ++r)
-        if (drank[r] == target) mine = top[r];
-    uint32_t tau = __reduce_max_sync(kFull, mine);
+    uint32_t tau = narrow ? key_of_rank<2>(u2, dr2, target) : key_of_rank<4>(u4, dr4, target);
     if (tau == 0u) tau = 1u;
     // key(z) + 1 >= tau exactly when |z| >= the float with bits tau - 1
     const float tf = __uint_as_float(tau - 1u);
@@ -488,6 +513,7 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
         if (live) {
             const uint4 *row = reinterpret_cast<const uint4 *>(a.x + tok * d);
             float ss = 0.f;
+#pragma unroll 4  // the row's loads in flight together (4 chunks per lane at d = 1024)
             for (int ch = lane; ch < d / 8; ch += 32) {
                 const uint4 v = row[ch];
 #pragma unroll
@@ -514,7 +540,7 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
             };
             if (a.mu)
                 for (int i = lane; i < d; i += 32) standardise(0.f, (uint32_t)i, a, a.status);
-            select_level(scan0, 1.f, a.kl[0], wb, a, tok, a.off[0], L > 1);
+            select_level(scan0, 32, 1.f, a.kl[0], wb, a, tok, a.off[0], L > 1);  // d >= 64: every lane holds 2+
         } else if (warp < kTokens) {
             wb.par[lane] = 0u;
             __syncwarp();
@@ -702,7 +728,7 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
                             f(__uint_as_float(v[j]), j < 16 ? rv : hi, (j & 7) == 7, [&] { return p ^ gl[c0 + j]; });
                     }
                 };
-                select_level(scanl, scale, a.kl[l], wb, a, tok, a.off[l], l + 1 < L);
+                select_level(scanl, P, scale, a.kl[l], wb, a, tok, a.off[l], l + 1 < L);
             }
             asm volatile("tcgen05.fence::before_thread_sync;");
             __syncthreads();
