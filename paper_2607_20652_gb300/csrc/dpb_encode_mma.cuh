@@ -64,7 +64,7 @@ struct Args {
 // ---- shared-memory layout (32-bit words) ------------------------------------------
 
 __host__ __device__ inline int block_words(int levels, int nblk, int nkc) {
-    // frag [(L-1)][nblk][32][8], W5 [32], VH [nkc][32][32], DD [(L-1)][kDedupSlots], G [L][16]
+    // frag [(L-1)][nblk][2][32][4], W5 [32], VH [nkc][32][32], DD [(L-1)][kDedupSlots], G [L][16]
     return (levels - 1) * nblk * 256 + 32 + nkc * 1024 + (levels - 1) * kDedupSlots + 8 * 16;
 }
 
@@ -795,14 +795,14 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
                             for (int r = 0; r < 4; ++r) acc[u][c][h][r] = 0.f;
                 const uint4 *xa = reinterpret_cast<const uint4 *>(xt) + q4;
                 const uint4 *xb = reinterpret_cast<const uint4 *>(xt + (WIDE ? 0 : nblk * 16)) + q4;
-                const uint4 *fr = reinterpret_cast<const uint4 *>(frag) + lane * 2;
+                const uint4 *fr = reinterpret_cast<const uint4 *>(frag) + lane;
                 const int sh = 15 - q4;
 #pragma unroll 2
                 for (int m = 0; m < nblk; ++m) {
                     const uint4 va = xa[m * 4], vb = xb[m * 4];
                     const uint2 sg = sgn[m * 8 + slot];
                     const uint32_t s0 = sg.x, s1 = sg.y;
-                    const uint4 f0 = fr[m * 64], f1 = fr[m * 64 + 1];
+                    const uint4 f0 = fr[m * 64], f1 = fr[m * 64 + 32];
                     // chunk 0 holds pairs 0 and 1 of the block, chunk 1 pairs 2 and 3
                     const uint32_t a00 = va.x ^ ((s0 << sh) & 0x80008000u);
                     const uint32_t a01 = vb.x ^ ((s1 << sh) & 0x80008000u);

@@ -608,11 +608,11 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
                     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
                         mma_done(g)));
                     Gc = g + 1;
-                    // the tile nbs - 2 chunks ahead (nbs >= 3) or the next one (two
-                    // stages), past the first `ahead`, goes to the stage that chunk
-                    // next - nbs read, once that chunk's MMAs are done (a chunk of
-                    // an earlier level is done already)
-                    const int next = c + (nbs >= 3 ? nbs - 2 : 1);
+                    // the tile nbs - 1 chunks ahead, past the first `ahead`, goes to
+                    // the stage that chunk next - nbs = c - 1 read, once that chunk's
+                    // MMAs are done (they finish before chunk c's start; a chunk of an
+                    // earlier level is done already)
+                    const int next = c + nbs - 1;
                     if (next >= ahead && next < nch) {
                         const uint32_t prev = G0 + (uint32_t)next - (uint32_t)nbs;
                         if (next >= nbs && !mbar_wait(mma_done(prev), phase(prev), a.spin)) {

@@ -26,8 +26,9 @@ struct dpb_plan {
     std::vector<uint32_t> VH;   // [kvh][32][32]
     int kvh = 0;                // chunks of the high half: ceil(t / 5)
     // Tensor-core encoder tables (built when mma_encode is set):
-    //  FRAG[l-1][m][lane][8]: the generator signs gamma_j of level l over
-    //    32-coordinate block m, as bf16 +-1 pairs in mma.sync B-fragment order;
+    //  FRAG[l-1][m][chunk][lane][4]: the generator signs gamma_j of level l
+    //    over 32-coordinate block m, as bf16 +-1 pairs in mma.sync B-fragment
+    //    order (chunk 0: pairs 0 and 1 of the block, chunk 1: pairs 2 and 3);
     //  DD[l-1][kDedupSlots]: open-addressing table of the differences
     //    g_j ^ g_j' (j != j') of level l below 2^bits[l-1], one word per
     //    entry: (difference + 1) << 4 | j (0 = empty).

@@ -173,7 +173,10 @@ void build_mma_tables(dpb_plan *p) {
                     const int n = 8 * half + lane / 4, q4 = lane % 4, pair = 2 * chunk + reg;
                     const uint32_t g = p->G[(size_t)l * DPB_MAX_CHILDREN + n];
                     const int ia = 32 * m + frag_coord(q4, pair, 0), ib = 32 * m + frag_coord(q4, pair, 1);
-                    p->FRAG[(((size_t)(l - 1) * nblk + m) * 32 + lane) * 8 + w] = sign_bf16(g, ia) | (sign_bf16(g, ib) << 16);
+                    // chunk-major: a warp's 128-bit loads of one chunk read 512
+                    // contiguous bytes (no bank conflict)
+                    p->FRAG[((((size_t)(l - 1) * nblk + m) * 2 + chunk) * 32 + lane) * 4 + w % 4] =
+                        sign_bf16(g, ia) | (sign_bf16(g, ib) << 16);
                 }
     p->DD.assign((size_t)(c.levels - 1) * kDedupSlots, 0u);
     for (int l = 1; l < c.levels; ++l) {
