@@ -323,11 +323,78 @@ __device__ __forceinline__ void warp_sort_desc_runs(W (&v)[R]) {
 // prefix of L, found by bisection); a list word moves down by the entrants
 // ahead of it; whatever lands at k or beyond drops out. When 8..32 words enter
 // and `beam` is given, the first 8 entrants become the beam.
+//
+// Up to 32 entrants (the usual case) take another route, free of a loop over
+// the entrants: each finds its gap in the list by bisection (pos = list words
+// ahead of it) and a histogram H of the gaps (in E, past the entrants) gives
+// by prefix sums how far each list word moves (the entrants in gaps at or
+// before it) and how many entrants are ahead of each entrant (those in
+// earlier gaps, and those of its own gap that are larger, compared directly).
 template <int KPL>
-__device__ __noinline__ void merge_sorted(uint64_t *L, int k, const uint64_t *E, int m, uint32_t *beam) {
+__device__ __noinline__ void merge_sorted(uint64_t *L, int k, uint64_t *E, int m, uint32_t *beam) {
     const int lane = threadIdx.x & 31;
-    int top = 1;
-    while (2 * top <= k) top <<= 1;
+    const int top = 1 << (31 - __clz(k));  // the largest power of 2 <= k
+    if (m <= 32) {
+        uint32_t *H = reinterpret_cast<uint32_t *>(E + 32);  // [k] entrants per gap
+        const uint64_t mine = lane < m ? E[lane] : 0ull;
+        uint64_t lv[KPL];
+#pragma unroll
+        for (int r = 0; r < KPL; ++r) {
+            const int e = lane + 32 * r;
+            lv[r] = e < k ? L[e] : 0ull;
+            if (e < k) H[e] = 0u;
+        }
+        int pos = 0;  // list words ahead of mine (< k: an entrant is ahead of L[k-1])
+        for (int step = top; step > 0; step >>= 1) {
+            const int np = pos + step;
+            if (np <= k && L[np - 1] > mine) pos = np;
+        }
+        __syncwarp();
+        if (lane < m) atomicAdd(&H[pos], 1u);
+        __syncwarp();
+        // cum[r] = entrants in gaps 0 .. lane + 32 r: how far list word lane + 32 r moves
+        int cum[KPL];
+        int carry = 0;
+#pragma unroll
+        for (int r = 0; r < KPL; ++r) {
+            const int e = lane + 32 * r;
+            int v = e < k ? (int)H[e] : 0;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int t = __shfl_up_sync(kFull, v, o);
+                if (lane >= o) v += t;
+            }
+            cum[r] = carry + v;
+            carry += __shfl_sync(kFull, v, 31);
+        }
+        // entrants ahead of mine: those of the gaps before pos ...
+        int rs = 0;
+        const int q = pos - 1;
+#pragma unroll
+        for (int r = 0; r < KPL; ++r) {
+            const int v = __shfl_sync(kFull, cum[r], q & 31);
+            if (q >= 0 && (q >> 5) == r) rs = v;
+        }
+        // ... and the larger ones of its own gap (lanes past m never match)
+        unsigned same = __match_any_sync(kFull, lane < m ? pos : -1 - lane) & ~(1u << lane);
+        const int rounds = (int)__reduce_max_sync(kFull, (uint32_t)__popc(same));
+        for (int it = 0; it < rounds; ++it) {
+            const int src = same ? __ffs(same) - 1 : lane;
+            same &= same - 1u;
+            const uint64_t o = __shfl_sync(kFull, mine, src);
+            rs += src != lane && o > mine;
+        }
+        __syncwarp();
+        if (lane < m && rs + pos < k) L[rs + pos] = mine;
+#pragma unroll
+        for (int r = 0; r < KPL; ++r) {
+            const int e = lane + 32 * r;
+            if (e < k && e + cum[r] < k) L[e + cum[r]] = lv[r];
+        }
+        if (beam && m >= kBeam && lane < m && rs < kBeam) beam[rs] = cword_idx(mine);
+        __syncwarp();
+        return;
+    }
     for (int q0 = 0; q0 < m; q0 += 32) {
         const int mq = min(32, m - q0);
         const uint64_t mine = lane < mq ? E[q0 + lane] : 0ull;
