@@ -494,8 +494,9 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
     auto a_full = [&](uint32_t g) { return mbar0 + 8u * (2 * kMaxStages + (g & 1u)); };
     uint32_t G = 0;  // chunks of the levels done so far (every thread)
     bool failed = false;
-    // the issuer: generator tiles are copied and consumed in chunk order (the
-    // copies of chunks [consumed, issued) are in flight); Gc chunks committed
+    // generator tiles are copied (by thread 0) and consumed (by the issuer) in
+    // chunk order: the copies of chunks [consumed, issued) are in flight; the
+    // issuer has committed the MMAs of Gc chunks
     uint32_t issued = 0, consumed = 0, Gc = 0;
     bool tfail = false;  // a wait of this thread gave up
     auto issue_b = [&](uint32_t g, const uint32_t *src, int D) {
@@ -574,15 +575,10 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
             const uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(D >> 3) << 17) | (8u << 24);
             const uint32_t *gt = a.GT + a.gt_off[l];
             const uint32_t G0 = G;
-            // the level's first tiles (every earlier MMA is done, so every stage
-            // is free): every stage with three or more, one with two
-            const int ahead = nbs >= 3 ? nbs : nbs - 1;
             bool bfail = false;  // a builder's wait gave up
             if (tid == kIssuer) {
                 // ---- the issuer: for each chunk, once its A stage is built and
-                // its generator tile has landed, the MMAs and their commit; it
-                // refills a generator stage once the MMAs that read it are done
-                for (int c = 0; c < min(ahead, nch); ++c) issue_b(G0 + c, gt + (int64_t)c * D * 32, D);
+                // its generator tile has landed, the MMAs and their commit
                 for (int c = 0; c < nch; ++c) {
                     const uint32_t g = G0 + c;
                     if (!mbar_wait(a_full(g), (g >> 1) & 1u, a.spin) || !mbar_wait(full_b(g), phase(g), a.spin)) {
@@ -608,30 +604,23 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
                     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
                         mma_done(g)));
                     Gc = g + 1;
-                    // the tile nbs - 1 chunks ahead, past the first `ahead`, goes to
-                    // the stage that chunk next - nbs = c - 1 read, once that chunk's
-                    // MMAs are done (they finish before chunk c's start; a chunk of an
-                    // earlier level is done already)
-                    const int next = c + nbs - 1;
-                    if (next >= ahead && next < nch) {
-                        const uint32_t prev = G0 + (uint32_t)next - (uint32_t)nbs;
-                        if (next >= nbs && !mbar_wait(mma_done(prev), phase(prev), a.spin)) {
-                            set_status(a.status, DPB_DEV_TIMEOUT);
-                            tfail = true;
-                            break;
-                        }
-                        issue_b(G0 + next, gt + (int64_t)next * D * 32, D);
-                    }
                 }
             } else if (tid < kIssuer) {
                 // ---- the token warps build A: chunk g's stage is free once the
-                // MMAs of chunk g - 2 are done
+                // MMAs of chunk g - 2 are done. Thread 0 also copies the generator
+                // tiles: the level's first nbs at its start (every earlier MMA is
+                // done, so every stage is free), then, once chunk g - 2's MMAs are
+                // done, the tile of chunk g + nbs - 2 into the stage they read
+                if (tid == 0)
+                    for (int c = 0; c < min(nbs, nch); ++c) issue_b(G0 + c, gt + (int64_t)c * D * 32, D);
                 for (int c = 0; c < nch; ++c) {
                     const uint32_t g = G0 + c;
                     if (c >= 2 && !mbar_wait(mma_done(g - 2), phase(g - 2), a.spin)) {
                         bfail = true;
                         break;
                     }
+                    const int next = c + nbs - 2;
+                    if (tid == 0 && c >= 2 && next < nch) issue_b(G0 + next, gt + (int64_t)next * D * 32, D);
                     uint8_t *As = sA + (g & 1u) * 2 * kATile;
 #pragma unroll
                     for (int tt = 0; tt < 2; ++tt) {
@@ -737,10 +726,20 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
     if (failed) set_status(a.status, DPB_DEV_TIMEOUT);
     // drain (bounded, with the default bound): every generator-tile copy still
     // in flight lands, and the last commit (which covers every MMA issued)
-    // arrives, before the block frees its TMEM and its shared memory
-    if (failed && tid == kIssuer) {
-        for (uint32_t g = consumed; g < issued; ++g) mbar_wait(full_b(g), phase(g), kSpin);
-        if (Gc > 0) mbar_wait(mma_done(Gc - 1), phase(Gc - 1), kSpin);
+    // arrives, before the block frees its TMEM and its shared memory. The
+    // issuer's counts reach thread 0 through shared memory (failed is the
+    // block's, so every thread is here)
+    if (failed) {
+        if (tid == kIssuer) {
+            tmem_slot[1] = consumed;
+            tmem_slot[2] = Gc;
+        }
+        __syncthreads();
+        if (tid == 0) {
+            for (uint32_t g = tmem_slot[1]; g < issued; ++g) mbar_wait(full_b(g), phase(g), kSpin);
+            const uint32_t gc = tmem_slot[2];
+            if (gc > 0) mbar_wait(mma_done(gc - 1), phase(gc - 1), kSpin);
+        }
     }
     asm volatile("tcgen05.fence::before_thread_sync;");
     __syncthreads();
