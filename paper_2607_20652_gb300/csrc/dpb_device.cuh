@@ -80,7 +80,7 @@ struct RowOps {
     __device__ __forceinline__ static void scale_in(float *buf, const T *row, int d, float c) {
         const int lane = threadIdx.x & 31;
         if (VEC) {
-#pragma unroll 3
+#pragma unroll 2
             for (int i = 4 * lane; i < d; i += 128) {
                 const float4 v = ld4(row + i);
                 *reinterpret_cast<float4 *>(buf + i) = make_float4(c * v.x, c * v.y, c * v.z, c * v.w);
@@ -114,7 +114,7 @@ struct RowOps {
                                                  float &sxx, float &srr, float &sgr) {
         const int lane = threadIdx.x & 31;
         if (VEC) {
-#pragma unroll 3  // three rows' loads of three trips in flight together
+#pragma unroll 2  // the rows' loads of two trips in flight together
             for (int i = 4 * lane; i < d; i += 128) {
                 const float4 xv = ld4(x + i), gv = ld4(g + i);
                 const float4 rv = *reinterpret_cast<const float4 *>(r + i);
@@ -138,7 +138,7 @@ struct RowOps {
     __device__ __forceinline__ static void project(float *buf, const T *row, int d, float c, float beta) {
         const int lane = threadIdx.x & 31;
         if (VEC) {
-#pragma unroll 3
+#pragma unroll 2
             for (int i = 4 * lane; i < d; i += 128) {
                 const float4 r = *reinterpret_cast<const float4 *>(buf + i), g = ld4(row + i);
                 *reinterpret_cast<float4 *>(buf + i) =
