@@ -324,8 +324,9 @@ __device__ __forceinline__ void warp_sort_desc_runs(W (&v)[R]) {
 // ahead of it; whatever lands at k or beyond drops out. When 8..32 words enter
 // and `beam` is given, the first 8 entrants become the beam.
 //
-// Up to 32 entrants (the usual case) take another route, free of a loop over
-// the entrants: each finds its gap in the list by bisection (pos = list words
+// 8 to 32 entrants (the usual case) take another route, free of a loop over
+// the entrants (its fixed cost loses to the loop below 8): each finds its gap
+// in the list by bisection (pos = list words
 // ahead of it) and a histogram H of the gaps (in E, past the entrants) gives
 // by prefix sums how far each list word moves (the entrants in gaps at or
 // before it) and how many entrants are ahead of each entrant (those in
@@ -334,7 +335,7 @@ template <int KPL>
 __device__ __noinline__ void merge_sorted(uint64_t *L, int k, uint64_t *E, int m, uint32_t *beam) {
     const int lane = threadIdx.x & 31;
     const int top = 1 << (31 - __clz(k));  // the largest power of 2 <= k
-    if (m <= 32) {
+    if (m >= 8 && m <= 32) {
         uint32_t *H = reinterpret_cast<uint32_t *>(E + 32);  // [k] entrants per gap
         const uint64_t mine = lane < m ? E[lane] : 0ull;
         uint64_t lv[KPL];
