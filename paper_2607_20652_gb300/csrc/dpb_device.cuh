@@ -296,6 +296,16 @@ __device__ __forceinline__ void set_status(int32_t *status, int32_t bit) {
 // (nullable) holds the pairs (mu_c, r_c): one 8-byte load instead of one from
 // each table. A sigma that is not a positive finite number (r_c outside
 // (0, inf)) sets DPB_DEV_BAD_SIGMA when `status` is given.
+// The table entries (mu_c, 1 / sigma_c) of feature c: the packed pair, or one
+// load from each table. No side effect, so that callers can issue a batch of
+// them before using any: z = (s - e.x) * e.y, and zbad(e.y) flags a sigma that
+// is not a positive finite number.
+__device__ __forceinline__ float2 ztab(uint32_t c, const float *mu, const float *sigma, const float2 *tab) {
+    if (tab) return tab[c];
+    return make_float2(mu[c], __frcp_rn(sigma[c]));
+}
+__device__ __forceinline__ bool zbad(float r) { return !(r > 0.f && r <= 3.402823466e38f); }
+
 __device__ __forceinline__ float zscore(float s, uint32_t c, const float *mu, const float *sigma,
                                         const float2 *tab, int32_t *status) {
     float m, r;

@@ -437,6 +437,35 @@ __device__ __forceinline__ float standardise(float s, uint32_t c, const Args &a,
     return a.mu ? zscore(s, c, a.mu, a.sigma, a.tab, status) : s;
 }
 
+// Standardised scores of one warp's TMEM rows, columns [cb, ce) (Delta = D
+// children of parent p, live when ok): z = (s / sqrt(d) - mu_c) / sigma_c in
+// place of s. Four columns' table loads are in flight at a time. Not inlined:
+// its registers do not count against the kernel's, whose plain path runs
+// without it.
+__device__ __noinline__ void standardise_cols(const float *mu, const float *sigma, const float2 *tab,
+                                              int32_t *status, float inv_sqrt_d, uint32_t taddr, int cb, int ce,
+                                              int D, bool ok, uint32_t p, const uint32_t *gl) {
+    bool bad = false;
+    for (int c0 = cb; c0 < ce; c0 += 32) {
+        uint32_t v[32];
+        tmem_ld32(taddr + c0, v);
+#pragma unroll
+        for (int h = 0; h < 32; h += 4) {
+            float2 e[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+                e[j] = ok && c0 + h + j < D ? ztab(p ^ gl[c0 + h + j], mu, sigma, tab) : make_float2(0.f, 1.f);
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                v[h + j] = __float_as_uint((__uint_as_float(v[h + j]) * inv_sqrt_d - e[j].x) * e[j].y);
+                bad |= zbad(e[j].y);
+            }
+        }
+        tmem_st32(taddr + c0, v);
+    }
+    if (bad) set_status(status, DPB_DEV_BAD_SIGMA);
+}
+
 // ---- the kernel ----------------------------------------------------------------------
 
 __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
@@ -680,16 +709,7 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
                     const bool ok = grp * kTokens + tokw < a.T && slot < P;
                     const uint32_t p = ok ? reinterpret_cast<const uint32_t *>(smem + lay.par)[tokw * kRows + slot] : 0u;
                     const uint32_t taddr = tmem + ((uint32_t)(32 * q) << 16) + 256u * tile;
-                    for (int c0 = cb; c0 < ce; c0 += 32) {
-                        uint32_t v[32];
-                        tmem_ld32(taddr + c0, v);
-#pragma unroll
-                        for (int j = 0; j < 32; ++j)
-                            if (ok && c0 + j < D)
-                                v[j] = __float_as_uint(standardise(__uint_as_float(v[j]) * a.inv_sqrt_d, p ^ gl[c0 + j], a,
-                                                                   a.status));
-                        tmem_st32(taddr + c0, v);
-                    }
+                    standardise_cols(a.mu, a.sigma, a.tab, a.status, a.inv_sqrt_d, taddr, cb, ce, D, ok, p, gl);
                 }
                 asm volatile("tcgen05.fence::before_thread_sync;");
                 __syncthreads();
