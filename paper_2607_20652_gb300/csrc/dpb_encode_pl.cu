@@ -51,8 +51,9 @@ namespace dpb {
 namespace {
 
 constexpr int kTokens = 8;      // tokens per block, one per warp
-constexpr int kThreads = (kTokens + 1) * 32;  // and a ninth warp, whose lane 0 issues the MMAs
-constexpr int kIssuer = kTokens * 32;         // that thread
+constexpr int kThreads = (kTokens + 2) * 32;  // and a ninth warp, whose lane 0 issues the MMAs,
+constexpr int kIssuer = kTokens * 32;         // and a tenth, whose lane 0 copies the generator tiles
+constexpr int kProducer = (kTokens + 1) * 32;
 constexpr int kRows = 32;       // tensor-core rows per token (parent slots)
 constexpr int kChunk = 64;      // coordinates per K chunk
 constexpr int kATile = 128 * kChunk * 2;  // one M = 128 tile of a chunk
@@ -103,7 +104,7 @@ __host__ __device__ inline Layout layout(int d, int levels, int kvh, int dmax, i
     l.w5 = l.g + levels * 256 * 4;
     l.par = l.w5 + 32 * 4;
     l.mbar = l.par + kTokens * kRows * 4;
-    l.total = l.mbar + (2 * kMaxStages + 2) * 8 + 16;
+    l.total = l.mbar + (2 * kMaxStages + 6) * 8 + 16;
     return l;
 }
 
@@ -479,9 +480,9 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
     uint32_t *vh = reinterpret_cast<uint32_t *>(smem + lay.vh);
     uint32_t *gs = reinterpret_cast<uint32_t *>(smem + lay.g);
     uint32_t *w5 = reinterpret_cast<uint32_t *>(smem + lay.w5);
-    // full_b[stages], mma_done[stages], a_full[2]
+    // full_b[stages], mma_done[stages], a_full[2 + 4]
     uint64_t *mbar = reinterpret_cast<uint64_t *>(smem + lay.mbar);
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(mbar + 2 * kMaxStages + 2);
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(mbar + 2 * kMaxStages + 6);
     WarpBufs wb;
     wb.par = reinterpret_cast<uint32_t *>(smem + lay.par) + warp * kRows;
     wb.z = reinterpret_cast<float *>(sB + warp * kSelBytes);
@@ -496,7 +497,7 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
     if (tid == 0) {
         for (int i = 0; i < 2 * kMaxStages; ++i)
             asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(mbar + i)));
-        for (int i = 0; i < 2; ++i)  // an A stage is built once each of the token warps arrives
+        for (int i = 0; i < 6; ++i)  // an A stage is built once each of the token warps arrives
             asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(mbar + 2 * kMaxStages + i)),
                          "r"(kTokens));
         asm volatile("fence.mbarrier_init.release.cluster;");
@@ -519,11 +520,16 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
     auto mma_done = [&](uint32_t g) { return mbar0 + 8u * (kMaxStages + g % (uint32_t)nbs); };
     auto phase = [&](uint32_t g) { return (g / (uint32_t)nbs) & 1u; };
     auto stage_b = [&](uint32_t g) { return sB + (g % (uint32_t)nbs) * a.dmax * 128; };
-    // A stage g & 1 is built for chunk g the (g / 2)-th time
-    auto a_full = [&](uint32_t g) { return mbar0 + 8u * (2 * kMaxStages + (g & 1u)); };
+    // A stages: a level of two M = 128 tiles has two of 32 KB, a level of one
+    // tile four of 16 KB (the same region; two of them with fewer than four
+    // generator stages). Counting the chunks of each kind
+    // of level over every level and group (ga), chunk ga of a two-tile level
+    // uses stage and mbarrier a_full[ga & 1] and of a one-tile level stage
+    // ga & 3 and a_full[2 + (ga & 3)], each the (ga / stages)-th time.
     uint32_t G = 0;  // chunks of the levels done so far (every thread)
+    uint32_t GA2 = 0, GA4 = 0;  // chunks of two-tile and of one-tile levels done so far
     bool failed = false;
-    // generator tiles are copied (by thread 0) and consumed (by the issuer) in
+    // generator tiles are copied (by the producer) and consumed (by the issuer) in
     // chunk order: the copies of chunks [consumed, issued) are in flight; the
     // issuer has committed the MMAs of Gc chunks
     uint32_t issued = 0, consumed = 0, Gc = 0;
@@ -604,13 +610,46 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
             const uint32_t idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(D >> 3) << 17) | (8u << 24);
             const uint32_t *gt = a.GT + a.gt_off[l];
             const uint32_t G0 = G;
+            // four A stages of one tile; the builders then wait for chunk c - 4's
+            // MMAs, on the mbarrier of generator stage (c - 4) % nbs, which no
+            // later chunk before c reuses only when nbs >= 4
+            const bool a4 = ntiles == 1 && nbs >= 4;
+            const int na = a4 ? 4 : 2;
+            const uint32_t GA0 = a4 ? GA4 : GA2;
+            auto a_stage = [&](int c) {
+                const uint32_t ga = GA0 + (uint32_t)c;
+                return a4 ? sA + (ga & 3u) * kATile : sA + (ga & 1u) * 2 * kATile;
+            };
+            auto a_full = [&](int c) {
+                const uint32_t ga = GA0 + (uint32_t)c;
+                return mbar0 + 8u * (2 * kMaxStages + (a4 ? 2u + (ga & 3u) : (ga & 1u)));
+            };
+            auto a_phase = [&](int c) {
+                const uint32_t ga = GA0 + (uint32_t)c;
+                return a4 ? (ga >> 2) & 1u : (ga >> 1) & 1u;
+            };
             bool bfail = false;  // a builder's wait gave up
-            if (tid == kIssuer) {
+            if (tid == kProducer) {
+                // ---- the producer: the level's first nbs tiles at its start (every
+                // earlier MMA is done, so every stage is free), then, once chunk
+                // c - 2's MMAs are done, the tile of chunk c + nbs - 2 into the stage
+                // they read
+                for (int c = 0; c < min(nbs, nch); ++c) issue_b(G0 + c, gt + (int64_t)c * D * 32, D);
+                for (int c = 2; c + nbs - 2 < nch; ++c) {
+                    if (!mbar_wait(mma_done(G0 + c - 2), phase(G0 + c - 2), a.spin)) {
+                        set_status(a.status, DPB_DEV_TIMEOUT);
+                        tfail = true;
+                        break;
+                    }
+                    const int next = c + nbs - 2;
+                    issue_b(G0 + next, gt + (int64_t)next * D * 32, D);
+                }
+            } else if (tid == kIssuer) {
                 // ---- the issuer: for each chunk, once its A stage is built and
                 // its generator tile has landed, the MMAs and their commit
                 for (int c = 0; c < nch; ++c) {
                     const uint32_t g = G0 + c;
-                    if (!mbar_wait(a_full(g), (g >> 1) & 1u, a.spin) || !mbar_wait(full_b(g), phase(g), a.spin)) {
+                    if (!mbar_wait(a_full(c), a_phase(c), a.spin) || !mbar_wait(full_b(g), phase(g), a.spin)) {
                         set_status(a.status, DPB_DEV_TIMEOUT);
                         tfail = true;
                         break;
@@ -618,7 +657,7 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
                     consumed = g + 1;
                     asm volatile("tcgen05.fence::after_thread_sync;");
                     const uint32_t bb = smem_u32(stage_b(g));
-                    const uint8_t *As = sA + (g & 1u) * 2 * kATile;
+                    const uint8_t *As = a_stage(c);
                     for (int tt = 0; tt < ntiles; ++tt) {
                         const uint32_t ab = smem_u32(As + tt * kATile);
 #pragma unroll
@@ -635,22 +674,15 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
                     Gc = g + 1;
                 }
             } else if (tid < kIssuer) {
-                // ---- the token warps build A: chunk g's stage is free once the
-                // MMAs of chunk g - 2 are done. Thread 0 also copies the generator
-                // tiles: the level's first nbs at its start (every earlier MMA is
-                // done, so every stage is free), then, once chunk g - 2's MMAs are
-                // done, the tile of chunk g + nbs - 2 into the stage they read
-                if (tid == 0)
-                    for (int c = 0; c < min(nbs, nch); ++c) issue_b(G0 + c, gt + (int64_t)c * D * 32, D);
+                // ---- the token warps build A: chunk c's stage is free once the
+                // MMAs of chunk c - na are done (a stage of an earlier level is free)
                 for (int c = 0; c < nch; ++c) {
                     const uint32_t g = G0 + c;
-                    if (c >= 2 && !mbar_wait(mma_done(g - 2), phase(g - 2), a.spin)) {
+                    if (c >= na && !mbar_wait(mma_done(g - na), phase(g - na), a.spin)) {
                         bfail = true;
                         break;
                     }
-                    const int next = c + nbs - 2;
-                    if (tid == 0 && c >= 2 && next < nch) issue_b(G0 + next, gt + (int64_t)next * D * 32, D);
-                    uint8_t *As = sA + (g & 1u) * 2 * kATile;
+                    uint8_t *As = a_stage(c);
 #pragma unroll
                     for (int tt = 0; tt < 2; ++tt) {
                         if (tt < ntiles) {
@@ -679,7 +711,7 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
                     // cores once the issuer has seen the warp's arrival
                     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                     __syncwarp();
-                    if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(a_full(g)) : "memory");
+                    if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(a_full(c)) : "memory");
                 }
             }
             {
@@ -692,6 +724,10 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
                 }
             }
             G = G0 + nch;
+            if (a4)
+                GA4 += nch;
+            else
+                GA2 += nch;
             asm volatile("tcgen05.fence::after_thread_sync;");
             const uint32_t *gl = gs + l * 256;
             // ---- standardised scores, once per candidate (§2.2): z replaces s in
@@ -747,7 +783,7 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
     // drain (bounded, with the default bound): every generator-tile copy still
     // in flight lands, and the last commit (which covers every MMA issued)
     // arrives, before the block frees its TMEM and its shared memory. The
-    // issuer's counts reach thread 0 through shared memory (failed is the
+    // issuer's counts reach the producer through shared memory (failed is the
     // block's, so every thread is here)
     if (failed) {
         if (tid == kIssuer) {
@@ -755,7 +791,7 @@ __global__ void __launch_bounds__(kThreads, 1) encode_pl_kernel(Args a) {
             tmem_slot[2] = Gc;
         }
         __syncthreads();
-        if (tid == 0) {
+        if (tid == kProducer) {
             for (uint32_t g = tmem_slot[1]; g < issued; ++g) mbar_wait(full_b(g), phase(g), kSpin);
             const uint32_t gc = tmem_slot[2];
             if (gc > 0) mbar_wait(mma_done(gc - 1), phase(gc - 1), kSpin);
