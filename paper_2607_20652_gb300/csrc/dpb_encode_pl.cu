@@ -20,12 +20,14 @@
 //    32-coordinate block hold coordinates (i, i + 16), whose sign bits one
 //    shift moves to the bf16 sign positions;
 //  - B (Delta_l x 64 bf16, the generators' +-1 signs in the same order) is
-//    one bulk copy of the plan's precomputed tile;
+//    one bulk copy of the plan's precomputed tile, issued by a tenth warp's
+//    lane 0 (the producer) once the MMAs that last read its stage are done;
 //  - a ninth warp's lane 0 issues the MMAs of a chunk once the 8 token
 //    warps have arrived on the A stage's mbarrier and the generator tile has
 //    landed, and commits them to an mbarrier that frees the chunk's buffers;
-//    scores accumulate in TMEM. The token warps build the next A stage
-//    meanwhile (two stages), so no warp both builds A and waits to issue.
+//    scores accumulate in TMEM. The token warps build the next A stages
+//    meanwhile (two of two tiles, or four of one tile), so no warp both
+//    builds A and waits to issue.
 // Every mbarrier wait is bounded; a wait that gives up sets
 // DPB_DEV_TIMEOUT and stops the block, which then waits (again bounded) for
 // its bulk copies and MMAs still in flight and frees its TMEM.
