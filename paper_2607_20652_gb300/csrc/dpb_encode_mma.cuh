@@ -540,7 +540,8 @@ __device__ __forceinline__ bool level0_union(const uint4 *row, int nch, int k, u
 // of z = (x_i - mu_i) / sigma_i (a standardised score does not fit the 16-bit
 // key of a bf16 coordinate). Each lane keeps its R best words; the k-th of the
 // union is the threshold, and the few words at or above it that a lane did not
-// keep are merged in. Returns false (nothing written) when they overflow E.
+// keep (found by rescanning only the lanes that can hold them) are merged in.
+// Returns false (nothing written) when they overflow E.
 template <int R, int KPL>
 __device__ __forceinline__ bool level0_union_std(const Args &a, const uint16_t *xh, int k, uint64_t *E, int ecap,
                                                  uint64_t *L, uint32_t *beam) {
@@ -565,32 +566,42 @@ __device__ __forceinline__ bool level0_union_std(const Args &a, const uint16_t *
     for (int r = 0; r < R; ++r)
         if (r == (k - 1) % R) mine = top[r];
     const uint64_t tau = __shfl_sync(kFull, mine, (k - 1) / R);
-    int nx = 0;
+    // Extras are unkept words in [tau, kept_min): only lanes whose R kept
+    // words all reach tau can have them. The warp rescans just those lanes'
+    // coordinates (lane l owns l + 32 j) together, a few per lane, each with
+    // its table entries, gathering the extras into E.
+    const bool flag = kept_min >= tau && kept_min != 0ull;
+    const unsigned fm = __ballot_sync(kFull, flag);
+    const int nf = __popc(fm), ne = (d + 31) / 32;  // flagged lanes; coordinates per lane
+    const int cap = ecap - 16;                      // E's last 16 entries hold the flagged lanes
+    int total = 0;
+    if (nf) {
+        uint32_t *fl = reinterpret_cast<uint32_t *>(E + cap);
+        if (flag) fl[__popc(fm & lanes_below())] = (uint32_t)lane;
+        __syncwarp();
 #pragma unroll 1
-    for (int i = lane; i < d; i += 32) {
-        const uint64_t w = cword(standardise(x_at(xh, i), (uint32_t)i, a, nullptr), (uint32_t)i);
-        nx += (w >= tau) & (w < kept_min);
+        for (int q0 = 0; q0 < nf * ne; q0 += 32) {
+            const int q = q0 + lane, f = q / ne, j = q - f * ne;
+            const int owner = q < nf * ne ? (int)fl[f] : 0;
+            const int i = owner + 32 * j;
+            const uint64_t km = __shfl_sync(kFull, kept_min, owner);
+            uint64_t w = 0ull;
+            if (q < nf * ne && i < d) w = cword(standardise(x_at(xh, i), (uint32_t)i, a, nullptr), (uint32_t)i);
+            const bool take = w >= tau && w < km && w != 0ull;
+            const unsigned mb = __ballot_sync(kFull, take);
+            const int pos = total + __popc(mb & lanes_below());
+            if (take && pos < cap) E[pos] = w;
+            total += __popc(mb);
+        }
+        __syncwarp();
     }
-    const int total = __reduce_add_sync(kFull, nx);
-    if (total > ecap) return false;
+    if (total > cap) return false;
 #pragma unroll
     for (int r = 0; r < R; ++r) {
         const int e = lane * R + r;
         if (e < k) L[e] = top[r];
     }
     if (total > 0) {
-        int off = nx;  // exclusive prefix of the extras over the lanes
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int v = __shfl_up_sync(kFull, off, o);
-            if (lane >= o) off += v;
-        }
-        off -= nx;
-#pragma unroll 1
-        for (int i = lane; i < d; i += 32) {
-            const uint64_t w = cword(standardise(x_at(xh, i), (uint32_t)i, a, nullptr), (uint32_t)i);
-            if (w >= tau && w < kept_min) E[off++] = w;
-        }
         __syncwarp();
         merge_sorted<KPL>(L, k, E, total, nullptr);
         if (lane < kBeam) beam[lane] = cword_idx(L[lane]);
@@ -713,7 +724,9 @@ __device__ __forceinline__ void level0_bisect(const Args &a, const uint16_t *xh,
 // 0..7 and 8..15 take the places of the two tokens (same x, one code list);
 // repeats are found over all 120 slot pairs and the next beam is the top of
 // both halves' children.
-template <int NKC, int KPL, bool COSET, bool WIDE>
+// STD: standardisation tables are given (a separate instantiation, so that
+// the plain kernel carries none of their code).
+template <int NKC, int KPL, bool COSET, bool WIDE, bool STD>
 __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
     extern __shared__ __align__(16) uint32_t smem[];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
@@ -784,9 +797,12 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
             uint32_t *bt = beams + tk * kBeam;
             bool done = false;
             // each lane keeps R words, so the union of 32 R holds at least 2 k
-            if (KPL <= 4)
-                done = a.mu ? level0_union_std<(KPL <= 2 ? 4 : 8), KPL>(a, xh + tk * nblk * 32, k, E, a.ecap, Lt, bt)
-                            : level0_union<(KPL <= 2 ? 4 : 8), KPL>(row, nch, k, E, a.ecap, Lt, bt);
+            if constexpr (KPL <= 4) {
+                if constexpr (STD)
+                    done = level0_union_std<(KPL <= 2 ? 4 : 8), KPL>(a, xh + tk * nblk * 32, k, E, a.ecap, Lt, bt);
+                else
+                    done = level0_union<(KPL <= 2 ? 4 : 8), KPL>(row, nch, k, E, a.ecap, Lt, bt);
+            }
             if (!done)
                 level0_bisect(a, xh + tk * nblk * 32, reinterpret_cast<float *>(E),
                               reinterpret_cast<uint32_t *>(E) + a.ecap, a.ecap, Lt, bt);
@@ -896,7 +912,7 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
                             ((acc[0][0][h][r] + acc[0][1][h][r]) + (acc[1][0][h][r] + acc[1][1][h][r])) * a.inv_sqrt_d;
             }
             const uint32_t *gl = s_g + l * 16;
-            if (a.mu) {  // standardise both rows' children now: their table loads go out together
+            if constexpr (STD) {  // standardise both rows' children now: their table loads go out together
 #pragma unroll
                 for (int tk = 0; tk < 2; ++tk)
 #pragma unroll
@@ -1032,15 +1048,21 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
     }
 }
 
-template <int NKC, int KPL, bool COSET, bool WIDE = false>
-cudaError_t launch_kpl(const dpb_plan *p, const Args &a, int warps, cudaStream_t stream) {
+template <int NKC, int KPL, bool COSET, bool WIDE, bool STD>
+cudaError_t launch_kpl_std(const dpb_plan *p, const Args &a, int warps, cudaStream_t stream) {
     const size_t smem = encode_mma_smem(p, warps);
-    const cudaError_t e = allow_smem((const void *)encode_kernel<NKC, KPL, COSET, WIDE>, smem);
+    const cudaError_t e = allow_smem((const void *)encode_kernel<NKC, KPL, COSET, WIDE, STD>, smem);
     if (e != cudaSuccess) return e;
     const int64_t pairs = WIDE ? a.T : (a.T + 1) / 2;
     const int grid = (int)std::min<int64_t>((pairs + warps - 1) / warps, (int64_t)std::max(p->sms, 1));
-    encode_kernel<NKC, KPL, COSET, WIDE><<<grid, warps * 32, smem, stream>>>(a);
+    encode_kernel<NKC, KPL, COSET, WIDE, STD><<<grid, warps * 32, smem, stream>>>(a);
     return cudaGetLastError();
+}
+
+template <int NKC, int KPL, bool COSET, bool WIDE = false>
+cudaError_t launch_kpl(const dpb_plan *p, const Args &a, int warps, cudaStream_t stream) {
+    return a.mu ? launch_kpl_std<NKC, KPL, COSET, WIDE, true>(p, a, warps, stream)
+                : launch_kpl_std<NKC, KPL, COSET, WIDE, false>(p, a, warps, stream);
 }
 
 template <int NKC>
