@@ -159,6 +159,12 @@ __device__ __forceinline__ float x_at(const uint16_t *xh, int i) {
 __device__ __forceinline__ float standardise(float s, uint32_t c, const Args &a, int32_t *status) {
     return a.mu ? zscore(s, c, a.mu, a.sigma, a.tab, status) : s;
 }
+// The same, fixed at compile time (STD: tables are given).
+template <bool STD>
+__device__ __forceinline__ float stdz(float s, uint32_t c, const Args &a, int32_t *status) {
+    if constexpr (STD) return zscore(s, c, a.mu, a.sigma, a.tab, status);
+    return s;
+}
 
 // bf16 element e (0..7) of a 16-byte chunk.
 __device__ __forceinline__ uint32_t elem16(const uint4 &v, int e) {
@@ -618,10 +624,11 @@ __device__ __forceinline__ bool level0_union_std(const Args &a, const uint16_t *
 // candidate; a threshold that at least k of them reach keeps them in the
 // scratch (z, id) lists of capacity `cap`, the k-th is found by bisection, and
 // the first k, sorted, become the code list; its first 8 are the beam.
+template <bool STD>
 __device__ __forceinline__ void level0_bisect(const Args &a, const uint16_t *xh, float *pz, uint32_t *pid, int cap,
                                               uint64_t *L, uint32_t *beam) {
     const int lane = threadIdx.x & 31, d = a.d, k = a.k;
-    const int lowbit = a.mu ? 0 : 16;  // keys of unstandardised bf16 values have 16 zero bits
+    const int lowbit = STD ? 0 : 16;  // keys of unstandardised bf16 values have 16 zero bits
     // Each lane's R best keys, R = 2 ceil(k / 32) (at most 8): their union
     // holds at least k keys, and its k-th largest is a threshold that at least
     // k candidates reach and, unlike the smallest of the lanes' R-th keys,
@@ -631,7 +638,7 @@ __device__ __forceinline__ void level0_bisect(const Args &a, const uint16_t *xh,
 #pragma unroll
     for (int r = 0; r < 8; ++r) best[r] = 0u;
     for (int i = lane; i < d; i += 32) {
-        uint32_t kv = akey(standardise(x_at(xh, i), (uint32_t)i, a, a.status)) + 1u;
+        uint32_t kv = akey(stdz<STD>(x_at(xh, i), (uint32_t)i, a, a.status)) + 1u;
 #pragma unroll
         for (int r = 0; r < 8; ++r) {
             if (r < R && kv > best[r]) {
@@ -656,7 +663,7 @@ __device__ __forceinline__ void level0_bisect(const Args &a, const uint16_t *xh,
         float z = 0.f;
         bool take = false;
         if (i < d) {
-            z = standardise(x_at(xh, i), (uint32_t)i, a, nullptr);
+            z = stdz<STD>(x_at(xh, i), (uint32_t)i, a, nullptr);
             take = akey(z) + 1u >= tau_low;
         }
         if (n + __popc(__ballot_sync(kFull, take)) > cap) {
@@ -674,14 +681,14 @@ __device__ __forceinline__ void level0_bisect(const Args &a, const uint16_t *xh,
             const uint32_t c = tau | (1u << b);
             int cnt = 0;
             for (int i = lane; i < d; i += 32)
-                cnt += akey(standardise(x_at(xh, i), (uint32_t)i, a, nullptr)) >= c;
+                cnt += akey(stdz<STD>(x_at(xh, i), (uint32_t)i, a, nullptr)) >= c;
             if (__reduce_add_sync(kFull, cnt) >= k) tau = c;
         }
         n = 0;
         for (int i0 = 0; i0 < d; i0 += 32) {
             const int i = i0 + lane;
             float z = 0.f;
-            if (i < d) z = standardise(x_at(xh, i), (uint32_t)i, a, nullptr);
+            if (i < d) z = stdz<STD>(x_at(xh, i), (uint32_t)i, a, nullptr);
             n = warp_append(pz, pid, n, i < d && akey(z) > tau, z, (uint32_t)i);
         }
         for (int i0 = 0; i0 < d && n < k; i0 += 32) {
@@ -689,7 +696,7 @@ __device__ __forceinline__ void level0_bisect(const Args &a, const uint16_t *xh,
             float z = 0.f;
             bool tie = false;
             if (i < d) {
-                z = standardise(x_at(xh, i), (uint32_t)i, a, nullptr);
+                z = stdz<STD>(x_at(xh, i), (uint32_t)i, a, nullptr);
                 tie = akey(z) == tau;
             }
             const unsigned mb = __ballot_sync(kFull, tie);
@@ -804,7 +811,7 @@ __global__ void __launch_bounds__(kMaxWarps * 32, 1) encode_kernel(Args a) {
                     done = level0_union<(KPL <= 2 ? 4 : 8), KPL>(row, nch, k, E, a.ecap, Lt, bt);
             }
             if (!done)
-                level0_bisect(a, xh + tk * nblk * 32, reinterpret_cast<float *>(E),
+                level0_bisect<STD>(a, xh + tk * nblk * 32, reinterpret_cast<float *>(E),
                               reinterpret_cast<uint32_t *>(E) + a.ecap, a.ecap, Lt, bt);
             if constexpr (WIDE) {  // the beam: the first 16 of the sorted list (k >= beam)
                 if (lane < 16) beams[lane] = cword_idx(Lt[lane]);
