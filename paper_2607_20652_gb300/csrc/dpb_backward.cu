@@ -301,7 +301,9 @@ __device__ __forceinline__ void analyse(const BwdWarp &w, int nh, int d, const u
     }
 }
 
-template <typename Tio, int NKC, bool VEC>
+// KEPT: norm matching with the decode's r given (a separate instantiation,
+// without the path that rebuilds r).
+template <typename Tio, int NKC, bool VEC, bool KEPT>
 __global__ void __launch_bounds__(kBwdWarps * 32, 2) backward_lut_kernel(BackwardArgs a, int t) {
     extern __shared__ __align__(16) uint32_t smem_raw[];
     uint32_t *smem = aligned_smem<256>(smem_raw);
@@ -352,7 +354,7 @@ __global__ void __launch_bounds__(kBwdWarps * 32, 2) backward_lut_kernel(Backwar
         // With norm matching and the decode's r, dL/dr comes first, from one
         // sweep over x, grad_y and r; otherwise buf starts as the basis part
         // of r (rebuilt below) or as grad_y.
-        const bool kept_r = a.norm_match && a.R;
+        constexpr bool kept_r = KEPT;  // the launcher's choice: a.norm_match && a.R
         float nx, direct = 0.f;  // direct: coefficient of x / |x| in grad_x
         if (kept_r) {
             float sxx = 0.f, srr = 0.f, sgr = 0.f;
@@ -391,7 +393,7 @@ __global__ void __launch_bounds__(kBwdWarps * 32, 2) backward_lut_kernel(Backwar
                 w.cmap[e] = INT_MIN;
             }
             if (valid && !hashed) {
-                if (a.norm_match && !kept_r) atomicAdd(&w.buf[ci], v);
+                if (!kept_r && a.norm_match) atomicAdd(&w.buf[ci], v);
                 w.cmap[e] = -(ci + 1);
             }
             const unsigned m = __ballot_sync(kFull, hashed);
@@ -407,7 +409,7 @@ __global__ void __launch_bounds__(kBwdWarps * 32, 2) backward_lut_kernel(Backwar
         }
         __syncwarp();
         if (!kept_r) nx = sqrtf(warp_sum(RowOps<VEC>::sumsq(xr, d)));
-        if (!a.norm_match) {
+        if (!kept_r && !a.norm_match) {
             RowOps<VEC>::scale_in(w.buf, gr, d, 1.f);
             __syncwarp();
         }
@@ -415,7 +417,7 @@ __global__ void __launch_bounds__(kBwdWarps * 32, 2) backward_lut_kernel(Backwar
         // matching only) and turns it into dL/dr; pass 1 adds the hashed
         // entries' sum to grad_x.
 #pragma unroll 1
-        for (int pass = a.norm_match && !kept_r ? 0 : 1;; ++pass) {
+        for (int pass = !kept_r && a.norm_match ? 0 : 1;; ++pass) {
             if (pass == 1) {
                 // ---- grad_val = <phi_e, dL/dr> ----
                 analyse<NKC>(w, nh, d, vh2);
@@ -480,17 +482,17 @@ int grid_for(const dpb_plan *p, int64_t T, int warps) {
     return (int)std::min<int64_t>((T + warps - 1) / warps, (int64_t)std::max(p->sms, 1) * 16);
 }
 
-template <typename Tio, int NKC, bool VEC>
+template <typename Tio, int NKC, bool VEC, bool KEPT>
 cudaError_t run_backward_lut(const dpb_plan *p, const BackwardArgs &a, int64_t T, cudaStream_t stream) {
     const size_t per_block = 256 /* alignment */ + sizeof(uint32_t) * (size_t)bwd_block_words(p->cfg.d, NKC);
     const size_t per_warp = sizeof(uint32_t) * (size_t)bwd_warp_words(p->cfg.d, p->code_len, NKC);
-    const void *fn = (const void *)backward_lut_kernel<Tio, NKC, VEC>;
+    const void *fn = (const void *)backward_lut_kernel<Tio, NKC, VEC, KEPT>;
     const int warps = best_warps(fn, kBwdWarps, per_block, per_warp);
     if (warps <= 0) return cudaErrorInvalidConfiguration;
     const size_t smem = per_block + (size_t)warps * per_warp;
-    const cudaError_t e = allow_smem((const void *)backward_lut_kernel<Tio, NKC, VEC>, smem);
+    const cudaError_t e = allow_smem((const void *)backward_lut_kernel<Tio, NKC, VEC, KEPT>, smem);
     if (e != cudaSuccess) return e;
-    backward_lut_kernel<Tio, NKC, VEC><<<grid_for(p, T, warps), warps * 32, smem, stream>>>(a, p->t);
+    backward_lut_kernel<Tio, NKC, VEC, KEPT><<<grid_for(p, T, warps), warps * 32, smem, stream>>>(a, p->t);
     return cudaGetLastError();
 }
 
@@ -502,6 +504,12 @@ bool rows_vec(int d, std::initializer_list<const void *> ptrs) {
     for (const void *q : ptrs)
         if (reinterpret_cast<uintptr_t>(q) % (4 * sizeof(Tio)) != 0) return false;
     return true;
+}
+
+template <typename Tio, int NKC, bool VEC>
+cudaError_t run_backward_lut(const dpb_plan *p, const BackwardArgs &a, int64_t T, cudaStream_t stream) {
+    if (a.norm_match && a.R) return run_backward_lut<Tio, NKC, VEC, true>(p, a, T, stream);
+    return run_backward_lut<Tio, NKC, VEC, false>(p, a, T, stream);
 }
 
 template <typename Tio, int NKC>
