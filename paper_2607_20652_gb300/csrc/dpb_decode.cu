@@ -98,7 +98,8 @@ __host__ __device__ constexpr int decode_warp_words(int d, int k, int nkc) {
 
 constexpr int kDecWarps = 9;  // at most per block; four such blocks per SM at 56 registers
 
-template <typename Tio, int NKC, bool VEC>
+// KEPT: norm matching, and r kept for the backward (a separate instantiation).
+template <typename Tio, int NKC, bool VEC, bool KEPT>
 __global__ void __launch_bounds__(kDecWarps * 32, 4) decode_lut_kernel(DecodeArgs a, int t) {
     extern __shared__ __align__(16) uint32_t smem_raw[];
     uint32_t *smem = aligned_smem<128>(smem_raw);
@@ -118,9 +119,9 @@ __global__ void __launch_bounds__(kDecWarps * 32, 4) decode_lut_kernel(DecodeArg
         __syncwarp();
         const int nh = split_code(a.idx + tk * a.k, a.val + tk * a.k, a.k, d, a.m_mask, r, hl, a.status);
         synthesise<NKC>(sw, hl.c, hl.a, nh, t, d, koff, a.inv_sqrt_d, r);
-        if (a.R) RowOps<VEC>::store(a.R + tk * d, r, d, 1.f);
+        if (KEPT || a.R) RowOps<VEC>::store(a.R + tk * d, r, d, 1.f);
         float scale = 1.f;
-        if (a.norm_match) {
+        if (KEPT || a.norm_match) {
             float ss = 0.f, unused = 0.f;
             RowOps<VEC>::dots(r, r, d, ss, unused);
             const float nr = sqrtf(warp_sum(ss));
@@ -139,18 +140,24 @@ int grid_for(const dpb_plan *p, int64_t T, int warps) {
 
 namespace {
 
-template <typename Tio, int NKC, bool VEC>
+template <typename Tio, int NKC, bool VEC, bool KEPT>
 cudaError_t run_decode_lut(const dpb_plan *p, const DecodeArgs &a, int64_t T, cudaStream_t stream) {
     const size_t per_block = 128 /* alignment */ + sizeof(uint32_t) * (size_t)pad32(p->cfg.d);
     const size_t per_warp = sizeof(uint32_t) * (size_t)decode_warp_words(p->cfg.d, p->code_len, NKC);
-    const void *fn = (const void *)decode_lut_kernel<Tio, NKC, VEC>;
+    const void *fn = (const void *)decode_lut_kernel<Tio, NKC, VEC, KEPT>;
     const int warps = best_warps(fn, kDecWarps, per_block, per_warp);
     if (warps <= 0) return cudaErrorInvalidConfiguration;
     const size_t smem = per_block + (size_t)warps * per_warp;
     const cudaError_t e = allow_smem(fn, smem);
     if (e != cudaSuccess) return e;
-    decode_lut_kernel<Tio, NKC, VEC><<<grid_for(p, T, warps), warps * 32, smem, stream>>>(a, p->t);
+    decode_lut_kernel<Tio, NKC, VEC, KEPT><<<grid_for(p, T, warps), warps * 32, smem, stream>>>(a, p->t);
     return cudaGetLastError();
+}
+
+template <typename Tio, int NKC, bool VEC>
+cudaError_t run_decode_lut(const dpb_plan *p, const DecodeArgs &a, int64_t T, cudaStream_t stream) {
+    if (a.norm_match && a.R) return run_decode_lut<Tio, NKC, VEC, true>(p, a, T, stream);
+    return run_decode_lut<Tio, NKC, VEC, false>(p, a, T, stream);
 }
 
 template <typename Tio, int NKC>
