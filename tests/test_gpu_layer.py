@@ -86,7 +86,7 @@ def test_small_parity_transformer_trains(ema):
         for p in model.parameters():
             assert p.grad is None or torch.isfinite(p.grad).all()
         opt.step()
-        losses.append(float(loss))
+        losses.append(float(loss.detach()))
     assert np.isfinite(losses).all() and losses[-1] < losses[0] - 0.5, losses
     for layer in model.dpb_layers():
         assert dpb.workspace_status(layer._ws) == 0
