@@ -98,6 +98,28 @@ __host__ __device__ constexpr int decode_warp_words(int d, int k, int nkc) {
 
 constexpr int kDecWarps = 9;  // at most per block; four such blocks per SM at 56 registers
 
+// R[i] = r[i] (r kept for the backward) and this lane's share of |r|^2, in
+// one pass over r.
+template <bool VEC>
+__device__ __forceinline__ float keep_r(float *R, const float *r, int d) {
+    const int lane = threadIdx.x & 31;
+    float ss = 0.f;
+    if (VEC) {
+        for (int i = 4 * lane; i < d; i += 128) {
+            const float4 v = *reinterpret_cast<const float4 *>(r + i);
+            *reinterpret_cast<float4 *>(R + i) = v;
+            ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+        }
+    } else {
+        for (int i = lane; i < d; i += 32) {
+            const float v = r[i];
+            R[i] = v;
+            ss += v * v;
+        }
+    }
+    return ss;
+}
+
 // KEPT: norm matching, and r kept for the backward (a separate instantiation).
 template <typename Tio, int NKC, bool VEC, bool KEPT>
 __global__ void __launch_bounds__(kDecWarps * 32, 4) decode_lut_kernel(DecodeArgs a, int t) {
@@ -119,13 +141,18 @@ __global__ void __launch_bounds__(kDecWarps * 32, 4) decode_lut_kernel(DecodeArg
         __syncwarp();
         const int nh = split_code(a.idx + tk * a.k, a.val + tk * a.k, a.k, d, a.m_mask, r, hl, a.status);
         synthesise<NKC>(sw, hl.c, hl.a, nh, t, d, koff, a.inv_sqrt_d, r);
-        if (KEPT || a.R) RowOps<VEC>::store(a.R + tk * d, r, d, 1.f);
         float scale = 1.f;
-        if (KEPT || a.norm_match) {
-            float ss = 0.f, unused = 0.f;
-            RowOps<VEC>::dots(r, r, d, ss, unused);
-            const float nr = sqrtf(warp_sum(ss));
+        if (KEPT) {  // r kept and its norm in one pass
+            const float nr = sqrtf(warp_sum(keep_r<VEC>(a.R + tk * d, r, d)));
             scale = nr > 0.f ? a.xnorm[tk] / nr : 0.f;
+        } else {
+            if (a.R) RowOps<VEC>::store(a.R + tk * d, r, d, 1.f);
+            if (a.norm_match) {
+                float ss = 0.f, unused = 0.f;
+                RowOps<VEC>::dots(r, r, d, ss, unused);
+                const float nr = sqrtf(warp_sum(ss));
+                scale = nr > 0.f ? a.xnorm[tk] / nr : 0.f;
+            }
         }
         RowOps<VEC>::store(Y + tk * d, r, d, scale);
         __syncwarp();
