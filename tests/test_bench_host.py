@@ -78,3 +78,22 @@ def test_roofline_arithmetic():
     r = bench.roofline_for("copy", {"bytes": 6781.4e9 * 1e-3}, 2e-3, peaks, "measured", clocks={"sm_mhz": 900.0})
     assert r["bound"] == "hbm" and abs(r["frac"] - 0.5) < 1e-6 and r["unit"] == "GB/s"
     assert abs(r["frac_nominal"] - 6781.4 / 2 / 7900.0) < 1e-4  # and the nominal 7.9 TB/s beside it
+
+
+def test_measured_traffic_follows_the_kernel_sources(monkeypatch, tmp_path):
+    # figures are read for the size they were taken at, while the kernel's
+    # sources hash as recorded; any other size or a changed source gives None
+    f = tmp_path / "traffic.txt"
+    h = bench.kernel_source_hash("decode")
+    f.write_text("# comment line\n"
+                 f"decode 65536 271791872 {h}\n"
+                 "backward 65536 535708928 0000000000000000\n")
+    monkeypatch.setattr(bench, "TRAFFIC_FILE", str(f))
+    assert bench.measured_traffic("decode", 65536) == 271791872
+    assert bench.measured_traffic("decode", 32768) is None
+    assert bench.measured_traffic("backward", 65536) is None  # recorded for other sources
+    assert bench.measured_traffic("encode", 65536) is None    # not recorded
+    monkeypatch.setattr(bench, "kernel_source_hash", lambda name: "ffffffffffffffff")
+    assert bench.measured_traffic("decode", 65536) is None
+    monkeypatch.setattr(bench, "TRAFFIC_FILE", str(tmp_path / "absent.txt"))
+    assert bench.measured_traffic("decode", 65536) is None
